@@ -1,0 +1,239 @@
+/*
+ * soniq.h -- C ABI of the GB300 (sm_103a) SONIQ inference library.
+ *
+ * SONIQ (arXiv 2311.14114) quantizes every input channel of a layer to one of
+ * two precisions.  Inference needs (Sec. 3 "Enabling Low-Cost Fixed-Point
+ * Operations", Sec. 4.1 "Channel re-ordering and padding"):
+ *   - a channel permutation that makes each precision group contiguous along
+ *     the reduction axis K (Sec. 3 "Dynamic channel re-ordering"),
+ *   - one max-abs scale per group (step 1),
+ *   - unsigned activation codes (step 2) and two's-complement-fraction weight
+ *     codes, Eq. (1) (step 3),
+ *   - integer dot products inside each group, combined by the group scales.
+ *
+ * Conventions for every call:
+ *   * Device pointers are CUDA global-memory addresses owned by the caller;
+ *     the library never allocates, frees or retains them.
+ *   * Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *     default stream).  Argument errors are detected on the host before any
+ *     CUDA call and returned synchronously.  Launch failures return
+ *     SONIQ_ERR_CUDA.  Kernels never trap: a bounded device-side wait that
+ *     runs out records an error word, read back by soniq_sync_status().
+ *   * No C++ exception crosses this interface.
+ *   * Packed rows, codes and accumulators follow the layout described at
+ *     soniq_layout below; packed bytes and int32 accumulators are bit-exact
+ *     functions of the inputs.
+ */
+#ifndef SONIQ_H_
+#define SONIQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SONIQ_ABI_VERSION 1
+
+/* Exported symbols (the library is built with hidden default visibility). */
+#if defined(__GNUC__)
+#define SONIQ_API __attribute__((visibility("default")))
+#else
+#define SONIQ_API
+#endif
+
+typedef enum soniq_status {
+    SONIQ_OK = 0,
+    SONIQ_ERR_INVALID_ARG = 1,  /* null pointer, negative size, inconsistent layout */
+    SONIQ_ERR_UNSUPPORTED = 2,  /* well-formed but outside the kernels' limits */
+    SONIQ_ERR_ALIGNMENT = 3,    /* a pointer is not aligned as the call requires */
+    SONIQ_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
+    SONIQ_ERR_TIMEOUT = 5       /* a kernel's bounded wait ran out (see soniq_sync_status) */
+} soniq_status;
+
+/* A cudaStream_t, passed opaquely so this header needs no CUDA headers. */
+typedef void *soniq_stream_t;
+
+/*
+ * Per-layer precision layout (Sec. 3 "Dynamic channel re-ordering"; Fig. 2;
+ * Sec. 4.1).  Group 0 is the low precision, group 1 the high one.
+ *
+ *   K          logical input channels (for a convolution: C_in).
+ *   n_groups   1 or 2; with 1, count[1] must be 0.
+ *   count[g]   channels in group g, count[0] + count[1] == K.
+ *   bits_w[g]  weight bits of group g, 1..8 (Eq. (1), n).
+ *   bits_a[g]  activation bits of group g, 1..8 (Sec. 3 step 2, n).
+ *   perm       DEVICE pointer, K int32: perm[j] is the original channel stored
+ *              at packed position j.  Positions [0,count[0]) form group 0,
+ *              [count[0],K) group 1.  Must be a permutation of 0..K-1
+ *              (soniq_validate_layout checks a host copy).
+ *   pad_unit   32 or 128: each group of a packed activation row holds
+ *              PA_g = roundup(count[g], pad_unit) codes; pad codes are 0.
+ *
+ * Packed rows.  An activation row is [group 0: PA_0 codes][group 1: PA_1
+ * codes].  A weight row for `taps` filter taps is [group 0: PW_0][group 1:
+ * PW_1] with PW_g = roundup(taps * PA_g, 128), in tap-major order (position p
+ * holds tap p / PA_g, channel p % PA_g of the group; positions beyond
+ * taps * PA_g are 0).  Codes are stored in blocks of 32: a block of n-bit
+ * codes is n little-endian 32-bit words; the code bits are cut into slices of
+ * width 4, 2, 1 (low bits first; n = 8 is one 8-bit slice); a w-bit slice
+ * takes w words and code i (t = i/4, b = i%4) sits in slice word t/(8/w) at
+ * bit 8*b + w*(t % (8/w)).  Activation codes are unsigned, weight codes n-bit
+ * two's complement.  Row strides are soniq_packed_row_bytes().
+ */
+typedef struct soniq_layout {
+    int32_t K;
+    int32_t n_groups;
+    int32_t count[2];
+    int32_t bits_w[2];
+    int32_t bits_a[2];
+    const int32_t *perm;
+    int32_t pad_unit;
+} soniq_layout;
+
+/* Scale granularity (Sec. 3 step 1: one max-abs scale per group; C2: one
+ * scale per fused dot product).  Scale arrays are fp32 with 2 entries per
+ * scale (group 0, group 1). */
+enum {
+    SONIQ_SCALE_PER_TENSOR = 0,  /* one scale per (tensor, group): [2] ([N][2] replicated for weights) */
+    SONIQ_SCALE_PER_ROW = 1,     /* one scale per (row, group): [rows][2] */
+    SONIQ_SCALE_CALIBRATED = 2   /* activations only: caller supplies s_a[2]; inputs beyond it clip */
+};
+
+enum { SONIQ_OUT_F16 = 0, SONIQ_OUT_BF16 = 1 };
+
+enum {
+    SONIQ_FLAG_FORCE_GEMV = 1u,          /* soniq_mp_gemm: use the CUDA-core GEMV for any M <= 16 */
+    SONIQ_FLAG_FORCE_MMA = 2u,           /* soniq_mp_gemm: use the tensor-core kernel for any M */
+    SONIQ_FLAG_TEST_DROP_ARRIVE = 0x100u /* test hook: the tensor-core kernel's operand producer
+                                            skips its first arrival, so the consumer's bounded
+                                            wait runs out and the call reports SONIQ_ERR_TIMEOUT */
+};
+
+/* Convolution geometry.  Input NHWC [batch][H][W][C_in], output NHWC
+ * [batch][P][Q][C_out], P = (H + 2*pad_h - R)/stride_h + 1, Q likewise. */
+typedef struct soniq_conv_desc {
+    int32_t batch, H, W;
+    int32_t C_out;
+    int32_t R, S;
+    int32_t stride_h, stride_w;
+    int32_t pad_h, pad_w;
+} soniq_conv_desc;
+
+/* ---- sizes and checks (host only, no CUDA calls) ------------------------ */
+
+SONIQ_API int32_t soniq_abi_version(void);
+SONIQ_API const char *soniq_status_string(soniq_status status);
+
+/* Codes per row of group `group`: activation rows (is_weight = 0) or weight
+ * rows with `taps` taps (is_weight = 1).  -1 on a bad argument. */
+SONIQ_API int64_t soniq_group_codes(const soniq_layout *layout, int32_t group, int32_t is_weight,
+                          int32_t taps);
+
+/* Bytes per packed row (a multiple of 4; of 16 for weight rows).  -1 on a bad
+ * argument. */
+SONIQ_API int64_t soniq_packed_row_bytes(const soniq_layout *layout, int32_t is_weight, int32_t taps);
+
+/* Checks the layout fields; if perm_host is non-NULL also checks that it is a
+ * permutation of 0..K-1.  Does not read layout->perm. */
+SONIQ_API soniq_status soniq_validate_layout(const soniq_layout *layout, const int32_t *perm_host);
+
+/* Kernels this library has launched since load (all threads, all devices). */
+SONIQ_API int64_t soniq_launch_count(void);
+
+/* ---- the hot path ------------------------------------------------------- */
+
+/*
+ * Weight quantize-and-pack (offline, once per layer).  Sec. 3 steps 1 and 3,
+ * Eq. (1): per scale group s = max|w|, w' = w / s (fp32, IEEE), code
+ * j = clamp(round_half_even(w' * 2^(n-1)), -2^(n-1), 2^(n-1) - 1), the nearest
+ * level of Eq. (1); s = 0 gives j = 0.
+ *
+ *   W          device fp32 [N][taps][K] (taps = 1: a linear layer [N][K];
+ *              a convolution OHWI [C_out][R*S][C_in]), 4-byte aligned.
+ *   N          output rows (>= 0; 0 is a no-op).
+ *   taps       filter taps R*S (>= 1).
+ *   scale_mode SONIQ_SCALE_PER_ROW (one scale per (n, group) over all taps)
+ *              or SONIQ_SCALE_PER_TENSOR (one per group; written to every row).
+ *   Wp         device out [N][soniq_packed_row_bytes(layout, 1, taps)], 16-byte aligned.
+ *   s_w        device out fp32 [N][2].
+ */
+SONIQ_API soniq_status soniq_pack_weights(const soniq_layout *layout, const float *W, int32_t N,
+                                int32_t taps, int32_t scale_mode, uint8_t *Wp, float *s_w,
+                                soniq_stream_t stream);
+
+/*
+ * Activation quantize-and-pack (per inference call).  Sec. 3 steps 1 and 2:
+ * s = max|a| per scale group, code u = clip(round_half_even(fp32(a / s) *
+ * (2^n - 1)), 0, 2^n - 1); s = 0 gives u = 0.  Channels are gathered through
+ * layout->perm and each group is zero-padded to PA_g codes.
+ *
+ *   A          device fp16 [M][K] (IEEE binary16 bits), 2-byte aligned.
+ *   M          rows (tokens, or pixels of an NHWC image); 0 is a no-op.
+ *   scale_mode SONIQ_SCALE_PER_TENSOR: s_a is an output [2];
+ *              SONIQ_SCALE_PER_ROW:    s_a is an output [M][2];
+ *              SONIQ_SCALE_CALIBRATED: s_a is an input [2].
+ *   s_a        device fp32, see scale_mode.
+ *   Ap         device out [M][soniq_packed_row_bytes(layout, 0, 1)], 4-byte aligned.
+ */
+SONIQ_API soniq_status soniq_quantize_act(const soniq_layout *layout, const void *A, int64_t M,
+                                int32_t scale_mode, float *s_a, uint8_t *Ap,
+                                soniq_stream_t stream);
+
+/*
+ * Mixed-precision quantized GEMM Y = A W^T.  Sec. 3 (integer MAC per fused
+ * dot product, decode rules of steps 2-3) and Sec. 4.2 (unsigned x signed
+ * integer dot products):
+ *   Acc_g[m][n] = sum over k in group g of u[m][k] * j[n][k]   (exact int32)
+ *   Y[m][n]     = sum_g s_a(m,g) * s_w[n][g] / ((2^na_g - 1) * 2^(nw_g - 1)) * Acc_g[m][n]
+ * computed in fp32 and rounded to nearest fp16 (or bf16).  M <= 16 runs a
+ * bandwidth-bound CUDA-core GEMV, larger M the tcgen05 tensor-core kernel
+ * (flags can force either).
+ *
+ *   Ap, s_a    from soniq_quantize_act with the same layout (pad_unit 32 or 128);
+ *              s_a [2] (PER_TENSOR / CALIBRATED) or [M][2] (PER_ROW).
+ *   Wp, s_w    from soniq_pack_weights with the same layout and taps = 1.
+ *   Y          device out [M][N], fp16 or bf16 per out_dtype, 16-byte aligned.
+ *   acc_dbg    NULL, or device out int32 [2][M][N]: the exact Acc_g.
+ *   Limits (SONIQ_ERR_UNSUPPORTED otherwise): K <= 65536.  The tensor-core
+ *   kernel accumulates integer codes in fp32, exact while every partial sum
+ *   stays within 2^24; a group whose worst-case sum over its K range could
+ *   exceed that is accumulated in bounded segments that are drained to int32,
+ *   and at most one of the two groups may need segments.
+ */
+SONIQ_API soniq_status soniq_mp_gemm(const soniq_layout *layout, const uint8_t *Ap, const float *s_a,
+                           int32_t scale_mode, int64_t M, const uint8_t *Wp, const float *s_w,
+                           int32_t N, void *Y, int32_t out_dtype, int32_t *acc_dbg,
+                           uint32_t flags, soniq_stream_t stream);
+
+/*
+ * Mixed-precision quantized convolution as implicit GEMM (Sec. 4.1: the CPU
+ * and GPU back-ends run convolutions on the re-ordered, padded channel
+ * blocks; Sec. 6 evaluates conv layers).  K = R*S*C_in in the weight order
+ * (group, tap, channel); input positions outside the image contribute 0.
+ *
+ *   cd         geometry; P, Q > 0.
+ *   Xp, s_a    soniq_quantize_act of the NHWC input viewed as [batch*H*W][C_in],
+ *              with a per-tensor or calibrated scale (a per-pixel scale would
+ *              break the shared scale of one dot product, C2).
+ *   Wp, s_w    soniq_pack_weights of OHWI weights with taps = R*S.
+ *   Y          device out NHWC [batch][P][Q][C_out], 16-byte aligned.
+ *   acc_dbg    NULL or device out int32 [2][batch*P*Q][C_out].
+ */
+SONIQ_API soniq_status soniq_mp_conv2d(const soniq_layout *layout, const soniq_conv_desc *cd,
+                             const uint8_t *Xp, const float *s_a, int32_t scale_mode,
+                             const uint8_t *Wp, const float *s_w, void *Y, int32_t out_dtype,
+                             int32_t *acc_dbg, uint32_t flags, soniq_stream_t stream);
+
+/* Waits for `stream`, then returns SONIQ_ERR_TIMEOUT if any kernel of this
+ * library on the current device recorded a timed-out wait since the last
+ * call (and clears that record), SONIQ_ERR_CUDA on a CUDA error, else
+ * SONIQ_OK. */
+SONIQ_API soniq_status soniq_sync_status(soniq_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SONIQ_H_ */

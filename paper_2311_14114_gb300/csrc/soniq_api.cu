@@ -1,0 +1,309 @@
+// C-ABI entry points of the SONIQ library: argument validation (host only,
+// before any CUDA call), layout geometry, dispatch to the kernels and the
+// device-side error word that bounded waits report into.
+#include <atomic>
+#include <cstring>
+#include <vector>
+
+#include "soniq_internal.h"
+
+namespace soniq {
+
+namespace {
+
+// One word per device: kernels atomically OR error bits into it when a
+// bounded wait runs out; soniq_sync_status reads and clears it.
+__device__ unsigned g_error_word;
+
+std::atomic<int64_t> g_launches{0};
+
+constexpr int kMaxDevices = 64;
+unsigned* g_err_addr[kMaxDevices] = {};
+int g_sms[kMaxDevices] = {};
+
+int64_t roundup(int64_t x, int64_t u) { return (x + u - 1) / u * u; }
+
+bool aligned(const void* p, uintptr_t a) { return ((uintptr_t)p % a) == 0; }
+
+int current_device() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return -1;
+    return dev;
+}
+
+soniq_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return SONIQ_OK;
+    if (e == cudaErrorNotSupported) return SONIQ_ERR_UNSUPPORTED;
+    return SONIQ_ERR_CUDA;
+}
+
+}  // namespace
+
+unsigned* device_error_word() {
+    const int dev = current_device();
+    if (dev < 0) return nullptr;
+    if (g_err_addr[dev] == nullptr) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+        g_err_addr[dev] = static_cast<unsigned*>(p);
+    }
+    return g_err_addr[dev];
+}
+
+void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+int num_sms() {
+    const int dev = current_device();
+    if (dev < 0) return 148;
+    if (g_sms[dev] == 0) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+        g_sms[dev] = v > 0 ? v : 148;
+    }
+    return g_sms[dev];
+}
+
+soniq_status make_geom(const soniq_layout* L, int32_t taps, LayoutGeom* geo) {
+    if (L == nullptr || geo == nullptr) return SONIQ_ERR_INVALID_ARG;
+    if (L->K < 1 || L->K > 65536) return L->K < 1 ? SONIQ_ERR_INVALID_ARG : SONIQ_ERR_UNSUPPORTED;
+    if (L->n_groups != 1 && L->n_groups != 2) return SONIQ_ERR_INVALID_ARG;
+    if (L->pad_unit != 32 && L->pad_unit != 128) return SONIQ_ERR_INVALID_ARG;
+    if (taps < 1 || taps > 4096) return SONIQ_ERR_INVALID_ARG;
+    if (L->count[0] < 0 || L->count[1] < 0 || (int64_t)L->count[0] + L->count[1] != L->K)
+        return SONIQ_ERR_INVALID_ARG;
+    if (L->n_groups == 1 && L->count[1] != 0) return SONIQ_ERR_INVALID_ARG;
+    geo->K = L->K;
+    geo->taps = taps;
+    int64_t a_off = 0, w_off = 0;
+    for (int g = 0; g < 2; ++g) {
+        GroupGeom& G = geo->g[g];
+        const bool used = g < L->n_groups;
+        const int bw = used ? L->bits_w[g] : 1;
+        const int ba = used ? L->bits_a[g] : 1;
+        if (bw < 1 || bw > 8 || ba < 1 || ba > 8) return SONIQ_ERR_INVALID_ARG;
+        G.count = used ? L->count[g] : 0;
+        G.bits_a = ba;
+        G.bits_w = bw;
+        G.pa = (int32_t)roundup(G.count, L->pad_unit);
+        G.pw = (int32_t)roundup((int64_t)taps * G.pa, 128);
+        G.a_off = (int32_t)a_off;
+        G.w_off = (int32_t)w_off;
+        G.perm_base = g == 0 ? 0 : L->count[0];
+        a_off += (int64_t)G.pa / 32 * 4 * ba;
+        w_off += (int64_t)G.pw / 32 * 4 * bw;
+    }
+    if (a_off > (1 << 30) || w_off > (1 << 30)) return SONIQ_ERR_UNSUPPORTED;
+    geo->a_row_bytes = (int32_t)a_off;
+    geo->w_row_bytes = (int32_t)w_off;
+    return SONIQ_OK;
+}
+
+}  // namespace soniq
+
+using namespace soniq;
+
+namespace {
+
+cudaStream_t as_stream(soniq_stream_t s) { return reinterpret_cast<cudaStream_t>(s); }
+
+soniq_status check_scale_mode_act(int32_t mode) {
+    return (mode == SONIQ_SCALE_PER_TENSOR || mode == SONIQ_SCALE_PER_ROW || mode == SONIQ_SCALE_CALIBRATED)
+               ? SONIQ_OK
+               : SONIQ_ERR_INVALID_ARG;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t soniq_abi_version(void) { return SONIQ_ABI_VERSION; }
+
+const char* soniq_status_string(soniq_status s) {
+    switch (s) {
+        case SONIQ_OK: return "ok";
+        case SONIQ_ERR_INVALID_ARG: return "invalid argument";
+        case SONIQ_ERR_UNSUPPORTED: return "unsupported configuration";
+        case SONIQ_ERR_ALIGNMENT: return "misaligned pointer";
+        case SONIQ_ERR_CUDA: return "CUDA error";
+        case SONIQ_ERR_TIMEOUT: return "device wait timed out";
+    }
+    return "unknown status";
+}
+
+int64_t soniq_group_codes(const soniq_layout* L, int32_t group, int32_t is_weight, int32_t taps) {
+    LayoutGeom geo;
+    if (group < 0 || group > 1) return -1;
+    if (make_geom(L, is_weight ? taps : 1, &geo) != SONIQ_OK) return -1;
+    return is_weight ? geo.g[group].pw : geo.g[group].pa;
+}
+
+int64_t soniq_packed_row_bytes(const soniq_layout* L, int32_t is_weight, int32_t taps) {
+    LayoutGeom geo;
+    if (make_geom(L, is_weight ? taps : 1, &geo) != SONIQ_OK) return -1;
+    return is_weight ? geo.w_row_bytes : geo.a_row_bytes;
+}
+
+soniq_status soniq_validate_layout(const soniq_layout* L, const int32_t* perm_host) {
+    LayoutGeom geo;
+    soniq_status st = make_geom(L, 1, &geo);
+    if (st != SONIQ_OK) return st;
+    if (perm_host != nullptr) {
+        std::vector<unsigned char> seen((size_t)L->K, 0);
+        for (int32_t j = 0; j < L->K; ++j) {
+            const int32_t c = perm_host[j];
+            if (c < 0 || c >= L->K || seen[(size_t)c]) return SONIQ_ERR_INVALID_ARG;
+            seen[(size_t)c] = 1;
+        }
+    }
+    return SONIQ_OK;
+}
+
+int64_t soniq_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+soniq_status soniq_pack_weights(const soniq_layout* L, const float* W, int32_t N, int32_t taps,
+                                int32_t scale_mode, uint8_t* Wp, float* s_w, soniq_stream_t stream) {
+    LayoutGeom geo;
+    soniq_status st = make_geom(L, taps, &geo);
+    if (st != SONIQ_OK) return st;
+    if (N < 0) return SONIQ_ERR_INVALID_ARG;
+    if (scale_mode != SONIQ_SCALE_PER_ROW && scale_mode != SONIQ_SCALE_PER_TENSOR) return SONIQ_ERR_INVALID_ARG;
+    if (N == 0) return SONIQ_OK;
+    if (W == nullptr || Wp == nullptr || s_w == nullptr || L->perm == nullptr) return SONIQ_ERR_INVALID_ARG;
+    if (!aligned(W, 4) || !aligned(Wp, 16) || !aligned(s_w, 4)) return SONIQ_ERR_ALIGNMENT;
+    cudaStream_t s = as_stream(stream);
+    if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
+        cudaError_t e = launch_weight_absmax(geo, L->perm, W, N, s_w, s);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    return cuda_status(launch_pack_weights(geo, L->perm, W, N, scale_mode == SONIQ_SCALE_PER_ROW, Wp, s_w, s));
+}
+
+soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M, int32_t scale_mode,
+                                float* s_a, uint8_t* Ap, soniq_stream_t stream) {
+    LayoutGeom geo;
+    soniq_status st = make_geom(L, 1, &geo);
+    if (st != SONIQ_OK) return st;
+    if (L->K > 32768) return SONIQ_ERR_UNSUPPORTED;
+    if (M < 0) return SONIQ_ERR_INVALID_ARG;
+    if ((st = check_scale_mode_act(scale_mode)) != SONIQ_OK) return st;
+    if (M == 0) return SONIQ_OK;
+    if (A == nullptr || s_a == nullptr || Ap == nullptr || L->perm == nullptr) return SONIQ_ERR_INVALID_ARG;
+    if (!aligned(A, 2) || !aligned(Ap, 4) || !aligned(s_a, 4)) return SONIQ_ERR_ALIGNMENT;
+    cudaStream_t s = as_stream(stream);
+    const uint16_t* A16 = static_cast<const uint16_t*>(A);
+    if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
+        cudaError_t e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    return cuda_status(launch_quantize_act(geo, L->perm, A16, M, scale_mode, s_a, Ap, s));
+}
+
+soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float* s_a, int32_t scale_mode,
+                           int64_t M, const uint8_t* Wp, const float* s_w, int32_t N, void* Y,
+                           int32_t out_dtype, int32_t* acc_dbg, uint32_t flags, soniq_stream_t stream) {
+    LayoutGeom geo;
+    soniq_status st = make_geom(L, 1, &geo);
+    if (st != SONIQ_OK) return st;
+    if (M < 0 || N < 0) return SONIQ_ERR_INVALID_ARG;
+    if ((st = check_scale_mode_act(scale_mode)) != SONIQ_OK) return st;
+    if (out_dtype != SONIQ_OUT_F16 && out_dtype != SONIQ_OUT_BF16) return SONIQ_ERR_INVALID_ARG;
+    if ((flags & SONIQ_FLAG_FORCE_GEMV) && (flags & SONIQ_FLAG_FORCE_MMA)) return SONIQ_ERR_INVALID_ARG;
+    if (M == 0 || N == 0) return SONIQ_OK;
+    if (Ap == nullptr || s_a == nullptr || Wp == nullptr || s_w == nullptr || Y == nullptr)
+        return SONIQ_ERR_INVALID_ARG;
+    if (!aligned(Ap, 4) || !aligned(Wp, 16) || !aligned(Y, 16) || !aligned(s_a, 4) || !aligned(s_w, 4) ||
+        (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
+        return SONIQ_ERR_ALIGNMENT;
+    // K <= 65536 keeps |Acc| < 2^31 and the GEMV's unsigned offset sums below 2^32
+    const int per_row = scale_mode == SONIQ_SCALE_PER_ROW;
+    cudaStream_t s = as_stream(stream);
+    const bool want_gemv = (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= 16 && !(flags & SONIQ_FLAG_FORCE_MMA));
+    if (want_gemv && gemv_supported(geo, M)) {
+        GemvArgs a{Ap, Wp, s_a, s_w, Y, acc_dbg, (int32_t)M, N, per_row, out_dtype == SONIQ_OUT_BF16};
+        return cuda_status(launch_gemv(geo, a, s));
+    }
+    if (flags & SONIQ_FLAG_FORCE_GEMV) return SONIQ_ERR_UNSUPPORTED;
+    if ((st = mma_check(geo)) != SONIQ_OK) return st;
+    MmaArgs a{};
+    a.Ap = Ap;
+    a.Wp = Wp;
+    a.s_a = s_a;
+    a.s_w = s_w;
+    a.Y = Y;
+    a.acc_dbg = acc_dbg;
+    a.M = M;
+    a.N = N;
+    a.s_a_per_row = per_row;
+    a.out_bf16 = out_dtype == SONIQ_OUT_BF16;
+    a.flags = flags;
+    a.conv = 0;
+    return cuda_status(launch_mma(geo, a, s));
+}
+
+soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, const uint8_t* Xp,
+                             const float* s_a, int32_t scale_mode, const uint8_t* Wp, const float* s_w,
+                             void* Y, int32_t out_dtype, int32_t* acc_dbg, uint32_t flags,
+                             soniq_stream_t stream) {
+    if (cd == nullptr) return SONIQ_ERR_INVALID_ARG;
+    if (cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->pad_h < 0 || cd->pad_w < 0 ||
+        cd->batch < 0 || cd->H < 1 || cd->W < 1 || cd->C_out < 0)
+        return SONIQ_ERR_INVALID_ARG;
+    LayoutGeom geo;
+    soniq_status st = make_geom(L, cd->R * cd->S, &geo);
+    if (st != SONIQ_OK) return st;
+    if (scale_mode != SONIQ_SCALE_PER_TENSOR && scale_mode != SONIQ_SCALE_CALIBRATED) return SONIQ_ERR_INVALID_ARG;
+    if (out_dtype != SONIQ_OUT_F16 && out_dtype != SONIQ_OUT_BF16) return SONIQ_ERR_INVALID_ARG;
+    const int32_t P = (cd->H + 2 * cd->pad_h - cd->R) / cd->stride_h + 1;
+    const int32_t Q = (cd->W + 2 * cd->pad_w - cd->S) / cd->stride_w + 1;
+    if (cd->H + 2 * cd->pad_h < cd->R || cd->W + 2 * cd->pad_w < cd->S || P < 1 || Q < 1)
+        return SONIQ_ERR_INVALID_ARG;
+    const int64_t M = (int64_t)cd->batch * P * Q;
+    if (M == 0 || cd->C_out == 0) return SONIQ_OK;
+    if (Xp == nullptr || s_a == nullptr || Wp == nullptr || s_w == nullptr || Y == nullptr)
+        return SONIQ_ERR_INVALID_ARG;
+    if (!aligned(Xp, 4) || !aligned(Wp, 16) || !aligned(Y, 16) || !aligned(s_a, 4) || !aligned(s_w, 4) ||
+        (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
+        return SONIQ_ERR_ALIGNMENT;
+    if ((st = mma_check(geo)) != SONIQ_OK) return st;
+    MmaArgs a{};
+    a.Ap = Xp;
+    a.Wp = Wp;
+    a.s_a = s_a;
+    a.s_w = s_w;
+    a.Y = Y;
+    a.acc_dbg = acc_dbg;
+    a.M = M;
+    a.N = cd->C_out;
+    a.s_a_per_row = 0;
+    a.out_bf16 = out_dtype == SONIQ_OUT_BF16;
+    a.flags = flags;
+    a.conv = 1;
+    a.H = cd->H;
+    a.W = cd->W;
+    a.P = P;
+    a.Q = Q;
+    a.R = cd->R;
+    a.S = cd->S;
+    a.sh = cd->stride_h;
+    a.sw = cd->stride_w;
+    a.ph = cd->pad_h;
+    a.pw = cd->pad_w;
+    return cuda_status(launch_mma(geo, a, as_stream(stream)));
+}
+
+soniq_status soniq_sync_status(soniq_stream_t stream) {
+    cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+    if (e != cudaSuccess) return SONIQ_ERR_CUDA;
+    unsigned* addr = device_error_word();
+    if (addr == nullptr) return SONIQ_ERR_CUDA;
+    unsigned v = 0;
+    if (cudaMemcpy(&v, addr, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return SONIQ_ERR_CUDA;
+    if (v != 0) {
+        const unsigned zero = 0;
+        if (cudaMemcpy(addr, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return SONIQ_ERR_CUDA;
+        return SONIQ_ERR_TIMEOUT;
+    }
+    return SONIQ_OK;
+}
+
+}  // extern "C"

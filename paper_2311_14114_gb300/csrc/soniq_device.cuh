@@ -1,0 +1,129 @@
+// Device helpers shared by the SONIQ kernels: the quantizers (Sec. 3 steps
+// 2 and 3, Eq. (1)), packing of a 32-code block by one warp, and the
+// SIMD-in-register expansion of a packed block back to bytes.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+namespace soniq {
+
+// ---- quantizers ------------------------------------------------------------
+// Both decide the integer code in fp32 with the operation order of the
+// paper's formulas: divide by the group scale (IEEE, round to nearest), then
+// multiply by the level count, round half to even, clip.  A zero scale (an
+// all-zero group) gives code 0.
+
+// Activation (Sec. 3 step 2): u = clip(round(a / s * (2^n - 1)), 0, 2^n - 1).
+__device__ __forceinline__ uint32_t act_code(float a, float s, float levels) {
+    if (!(s > 0.0f)) return 0u;
+    float t = __fmul_rn(__fdiv_rn(a, s), levels);
+    float r = rintf(t);
+    r = fminf(fmaxf(r, 0.0f), levels);
+    return (uint32_t)r;
+}
+
+// Weight (Sec. 3 step 3, Eq. (1)): nearest level j / 2^(n-1) to w / s,
+// j in [-2^(n-1), 2^(n-1) - 1]; `half` = 2^(n-1).
+__device__ __forceinline__ int32_t weight_code(float w, float s, float half) {
+    if (!(s > 0.0f)) return 0;
+    float t = __fmul_rn(__fdiv_rn(w, s), half);
+    float r = rintf(t);
+    r = fminf(fmaxf(r, -half), half - 1.0f);
+    return (int32_t)r;
+}
+
+// ---- packed block layout ---------------------------------------------------
+// 32 codes of n bits -> n words.  Code bits are cut into slices of width 4,
+// 2, 1 (low bits first; n = 8 is one slice).  In a w-bit slice, code i
+// (t = i/4, b = i%4) sits in slice word t/(8/w) at bit 8*b + w*(t%(8/w)), so
+// shifting slice word q right by w*s and masking the low w bits of each byte
+// yields codes 4*(q*(8/w)+s) .. +3 in byte order.
+
+// One warp packs one block: lane i holds code pattern i; the return value of
+// lane q (q < n) is word q of the block.
+__device__ __forceinline__ uint32_t pack_block_warp(uint32_t code, int n) {
+    const int lane = threadIdx.x & 31;
+    const int t = lane >> 2, b = lane & 3;
+    uint32_t mine = 0u;
+    int word = 0, off = 0;
+    const int widths[3] = {n == 8 ? 8 : (n & 4), n == 8 ? 0 : (n & 2), n == 8 ? 0 : (n & 1)};
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+        const int w = widths[k];
+        if (w == 0) continue;
+        const int per = 8 / w;
+        const uint32_t v = (code >> off) & ((1u << w) - 1u);
+        const int my_q = t / per;
+        const uint32_t shifted = v << (8 * b + w * (t % per));
+        for (int q = 0; q < w; ++q) {
+            uint32_t r = __reduce_or_sync(0xffffffffu, my_q == q ? shifted : 0u);
+            if (lane == word + q) mine = r;
+        }
+        word += w;
+        off += w;
+    }
+    return mine;
+}
+
+// Expands one packed block (N words at w) to 8 words of bytes: byte b of
+// o[t] is the N-bit pattern of code 4*t + b.
+template <int N>
+__device__ __forceinline__ void block_to_bytes(const uint32_t* w, uint32_t* o) {
+    if constexpr (N == 8) {
+#pragma unroll
+        for (int t = 0; t < 8; ++t) o[t] = w[t];
+    } else {
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            uint32_t v = 0u;
+            int word = 0, off = 0;
+            if constexpr ((N & 4) != 0) {
+                v |= (w[word + t / 2] >> (4 * (t % 2))) & 0x0F0F0F0Fu;
+                word += 4;
+                off += 4;
+            }
+            if constexpr ((N & 2) != 0) {
+                v |= ((w[word + t / 4] >> (2 * (t % 4))) & 0x03030303u) << off;
+                word += 2;
+                off += 2;
+            }
+            if constexpr ((N & 1) != 0) {
+                v |= ((w[word] >> t) & 0x01010101u) << off;
+            }
+            o[t] = v;
+        }
+    }
+}
+
+// Byte-wise sign-bit flip: n-bit two's complement j -> offset binary j + 2^(n-1).
+__device__ __forceinline__ uint32_t sign_flip_mask(int n) { return 0x01010101u << (n - 1); }
+
+// Runtime-n dispatch of block_to_bytes.
+__device__ __forceinline__ void block_to_bytes_n(int n, const uint32_t* w, uint32_t* o) {
+    switch (n) {
+        case 1: block_to_bytes<1>(w, o); break;
+        case 2: block_to_bytes<2>(w, o); break;
+        case 3: block_to_bytes<3>(w, o); break;
+        case 4: block_to_bytes<4>(w, o); break;
+        case 5: block_to_bytes<5>(w, o); break;
+        case 6: block_to_bytes<6>(w, o); break;
+        case 7: block_to_bytes<7>(w, o); break;
+        default: block_to_bytes<8>(w, o); break;
+    }
+}
+
+// Four bytes -> two fp16x2 words holding 1024 + byte (the exponent field of
+// 1024.0 is placed above each byte; Kim et al. 2022 "magic number" conversion).
+__device__ __forceinline__ void bytes_to_magic_half2(uint32_t x, uint32_t& lo, uint32_t& hi) {
+    lo = __byte_perm(x, 0x64646464u, 0x5150);
+    hi = __byte_perm(x, 0x64646464u, 0x5352);
+}
+
+__device__ __forceinline__ uint32_t half2_sub(uint32_t a, __half2 b) {
+    __half2 h = *reinterpret_cast<__half2*>(&a);
+    h = __hsub2(h, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+}  // namespace soniq

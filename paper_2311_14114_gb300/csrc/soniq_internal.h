@@ -1,0 +1,91 @@
+// Internal declarations shared by the SONIQ CUDA translation units.
+// Host code (validation, dispatch) and kernels see the same geometry structs.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "soniq.h"
+
+namespace soniq {
+
+// One precision group as the kernels see it (Sec. 3 "Dynamic channel
+// re-ordering": each group is a contiguous run of packed channels).
+struct GroupGeom {
+    int32_t count;      // logical channels
+    int32_t bits_a;     // activation bits
+    int32_t bits_w;     // weight bits
+    int32_t pa;         // activation codes per row (per pixel for conv): roundup(count, pad)
+    int32_t pw;         // weight codes per row: roundup(taps * pa, 128)
+    int32_t a_off;      // byte offset of the group in a packed activation row
+    int32_t w_off;      // byte offset of the group in a packed weight row
+    int32_t perm_base;  // first packed position of the group
+};
+
+struct LayoutGeom {
+    int32_t K;
+    int32_t taps;
+    int32_t a_row_bytes;
+    int32_t w_row_bytes;
+    GroupGeom g[2];
+};
+
+// Fills `geo` from a layout; returns SONIQ_OK or the validation error.
+soniq_status make_geom(const soniq_layout* L, int32_t taps, LayoutGeom* geo);
+
+// Device address of the library's error word on the current device (0 on failure).
+unsigned* device_error_word();
+void note_launch(int n = 1);
+int num_sms();
+
+// ---- launchers (return the CUDA error of the launch) ----------------------
+
+cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
+                              int64_t M, float* s_out, cudaStream_t st);
+cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
+                                int64_t M, int32_t scale_mode, float* s_a, uint8_t* Ap,
+                                cudaStream_t st);
+cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, const float* W,
+                                 int32_t N, float* s_out, cudaStream_t st);
+cudaError_t launch_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W,
+                                int32_t N, int32_t per_row, uint8_t* Wp, float* s_w,
+                                cudaStream_t st);
+
+struct GemvArgs {
+    const uint8_t* Ap;
+    const uint8_t* Wp;
+    const float* s_a;
+    const float* s_w;
+    void* Y;
+    int32_t* acc_dbg;
+    int32_t M;
+    int32_t N;
+    int32_t s_a_per_row;
+    int32_t out_bf16;
+};
+// Returns cudaErrorNotSupported if the shape does not fit the GEMV kernel.
+cudaError_t launch_gemv(const LayoutGeom& geo, const GemvArgs& a, cudaStream_t st);
+bool gemv_supported(const LayoutGeom& geo, int64_t M);
+
+struct MmaArgs {
+    const uint8_t* Ap;
+    const uint8_t* Wp;
+    const float* s_a;
+    const float* s_w;
+    void* Y;
+    int32_t* acc_dbg;
+    int64_t M;        // output rows (conv: batch * P * Q)
+    int32_t N;        // output columns (conv: C_out)
+    int32_t s_a_per_row;
+    int32_t out_bf16;
+    uint32_t flags;
+    // convolution geometry; conv = 0 for a plain GEMM
+    int32_t conv;
+    int32_t H, W, P, Q, R, S, sh, sw, ph, pw;
+};
+// Host-side planning of the tensor-core kernel (exactness segments etc.).
+soniq_status mma_check(const LayoutGeom& geo);
+cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st);
+
+}  // namespace soniq

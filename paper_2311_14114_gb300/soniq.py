@@ -1,0 +1,229 @@
+"""ctypes binding of libsoniq.so (``include/soniq.h``).
+
+Argument marshalling only: torch supplies device memory and the current CUDA
+stream; every step of the quantize / pack / GEMM / conv path runs in the
+library's CUDA kernels.  There is no fallback: if the library is missing or
+no GPU is present the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence, Tuple
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libsoniq.so")
+
+SONIQ_OK = 0
+STATUS_NAMES = {0: "SONIQ_OK", 1: "SONIQ_ERR_INVALID_ARG", 2: "SONIQ_ERR_UNSUPPORTED",
+                3: "SONIQ_ERR_ALIGNMENT", 4: "SONIQ_ERR_CUDA", 5: "SONIQ_ERR_TIMEOUT"}
+SCALE_PER_TENSOR, SCALE_PER_ROW, SCALE_CALIBRATED = 0, 1, 2
+OUT_F16, OUT_BF16 = 0, 1
+FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_TEST_DROP_ARRIVE = 1, 2, 0x100
+
+EXPORTED = ["soniq_abi_version", "soniq_status_string", "soniq_group_codes",
+            "soniq_packed_row_bytes", "soniq_validate_layout", "soniq_launch_count",
+            "soniq_pack_weights", "soniq_quantize_act", "soniq_mp_gemm", "soniq_mp_conv2d",
+            "soniq_sync_status"]
+
+_SCALE = {"tensor": SCALE_PER_TENSOR, "row": SCALE_PER_ROW, "calibrated": SCALE_CALIBRATED}
+
+
+class SoniqError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}")
+
+
+class CLayout(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int32), ("n_groups", ctypes.c_int32),
+                ("count", ctypes.c_int32 * 2), ("bits_w", ctypes.c_int32 * 2),
+                ("bits_a", ctypes.c_int32 * 2), ("perm", ctypes.c_void_p),
+                ("pad_unit", ctypes.c_int32)]
+
+
+class CConvDesc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("H", ctypes.c_int32), ("W", ctypes.c_int32),
+                ("C_out", ctypes.c_int32), ("R", ctypes.c_int32), ("S", ctypes.c_int32),
+                ("stride_h", ctypes.c_int32), ("stride_w", ctypes.c_int32),
+                ("pad_h", ctypes.c_int32), ("pad_w", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Loads libsoniq.so (built by ``paper_2311_14114_gb300.build``)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libsoniq.so not built ({LIB_PATH}); run __graft_entry__.build()")
+        L = ctypes.CDLL(LIB_PATH)
+        P, i32, i64, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+        L.soniq_abi_version.restype = i32
+        L.soniq_status_string.argtypes = [i32]
+        L.soniq_status_string.restype = ctypes.c_char_p
+        L.soniq_group_codes.argtypes = [P, i32, i32, i32]
+        L.soniq_group_codes.restype = i64
+        L.soniq_packed_row_bytes.argtypes = [P, i32, i32]
+        L.soniq_packed_row_bytes.restype = i64
+        L.soniq_validate_layout.argtypes = [P, P]
+        L.soniq_validate_layout.restype = i32
+        L.soniq_launch_count.restype = i64
+        L.soniq_pack_weights.argtypes = [P, P, i32, i32, i32, P, P, P]
+        L.soniq_pack_weights.restype = i32
+        L.soniq_quantize_act.argtypes = [P, P, i64, i32, P, P, P]
+        L.soniq_quantize_act.restype = i32
+        L.soniq_mp_gemm.argtypes = [P, P, P, i32, i64, P, P, i32, P, i32, P, u32, P]
+        L.soniq_mp_gemm.restype = i32
+        L.soniq_mp_conv2d.argtypes = [P, P, P, P, i32, P, P, P, i32, P, u32, P]
+        L.soniq_mp_conv2d.restype = i32
+        L.soniq_sync_status.argtypes = [P]
+        L.soniq_sync_status.restype = i32
+        _lib = L
+    return _lib
+
+
+def _check(status: int, where: str):
+    if status != SONIQ_OK:
+        raise SoniqError(status, where)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t: torch.Tensor, dtype, name: str):
+    if not t.is_cuda or t.dtype != dtype or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous CUDA {dtype} tensor")
+
+
+class Layout:
+    """Per-layer precision layout: groups, bit widths, channel permutation.
+
+    perm[j] is the original channel at packed position j; positions
+    [0, count[0]) form the low-precision group 0.  The permutation is kept in
+    device memory (the kernels gather through it)."""
+
+    def __init__(self, perm: Sequence[int], count: Sequence[int], bits_w: Sequence[int],
+                 bits_a: Optional[Sequence[int]] = None, pad_unit: int = 128, device=None):
+        bits_a = bits_w if bits_a is None else bits_a
+        perm_t = torch.as_tensor(perm, dtype=torch.int32).contiguous()
+        self.K = int(perm_t.numel())
+        count = list(count) + [0] * (2 - len(count))
+        self.count = [int(count[0]), int(count[1])]
+        self.bits_w = [int(b) for b in list(bits_w)[:2]] + [1] * (2 - len(bits_w))
+        self.bits_a = [int(b) for b in list(bits_a)[:2]] + [1] * (2 - len(bits_a))
+        self.pad_unit = int(pad_unit)
+        n_groups = 2 if self.count[1] > 0 else 1
+        host = CLayout(self.K, n_groups, (ctypes.c_int32 * 2)(*self.count),
+                       (ctypes.c_int32 * 2)(*self.bits_w), (ctypes.c_int32 * 2)(*self.bits_a),
+                       None, self.pad_unit)
+        _check(lib().soniq_validate_layout(ctypes.byref(host),
+                                           perm_t.numpy().ctypes.data_as(ctypes.c_void_p)),
+               "soniq_validate_layout")
+        self.perm = perm_t.to(device if device is not None else "cuda")
+        host.perm = ctypes.c_void_p(self.perm.data_ptr())
+        self.c = host
+
+    def row_bytes(self, is_weight: bool = False, taps: int = 1) -> int:
+        v = lib().soniq_packed_row_bytes(ctypes.byref(self.c), int(is_weight), int(taps))
+        if v < 0:
+            raise SoniqError(1, "soniq_packed_row_bytes")
+        return int(v)
+
+    def group_codes(self, g: int, is_weight: bool = False, taps: int = 1) -> int:
+        return int(lib().soniq_group_codes(ctypes.byref(self.c), int(g), int(is_weight), int(taps)))
+
+
+def pack_weights(layout: Layout, W: torch.Tensor, scale_mode: str = "row",
+                 Wp: Optional[torch.Tensor] = None, s_w: Optional[torch.Tensor] = None,
+                 stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """soniq_pack_weights.  W: fp32 [N][K] or [N][taps][K] on the GPU."""
+    _need(W, torch.float32, "W")
+    N = W.shape[0]
+    taps = 1 if W.dim() == 2 else W.shape[1]
+    if Wp is None:
+        Wp = torch.empty((N, layout.row_bytes(True, taps)), dtype=torch.uint8, device=W.device)
+    if s_w is None:
+        s_w = torch.empty((N, 2), dtype=torch.float32, device=W.device)
+    mode = {"row": SCALE_PER_ROW, "tensor": SCALE_PER_TENSOR}[scale_mode]
+    _check(lib().soniq_pack_weights(ctypes.byref(layout.c), _ptr(W), N, taps, mode, _ptr(Wp),
+                                    _ptr(s_w), _stream(stream)), "soniq_pack_weights")
+    return Wp, s_w
+
+
+def quantize_act(layout: Layout, A: torch.Tensor, scale_mode: str = "tensor",
+                 s_a: Optional[torch.Tensor] = None, Ap: Optional[torch.Tensor] = None,
+                 stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """soniq_quantize_act.  A: fp16 [M][K] on the GPU.  For scale_mode
+    'calibrated', s_a ([2] fp32) is an input."""
+    _need(A, torch.float16, "A")
+    M = A.shape[0]
+    mode = _SCALE[scale_mode]
+    if s_a is None:
+        if mode == SCALE_CALIBRATED:
+            raise ValueError("calibrated mode needs s_a")
+        s_a = torch.empty((M, 2) if mode == SCALE_PER_ROW else (2,), dtype=torch.float32,
+                          device=A.device)
+    if Ap is None:
+        Ap = torch.empty((M, layout.row_bytes(False)), dtype=torch.uint8, device=A.device)
+    _check(lib().soniq_quantize_act(ctypes.byref(layout.c), _ptr(A), M, mode, _ptr(s_a), _ptr(Ap),
+                                    _stream(stream)), "soniq_quantize_act")
+    return Ap, s_a
+
+
+def mp_gemm(layout: Layout, Ap: torch.Tensor, s_a: torch.Tensor, Wp: torch.Tensor,
+            s_w: torch.Tensor, scale_mode: str = "tensor", out_dtype=torch.float16,
+            Y: Optional[torch.Tensor] = None, acc_dbg: Optional[torch.Tensor] = None,
+            flags: int = 0, stream=None) -> torch.Tensor:
+    """soniq_mp_gemm: Y[M][N] = dequantized (A W^T) from packed codes."""
+    M, N = Ap.shape[0], Wp.shape[0]
+    if Y is None:
+        Y = torch.empty((M, N), dtype=out_dtype, device=Ap.device)
+    od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
+    _check(lib().soniq_mp_gemm(ctypes.byref(layout.c), _ptr(Ap), _ptr(s_a), _SCALE[scale_mode], M,
+                               _ptr(Wp), _ptr(s_w), N, _ptr(Y), od, _ptr(acc_dbg), int(flags),
+                               _stream(stream)), "soniq_mp_gemm")
+    return Y
+
+
+def conv_desc(batch, H, W, C_out, R=3, S=3, stride=(1, 1), pad=(1, 1)) -> CConvDesc:
+    return CConvDesc(batch, H, W, C_out, R, S, stride[0], stride[1], pad[0], pad[1])
+
+
+def conv_out_hw(cd: CConvDesc) -> Tuple[int, int]:
+    P = (cd.H + 2 * cd.pad_h - cd.R) // cd.stride_h + 1
+    Q = (cd.W + 2 * cd.pad_w - cd.S) // cd.stride_w + 1
+    return P, Q
+
+
+def mp_conv2d(layout: Layout, cd: CConvDesc, Xp: torch.Tensor, s_a: torch.Tensor,
+              Wp: torch.Tensor, s_w: torch.Tensor, scale_mode: str = "tensor",
+              out_dtype=torch.float16, Y: Optional[torch.Tensor] = None,
+              acc_dbg: Optional[torch.Tensor] = None, flags: int = 0, stream=None) -> torch.Tensor:
+    """soniq_mp_conv2d: NHWC implicit-GEMM convolution from packed codes."""
+    P, Q = conv_out_hw(cd)
+    if Y is None:
+        Y = torch.empty((cd.batch, P, Q, cd.C_out), dtype=out_dtype, device=Xp.device)
+    od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
+    _check(lib().soniq_mp_conv2d(ctypes.byref(layout.c), ctypes.byref(cd), _ptr(Xp), _ptr(s_a),
+                                 _SCALE[scale_mode], _ptr(Wp), _ptr(s_w), _ptr(Y), od,
+                                 _ptr(acc_dbg), int(flags), _stream(stream)), "soniq_mp_conv2d")
+    return Y
+
+
+def sync_status(stream=None) -> int:
+    """soniq_sync_status: waits for the stream, returns the status code."""
+    return int(lib().soniq_sync_status(_stream(stream)))
+
+
+def launch_count() -> int:
+    return int(lib().soniq_launch_count())
