@@ -413,6 +413,56 @@ def run_reference(args):
     }), flush=True)
 
 
+def run_case(args):
+    """One kernel family on one workload, for profiling (ncu) and tuning:
+    conv_4b8b | conv_1b4b | quant_conv | gemm:MxNxK:lo:hi:frac | gemv:M."""
+    import torch
+    from paper_2311_14114_gb300 import soniq as sq
+    from paper_2311_14114_gb300 import workloads as wl
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    name = args.case
+    if name.startswith("conv") or name == "quant_conv":
+        spec = wl.CONV_RESNET_1B4B if name == "conv_1b4b" else wl.CONV_RESNET
+        d = wl.make_conv(spec)
+        lay = sq.Layout(d["perm"], d["count"], d["bits"], pad_unit=32)
+        X = torch.from_numpy(d["X"]).cuda().reshape(-1, spec.C)
+        Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
+        Xp, s_a = sq.quantize_act(lay, X)
+        cd = sq.conv_desc(spec.batch, spec.H, spec.W, spec.C_out, spec.R, spec.S, spec.stride, spec.pad)
+        Y = torch.empty((spec.batch, 14, 14, spec.C_out), dtype=torch.float16, device="cuda")
+        if name == "quant_conv":
+            fn, ops = (lambda: sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp)), 0
+        else:
+            fn, ops = (lambda: sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y)), spec.ops
+    elif name.startswith("gemm:"):
+        _, shape, lo, hi, frac = name.split(":")
+        M, N, K = (int(x) for x in shape.split("x"))
+        spec = wl.LinearSpec(name, M=M, K=K, N=N, bits_lo=int(lo), bits_hi=int(hi), frac_hi=float(frac))
+        d = wl.make_linear(spec)
+        lay = sq.Layout(d["perm"], d["count"], d["bits"])
+        Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
+        Ap, s_a = sq.quantize_act(lay, torch.from_numpy(d["A"]).cuda())
+        Y = torch.empty((M, N), dtype=torch.float16, device="cuda")
+        fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y, flags=sq.FLAG_FORCE_MMA)), spec.ops
+    elif name.startswith("gemv:"):
+        spec = wl.DECODE[int(name.split(":")[1])]
+        d = wl.make_linear(spec)
+        lay = sq.Layout(d["perm"], d["count"], d["bits"])
+        Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
+        Ap, s_a = sq.quantize_act(lay, torch.from_numpy(d["A"]).cuda())
+        Y = torch.empty((spec.M, spec.N), dtype=torch.float16, device="cuda")
+        fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y)), spec.ops
+    else:
+        raise SystemExit(f"unknown case {name}")
+    ms = _time_events(fn, args.steps, flush, stream)
+    if sq.sync_status() != 0:
+        raise RuntimeError("device error")
+    print(json.dumps({"case": name, "us": round(ms * 1e3, 2),
+                      "TOPS": round(ops / (ms * 1e-3) / 1e12, 2) if ops else None}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -423,10 +473,13 @@ def main():
     ap.add_argument("--full-sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--case", default=None, help="profile one kernel family on one workload")
     ap.add_argument("--traffic", type=float, default=None,
                     help="DRAM bytes per conv launch from an ncu capture of the same kernel")
     args = ap.parse_args()
-    if args.impl == "reference":
+    if args.case:
+        run_case(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)

@@ -20,19 +20,30 @@
 // segments short enough for the worst case, and the epilogue warps drain each
 // finished segment into an int32 sum kept in TMEM.
 //
+// Data movement.  K is walked in chunks of 128 codes.  Each chunk's packed
+// activation rows (128 x 16*na bytes) and packed weight rows (128 x 16*nw
+// bytes) land in one slot of a byte ring in shared memory whose slots are
+// sized per precision group, so low-bit chunks keep many copies in flight.
+// Weights always arrive by TMA; activations by TMA when the rows allow it
+// (GEMM with 128-code padding), otherwise the producer warp gathers them with
+// cp.async (implicit-GEMM conv: one pixel row per output row and tap, zero
+// fill outside the image).  Packed tiles with 2-, 4- or 8-bit codes use the
+// TMA 32/64/128-byte swizzle so the converters read them without bank
+// conflicts.
+//
 // CTA = 128x128 output tile, 14 warps:
-//   warp 0      TMA producer: packed weight tiles -> shared memory ring
+//   warp 0      producer: ring space, TMA copies, cp.async gathers
 //   warp 1      MMA issuer (one thread) + TMEM owner
-//   warps 2-5   expand the 128 activation rows of each K-stage (a conv gathers
-//               its im2col rows here; pixels outside the image are code 0)
-//   warps 6-9   expand the 128 weight rows from the TMA ring
+//   warps 2-5   convert the 128 activation rows of each K-stage
+//   warps 6-9   convert the 128 weight rows
 //   warps 10-13 segment drains and the epilogue (tcgen05.ld -> fp32 -> fp16)
-// A K-stage is 128 bytes of operand per row (128 E4M3 codes or 64 fp16
-// codes) in the 128-byte-swizzled K-major layout the MMA descriptors read.
+// A K-stage is 128 bytes of MMA operand per row (128 E4M3 codes or 64 fp16
+// codes) in the 128-byte-swizzled K-major layout the MMA descriptors read;
+// an E4M3 chunk is one stage, an fp16 chunk two.
 //
 // Every wait is bounded; a wait that runs out records an error bit in the
 // device error word, raises a CTA-wide abort flag and the CTA winds down
-// (in-flight MMAs and TMA copies are waited for, TMEM is freed).
+// (in-flight MMAs and copies are waited for, TMEM is freed).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -46,26 +57,24 @@ namespace mma {
 
 constexpr int BM = 128;
 constexpr int BN = 128;
-constexpr int OP_STAGES = 4;
-constexpr int W_STAGES = 3;
+constexpr int OP_STAGES = 3;
 constexpr int ROW_BYTES = 128;                       // operand bytes per row per K-stage
 constexpr int OP_A_BYTES = BM * ROW_BYTES;           // 16 KB
 constexpr int OP_B_BYTES = BN * ROW_BYTES;           // 16 KB
 constexpr int OP_STAGE_BYTES = OP_A_BYTES + OP_B_BYTES;
-constexpr int W_STAGE_BYTES = BN * 128;              // BN rows x (16 * n <= 128) packed bytes
+constexpr int PK_BYTES = 96 * 1024;                  // packed chunk ring
+constexpr int PK_SLOTS = 16;                         // chunks in flight at most
 constexpr int NUM_WARPS = 14;
 constexpr int NUM_THREADS = NUM_WARPS * 32;
-constexpr int WARP_TMA = 0, WARP_MMA = 1, WARP_EXPA = 2, WARP_EXPW = 6, WARP_EPI = 10;
+constexpr int WARP_PROD = 0, WARP_MMA = 1, WARP_CVA = 2, WARP_CVW = 6, WARP_EPI = 10;
 
 constexpr int SMEM_OP = 0;
-constexpr int SMEM_W = SMEM_OP + OP_STAGES * OP_STAGE_BYTES;
-constexpr int SMEM_BAR = SMEM_W + W_STAGES * W_STAGE_BYTES;
-// barriers: w_full[3] w_empty[3] op_full[4] op_empty[4] seg_full[2] slot_free[2]
-//           acc_full rowsum_ready teardown
-constexpr int BAR_W_FULL = 0, BAR_W_EMPTY = 3, BAR_OP_FULL = 6, BAR_OP_EMPTY = 10,
-              BAR_SEG_FULL = 14, BAR_SLOT_FREE = 16, BAR_ACC_FULL = 18, BAR_ROWSUM = 19,
-              BAR_TEARDOWN = 20, NUM_BARS = 21;
-constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;   // tmem base, abort flag
+constexpr int SMEM_PK = SMEM_OP + OP_STAGES * OP_STAGE_BYTES;
+constexpr int SMEM_BAR = SMEM_PK + PK_BYTES;
+constexpr int BAR_PK_FULL = 0, BAR_PK_EMPTY = 16, BAR_OP_FULL = 32, BAR_OP_EMPTY = 35,
+              BAR_SEG_FULL = 38, BAR_SLOT_FREE = 40, BAR_ACC_FULL = 42, BAR_ROWSUM = 43,
+              BAR_TEARDOWN = 44, NUM_BARS = 45;
+constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;         // tmem base, abort flag
 constexpr int SMEM_ROWSUM = (SMEM_MISC + 16 + 15) & ~15;   // int32 [2][128]
 constexpr int SMEM_SW = SMEM_ROWSUM + 2 * BM * 4;          // fp32 [2][128]
 constexpr int SMEM_TOTAL = SMEM_SW + 2 * BN * 4;
@@ -76,18 +85,22 @@ struct Group {
     int32_t kind;          // 0: E4M3 codes (offset-binary weights), 1: fp16 codes
     int32_t pa;            // activation codes per tap
     int32_t pw;            // weight codes per row
-    int32_t a_off, w_off;
+    int32_t a_off, w_off;  // byte offsets of the group in packed rows
     int32_t n_stages;      // K-stages
     int32_t seg_stages;    // K-stages per exact accumulation segment
     int32_t n_seg;
     int32_t w_offset;      // 2^(nw-1) for kind 0, else 0
-    int32_t chunk_base;    // index of the group's first 128-code weight chunk
+    int32_t chunk_base;    // index of the group's first 128-code chunk
+    int32_t a_bytes;       // packed activation bytes of one chunk (128 rows)
+    int32_t w_bytes;       // packed weight bytes of one chunk (128 rows)
+    int32_t copy_bytes;    // cp.async width of the activation gather (4, 8 or 16)
     float acc_scale;       // 2^18 for kind 0 (E4M3 codes carry 2^-9 each), 1 for kind 1
     float inv_levels;      // 1 / ((2^na - 1) * 2^(nw-1))
 };
 
 struct Params {
     CUtensorMap tmw[2];    // packed weights, one box width per group
+    CUtensorMap tma[2];    // packed activations (used when a_tma)
     const uint8_t* Ap;
     const uint8_t* Wp;
     const float* s_a;
@@ -99,6 +112,7 @@ struct Params {
     int32_t N;
     int32_t a_row_bytes;
     int32_t conv;
+    int32_t a_tma;         // 1: activation chunks by TMA, 0: cp.async gather
     int32_t H, W, P, Q, R, S, sh, sw, ph, pw;
     int32_t s_a_per_row;
     int32_t out_bf16;
@@ -254,19 +268,52 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
         : "memory");
 }
 
-// Swizzled byte offset of 16-byte chunk `chunk` of operand row `row`.
+// cp.async copies of 4, 8 or 16 bytes; src_bytes = 0 zero-fills the destination.
+__device__ __forceinline__ void cp_async(uint32_t dst, const void* src, int bytes, uint32_t src_bytes) {
+    if (bytes == 16)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+    else if (bytes == 8)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+    else
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+
+// Arrives on `bar` once all of this thread's earlier cp.async copies have landed.
+__device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+// XOR applied to the 16-byte chunk index of a packed row of n-bit codes
+// (16*n bytes per 128 codes): the TMA 32/64/128-byte swizzle for n = 2/4/8,
+// none otherwise.  Address bits [4, 4+k) are XORed with bits [7, 7+k).
+__device__ __forceinline__ uint32_t pk_xor(int n, uint32_t row) {
+    return (n == 2 || n == 4 || n == 8) ? ((row * (uint32_t)n) >> 3) & (uint32_t)(n - 1) : 0u;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+
+// Byte offset of 16-byte chunk `chunk` of operand row `row` in the MMA tile
+// (128-byte swizzle: 8-row x 128-byte atoms).
 __device__ __forceinline__ uint32_t sw128_off(uint32_t row, uint32_t chunk) {
     return row * 128u + ((chunk ^ (row & 7u)) << 4);
 }
 
-// ---- stage bookkeeping -------------------------------------------------------
+// ---- stage and chunk bookkeeping --------------------------------------------
 
 struct StageInfo {
-    int g;        // group
-    int ls;       // stage index inside the group
+    int g;       // group
+    int ls;      // stage index inside the group
     int kind;
-    int kb0;      // first 32-code block of the stage inside the group's weight K range
-    int nblk;     // blocks per stage: 4 (E4M3) or 2 (fp16)
+    int half;    // fp16 stages: which half of the chunk
+    bool chunk_first, chunk_last;
 };
 
 __device__ __forceinline__ StageInfo stage_info(const Params& p, int s) {
@@ -274,115 +321,190 @@ __device__ __forceinline__ StageInfo stage_info(const Params& p, int s) {
     si.g = s < p.g[0].n_stages ? 0 : 1;
     si.ls = si.g ? s - p.g[0].n_stages : s;
     si.kind = p.g[si.g].kind;
-    si.nblk = si.kind == 0 ? 4 : 2;
-    si.kb0 = si.ls * si.nblk;
+    si.half = si.kind == 0 ? 0 : (si.ls & 1);
+    si.chunk_first = si.half == 0;
+    si.chunk_last = si.kind == 0 || si.half == 1;
     return si;
 }
 
-// ---- activation-side loads (GEMM rows or im2col gather) -----------------------
+__device__ __forceinline__ int chunk_group(const Params& p, int ci) { return ci < p.g[1].chunk_base ? 0 : 1; }
 
-// Loads the packed activation words of one K-stage for output row `m` into
-// `buf` (block i at buf[i * n]); blocks outside the data are zero.
-__device__ __forceinline__ void load_act_stage(const Params& p, const StageInfo& si, int64_t m,
-                                               int img, int pp, int qq, uint32_t* buf) {
-    const Group& G = p.g[si.g];
-    const int n = G.bits_a;
-    const int cpt = G.pa >> 5;           // blocks per tap
-    const int taps = p.conv ? p.R * p.S : 1;
+__device__ __forceinline__ uint32_t chunk_size(const Params& p, int ci) {
+    const Group& G = p.g[chunk_group(p, ci)];
+    return (uint32_t)(G.a_bytes + G.w_bytes);
+}
+
+// Ring offset of chunk ci+1 from that of chunk ci: slots follow each other and
+// wrap to 0 when the next one would not fit.
+__device__ __forceinline__ uint32_t ring_next(const Params& p, int ci, uint32_t off) {
+    uint32_t nxt = off + chunk_size(p, ci);
+    if (ci + 1 < p.total_chunks && nxt + chunk_size(p, ci + 1) > (uint32_t)PK_BYTES) nxt = 0;
+    return nxt;
+}
+
+// ---- conversion of packed codes into the MMA operand tile ---------------------
+
+// Reads this row's packed words of one chunk (n 16-byte pieces, swizzled).
+template <int N>
+__device__ __forceinline__ void read_chunk(uint32_t row_base, uint32_t xr, uint32_t* w) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        if (i >= si.nblk) break;
-        const int kb = si.kb0 + i;
-        const uint32_t* src = nullptr;
-        if (m < p.M && cpt > 0) {
-            const int tap = kb / cpt;
-            const int cb = kb - tap * cpt;
-            if (tap < taps) {
-                if (!p.conv) {
-                    src = reinterpret_cast<const uint32_t*>(p.Ap + m * p.a_row_bytes + G.a_off + cb * 4 * n);
-                } else {
-                    const int r = tap / p.S, s = tap - (tap / p.S) * p.S;
-                    const int h = pp * p.sh - p.ph + r, w = qq * p.sw - p.pw + s;
-                    if (h >= 0 && h < p.H && w >= 0 && w < p.W)
-                        src = reinterpret_cast<const uint32_t*>(
-                            p.Ap + (((int64_t)img * p.H + h) * p.W + w) * p.a_row_bytes + G.a_off + cb * 4 * n);
-                }
-            }
-        }
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            if (q >= n) break;
-            buf[i * 8 + q] = src ? __ldg(src + q) : 0u;
-        }
+    for (int j = 0; j < N; ++j) {
+        const uint4 v = lds128(row_base + ((j ^ xr) << 4));
+        w[4 * j] = v.x;
+        w[4 * j + 1] = v.y;
+        w[4 * j + 2] = v.z;
+        w[4 * j + 3] = v.w;
     }
 }
 
-// ---- expansion into the swizzled operand tile --------------------------------
-
-// Activation row: unsigned codes.  E4M3: the byte is the code (value c*2^-9);
-// fp16: 1024 + c - 1024.
-__device__ __forceinline__ uint32_t expand_act_stage(const StageInfo& si, int n, const uint32_t* buf,
-                                                     uint8_t* tile, int row) {
+// E4M3 stage: 4 blocks of 32 codes -> 128 bytes.  Activations: the byte is the
+// code; weights: sign bit flipped (offset binary).  Returns the code sum.
+template <int N, bool A_SIDE>
+__device__ __forceinline__ uint32_t cvt_e4m3(const uint32_t* w, uint32_t tile, uint32_t row) {
     uint32_t rsum = 0;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        if (i >= si.nblk) break;
         uint32_t o[8];
-        block_to_bytes_n(n, buf + i * 8, o);
-        if (si.kind == 0) {
+        block_to_bytes<N>(w + i * N, o);
 #pragma unroll
-            for (int t = 0; t < 8; ++t) rsum = __dp4a(o[t], 0x01010101u, rsum);
-            *reinterpret_cast<uint4*>(tile + sw128_off(row, 2 * i)) = make_uint4(o[0], o[1], o[2], o[3]);
-            *reinterpret_cast<uint4*>(tile + sw128_off(row, 2 * i + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
-        } else {
-            const __half2 bias = __half2half2(__ushort_as_half((unsigned short)0x6400u));
-            uint32_t h[16];
-#pragma unroll
-            for (int t = 0; t < 8; ++t) {
-                uint32_t lo, hi;
-                bytes_to_magic_half2(o[t], lo, hi);
-                h[2 * t] = half2_sub(lo, bias);
-                h[2 * t + 1] = half2_sub(hi, bias);
-            }
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                *reinterpret_cast<uint4*>(tile + sw128_off(row, 4 * i + c)) =
-                    make_uint4(h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
+        for (int t = 0; t < 8; ++t) {
+            if constexpr (A_SIDE) rsum = __dp4a(o[t], 0x01010101u, rsum);
+            else o[t] ^= 0x01010101u << (N - 1);
         }
+        sts128(tile + sw128_off(row, 2 * i), o[0], o[1], o[2], o[3]);
+        sts128(tile + sw128_off(row, 2 * i + 1), o[4], o[5], o[6], o[7]);
     }
     return rsum;
 }
 
-// Weight row: n-bit two's complement -> offset binary (sign-bit flip).
-// E4M3: the offset-binary byte is the code; fp16: 1024 + (j + 2^(n-1)) - (1024 + 2^(n-1)) = j.
-__device__ __forceinline__ void expand_w_stage(const StageInfo& si, int n, const uint32_t* buf,
-                                               uint8_t* tile, int row) {
-    const uint32_t flip = sign_flip_mask(n);
+// fp16 stage: blocks 2h, 2h+1 of the chunk -> 64 fp16 values (128 bytes).
+// Activations: 1024 + u - 1024; weights: 1024 + (j + 2^(n-1)) - (1024 + 2^(n-1)).
+template <int N, bool A_SIDE>
+__device__ __forceinline__ void cvt_f16(const uint32_t* w, int half, uint32_t tile, uint32_t row) {
+    const __half2 bias = __half2half2(
+        __ushort_as_half((unsigned short)(A_SIDE ? 0x6400u : (0x6400u + (1u << (N - 1))))));
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        uint32_t o[8];
+        block_to_bytes<N>(w + (2 * half + i) * N, o);
+        uint32_t h[16];
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            uint32_t lo, hi;
+            bytes_to_magic_half2(A_SIDE ? o[t] : (o[t] ^ (0x01010101u << (N - 1))), lo, hi);
+            h[2 * t] = half2_sub(lo, bias);
+            h[2 * t + 1] = half2_sub(hi, bias);
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+            sts128(tile + sw128_off(row, 4 * i + c), h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
+    }
+}
+
+// ---- activation gather (implicit GEMM / unaligned rows) -----------------------
+
+// Per-row state of the gather: output pixel coordinates of the 4 rows a lane owns.
+struct GatherRows {
+    int64_t base[4];   // GEMM: the row index m; conv: img * H (input row base)
+    int pp[4], qq[4];  // conv: output pixel coordinates
+    bool valid[4];
+};
+
+// Issues the cp.async copies of chunk (g, c) for the 4 rows of this lane into
+// the ring slot at `slot` (swizzled like the TMA tiles).  Block kb of the
+// group's weight K range holds tap kb / cpt, channel block kb % cpt; taps
+// beyond R*S and pixels outside the image are zero-filled.
+__device__ __forceinline__ void gather_chunk(const Params& p, const GatherRows& gr, int lane, int g, int c,
+                                             uint32_t slot) {
+    const Group& G = p.g[g];
+    const int n = G.bits_a;
+    const int cpt = G.pa >> 5;
+    const int taps = p.conv ? p.R * p.S : 1;
+    const int bw = G.copy_bytes;
+    const int blk_bytes = 4 * n;
+    const int row_bytes = 16 * n;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        if (i >= si.nblk) break;
-        uint32_t o[8];
-        block_to_bytes_n(n, buf + i * 8, o);
+        const int kb = 4 * c + i;
+        const int tap = cpt > 0 ? kb / cpt : taps;
+        const int cb = kb - tap * cpt;
+        const int r = tap / p.S, s = tap - r * p.S;
 #pragma unroll
-        for (int t = 0; t < 8; ++t) o[t] ^= flip;
-        if (si.kind == 0) {
-            *reinterpret_cast<uint4*>(tile + sw128_off(row, 2 * i)) = make_uint4(o[0], o[1], o[2], o[3]);
-            *reinterpret_cast<uint4*>(tile + sw128_off(row, 2 * i + 1)) = make_uint4(o[4], o[5], o[6], o[7]);
-        } else {
-            const __half2 bias = __half2half2(__ushort_as_half((unsigned short)(0x6400u + (1u << (n - 1)))));
-            uint32_t h[16];
-#pragma unroll
-            for (int t = 0; t < 8; ++t) {
-                uint32_t lo, hi;
-                bytes_to_magic_half2(o[t], lo, hi);
-                h[2 * t] = half2_sub(lo, bias);
-                h[2 * t + 1] = half2_sub(hi, bias);
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t row = (uint32_t)(lane + 32 * k);
+            const uint8_t* src = p.Ap;   // any valid address when zero-filling
+            uint32_t nbytes = 0;
+            if (gr.valid[k] && tap < taps) {
+                if (!p.conv) {
+                    src = p.Ap + gr.base[k] * p.a_row_bytes + G.a_off + cb * blk_bytes;
+                    nbytes = (uint32_t)bw;
+                } else {
+                    const int h = gr.pp[k] * p.sh - p.ph + r, w = gr.qq[k] * p.sw - p.pw + s;
+                    if (h >= 0 && h < p.H && w >= 0 && w < p.W) {
+                        src = p.Ap + ((gr.base[k] + h) * p.W + w) * p.a_row_bytes + G.a_off + cb * blk_bytes;
+                        nbytes = (uint32_t)bw;
+                    }
+                }
             }
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                *reinterpret_cast<uint4*>(tile + sw128_off(row, 4 * i + c)) =
-                    make_uint4(h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
+            const uint32_t xr = pk_xor(n, row);
+            for (int b = 0; b < blk_bytes; b += bw) {
+                const int byte = i * blk_bytes + b;   // within the row's 16*n bytes
+                const uint32_t dst = slot + row * row_bytes + ((((uint32_t)byte >> 4) ^ xr) << 4) + (byte & 15);
+                cp_async(dst, nbytes ? (const void*)(src + b) : (const void*)p.Ap, bw, nbytes);
+            }
         }
+    }
+}
+
+// ---- converter: one packed chunk of one row -> one or two MMA stages ---------------
+
+struct CvtCtx {
+    uint32_t smem;        // shared-memory address of the aligned base
+    uint32_t bar0;
+    volatile int* abort_flag;
+    int warp, lane;
+    uint32_t row;
+};
+
+// Waits for each operand stage of chunk ci (1 for E4M3, 2 for fp16), converts
+// this row into it and signals the MMA.  Returns false when the CTA aborts.
+template <int N, bool A_SIDE>
+__device__ __forceinline__ bool convert_chunk(const Params& p, const CvtCtx& cx, uint32_t row_base, int s0,
+                                              int nst, int kind, uint32_t& rsum) {
+    uint32_t w[4 * N];
+    read_chunk<N>(row_base, pk_xor(N, cx.row), w);
+    for (int h = 0; h < nst; ++h) {
+        const int s = s0 + h;
+        const int slot = s % OP_STAGES;
+        if (!__all_sync(0xffffffffu, wait_bounded(cx.bar0 + 8u * (BAR_OP_EMPTY + slot), ((s / OP_STAGES) & 1) ^ 1,
+                                                    cx.abort_flag, p)))
+            return false;
+        const uint32_t tile = cx.smem + SMEM_OP + slot * OP_STAGE_BYTES + (A_SIDE ? 0 : OP_A_BYTES);
+        if (kind == 0) {
+            if constexpr (N <= 4) rsum += cvt_e4m3<N, A_SIDE>(w, tile, cx.row);
+        } else {
+            cvt_f16<N, A_SIDE>(w, h, tile, cx.row);
+        }
+        fence_proxy_async();
+        __syncwarp();
+        const bool drop = (p.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) && s == 0 && cx.warp == WARP_CVA;
+        if (cx.lane == 0 && !drop) mbar_arrive(cx.bar0 + 8u * (BAR_OP_FULL + slot));
+    }
+    return true;
+}
+
+template <bool A_SIDE>
+__device__ __forceinline__ bool convert_chunk_n(int n, const Params& p, const CvtCtx& cx, uint32_t row_base,
+                                                int s0, int nst, int kind, uint32_t& rsum) {
+    switch (n) {
+        case 1: return convert_chunk<1, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
+        case 2: return convert_chunk<2, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
+        case 3: return convert_chunk<3, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
+        case 4: return convert_chunk<4, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
+        case 5: return convert_chunk<5, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
+        case 6: return convert_chunk<6, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
+        case 7: return convert_chunk<7, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
+        default: return convert_chunk<8, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
     }
 }
 
@@ -401,11 +523,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + SMEM_MISC + 4);
     int32_t* rowsum_s = reinterpret_cast<int32_t*>(smem + SMEM_ROWSUM);
     float* sw_s = reinterpret_cast<float*>(smem + SMEM_SW);
+    const uint32_t pk_base = smem_u32(smem + SMEM_PK);
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < W_STAGES; ++i) {
-            mbar_init(bar(BAR_W_FULL + i), 1);
-            mbar_init(bar(BAR_W_EMPTY + i), 4);
+        for (int i = 0; i < PK_SLOTS; ++i) {
+            // TMA arrival (+ the 32 gather lanes of the producer warp)
+            mbar_init(bar(BAR_PK_FULL + i), p.a_tma ? 1 : 33);
+            mbar_init(bar(BAR_PK_EMPTY + i), 8);
         }
         for (int i = 0; i < OP_STAGES; ++i) {
             mbar_init(bar(BAR_OP_FULL + i), 8);
@@ -440,28 +564,78 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    if (warp == WARP_TMA) {
-        // ------------------------------------------------------------------ TMA
-        if (lane == 0) {
-            int issued = 0;
-            for (int ci = 0; ci < p.total_chunks; ++ci) {
-                const int slot = ci % W_STAGES;
-                if (!wait_bounded(bar(BAR_W_EMPTY + slot), ((ci / W_STAGES) & 1) ^ 1, abort_flag, p)) break;
-                const int g = ci < p.g[1].chunk_base ? 0 : 1;
-                const Group& G = p.g[g];
-                const int c = ci - G.chunk_base;
-                const uint32_t bytes = (uint32_t)BN * 16u * (uint32_t)G.bits_w;
-                mbar_arrive_expect_tx(bar(BAR_W_FULL + slot), bytes);
-                tma_load_2d(smem_u32(smem + SMEM_W + slot * W_STAGE_BYTES), &p.tmw[g],
-                            G.w_off + c * 16 * G.bits_w, n0, bar(BAR_W_FULL + slot));
-                ++issued;
-            }
-            // copies still in flight must land before the CTA's memory is released
-            for (int ci = issued - W_STAGES < 0 ? 0 : issued - W_STAGES; ci < issued; ++ci) {
-                volatile int no_abort = 0;
-                wait_bounded(bar(BAR_W_FULL + ci % W_STAGES), (ci / W_STAGES) & 1, &no_abort, p);
+    if (warp == WARP_PROD) {
+        // ------------------------------------------------------------- producer
+        GatherRows gr;
+        if (!p.a_tma) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int64_t m = m0 + lane + 32 * k;
+                gr.valid[k] = m < p.M;
+                gr.base[k] = m;
+                gr.pp[k] = gr.qq[k] = 0;
+                if (p.conv && gr.valid[k]) {
+                    const int64_t pq = (int64_t)p.P * p.Q;
+                    const int64_t img = m / pq;
+                    const int rem = (int)(m - img * pq);
+                    gr.pp[k] = rem / p.Q;
+                    gr.qq[k] = rem - gr.pp[k] * p.Q;
+                    gr.base[k] = img * p.H;
+                }
             }
         }
+        // Ring bookkeeping (identical on all lanes): chunks rel..ci-1 are in
+        // flight; `tail` is the offset of chunk rel, `off` that of chunk ci and
+        // `head` the end of chunk ci-1 before the wrap decision.
+        int rel = 0;
+        int issued = 0;
+        uint32_t off = 0, tail = 0, head = 0;
+        bool ok = true;
+        for (int ci = 0; ci < p.total_chunks && ok; ++ci) {
+            const int g = chunk_group(p, ci);
+            const Group& G = p.g[g];
+            const int c = ci - G.chunk_base;
+            const uint32_t sz = (uint32_t)(G.a_bytes + G.w_bytes);
+            const int b = ci % PK_SLOTS;
+            while (rel < ci) {
+                // is [off, off + sz) clear of the chunks in flight, and is a barrier pair free?
+                bool fits;
+                if (ci - rel >= PK_SLOTS) fits = false;
+                else if (off == head) fits = head > tail || head + sz <= tail;   // tail == head: ring full
+                else fits = head > tail && sz <= tail;                           // wrapped to offset 0
+                if (fits) break;
+                if (!__all_sync(0xffffffffu,
+                                wait_bounded(bar(BAR_PK_EMPTY + rel % PK_SLOTS), (rel / PK_SLOTS) & 1, abort_flag, p))) {
+                    ok = false;
+                    break;
+                }
+                tail = ring_next(p, rel, tail);
+                ++rel;
+            }
+            if (!ok) break;
+            const uint32_t slot = pk_base + off;
+            if (lane == 0) {
+                mbar_arrive_expect_tx(bar(BAR_PK_FULL + b), (uint32_t)(G.w_bytes + (p.a_tma ? G.a_bytes : 0)));
+                tma_load_2d(slot + G.a_bytes, &p.tmw[g], G.w_off + c * 16 * G.bits_w, n0, bar(BAR_PK_FULL + b));
+                if (p.a_tma)
+                    tma_load_2d(slot, &p.tma[g], G.a_off + c * 16 * G.bits_a, (int)m0, bar(BAR_PK_FULL + b));
+            }
+            if (!p.a_tma) {
+                gather_chunk(p, gr, lane, g, c, slot);
+                cp_async_arrive(bar(BAR_PK_FULL + b));
+            }
+            head = off + sz;
+            off = ring_next(p, ci, off);
+            ++issued;
+        }
+        // copies still in flight must land before the CTA's memory is released
+        if (lane == 0) {
+            for (int ci = issued - PK_SLOTS < 0 ? 0 : issued - PK_SLOTS; ci < issued; ++ci) {
+                volatile int no_abort = 0;
+                wait_bounded(bar(BAR_PK_FULL + ci % PK_SLOTS), (ci / PK_SLOTS) & 1, &no_abort, p);
+            }
+        }
+        asm volatile("cp.async.wait_all;" ::: "memory");
     } else if (warp == WARP_MMA) {
         // ------------------------------------------------------------------ MMA
         if (lane == 0) {
@@ -515,84 +689,42 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
             wait_bounded(bar(BAR_TEARDOWN), 0, &no_abort, p);
         }
     } else if (warp < WARP_EPI) {
-        // ------------------------------------------------------------ expanders
-        const bool is_a = warp < WARP_EXPW;
-        const int row = threadIdx.x - (is_a ? WARP_EXPA : WARP_EXPW) * 32;
-        if (is_a) {
-            const int64_t m = m0 + row;
-            int img = 0, pp = 0, qq = 0;
-            if (p.conv && m < p.M) {
-                const int64_t pq = (int64_t)p.P * p.Q;
-                img = (int)(m / pq);
-                const int rem = (int)(m - (int64_t)img * pq);
-                pp = rem / p.Q;
-                qq = rem - pp * p.Q;
-            }
-            uint32_t cur[32], nxt[32];
-            if (p.total_stages > 0) load_act_stage(p, stage_info(p, 0), m, img, pp, qq, cur);
-            uint32_t rsum = 0;
-            for (int s = 0; s < p.total_stages; ++s) {
-                const StageInfo si = stage_info(p, s);
-                if (s + 1 < p.total_stages) load_act_stage(p, stage_info(p, s + 1), m, img, pp, qq, nxt);
-                const int slot = s % OP_STAGES;
-                if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_OP_EMPTY + slot), ((s / OP_STAGES) & 1) ^ 1,
-                                                            abort_flag, p)))
-                    break;
-                rsum += expand_act_stage(si, p.g[si.g].bits_a, cur, smem + SMEM_OP + slot * OP_STAGE_BYTES, row);
-                if (si.ls == p.g[si.g].n_stages - 1) {
-                    rowsum_s[si.g * BM + row] = (int32_t)rsum;
+        // ----------------------------------------------------------- converters
+        const bool a_side = warp < WARP_CVW;
+        CvtCtx cx{smem_u32(smem), bar0, abort_flag, warp, lane,
+                  (uint32_t)(threadIdx.x - (a_side ? WARP_CVA : WARP_CVW) * 32)};
+        uint32_t rsum = 0;
+        uint32_t off = 0;
+        int s0 = 0;
+        for (int ci = 0; ci < p.total_chunks; ++ci) {
+            const int g = chunk_group(p, ci);
+            const Group& G = p.g[g];
+            const int nst = G.kind == 0 ? 1 : 2;
+            if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_PK_FULL + ci % PK_SLOTS), (ci / PK_SLOTS) & 1,
+                                                        abort_flag, p)))
+                break;
+            bool ok;
+            if (a_side) {
+                const uint32_t rb = pk_base + off + cx.row * 16u * (uint32_t)G.bits_a;
+                ok = convert_chunk_n<true>(G.bits_a, p, cx, rb, s0, nst, G.kind, rsum);
+                if (ci == G.chunk_base + G.pw / 128 - 1) {   // last chunk of the group
+                    rowsum_s[g * BM + cx.row] = (int32_t)rsum;
                     rsum = 0;
                 }
-                fence_proxy_async();
-                __syncwarp();
-                const bool drop = (p.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) && s == 0 && warp == WARP_EXPA;
-                if (lane == 0 && !drop) mbar_arrive(bar(BAR_OP_FULL + slot));
-#pragma unroll
-                for (int i = 0; i < 32; ++i) cur[i] = nxt[i];
+            } else {
+                const uint32_t rb = pk_base + off + G.a_bytes + cx.row * 16u * (uint32_t)G.bits_w;
+                uint32_t unused = 0;
+                ok = convert_chunk_n<false>(G.bits_w, p, cx, rb, s0, nst, G.kind, unused);
             }
+            if (!ok) break;
+            // the slot goes back to the producer only after its words are consumed
+            if (lane == 0) mbar_arrive(bar(BAR_PK_EMPTY + ci % PK_SLOTS));
+            off = ring_next(p, ci, off);
+            s0 += nst;
+        }
+        if (a_side) {
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(BAR_ROWSUM));
-        } else {
-            int ci = 0;
-            for (int s = 0; s < p.total_stages; ++s) {
-                const StageInfo si = stage_info(p, s);
-                const Group& G = p.g[si.g];
-                const int n = G.bits_w;
-                const int half = si.kind == 0 ? 0 : (si.ls & 1);
-                const int wslot = ci % W_STAGES;
-                if (half == 0 &&
-                    !__all_sync(0xffffffffu, wait_bounded(bar(BAR_W_FULL + wslot), (ci / W_STAGES) & 1, abort_flag, p)))
-                    break;
-                // this stage's blocks of the packed row: 128 codes (E4M3) or one half of them (fp16)
-                uint32_t buf[32];
-                const uint32_t* src = reinterpret_cast<const uint32_t*>(
-                    smem + SMEM_W + wslot * W_STAGE_BYTES + row * 16 * n + half * 8 * n);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    if (i >= si.nblk) break;
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        if (q >= n) break;
-                        buf[i * 8 + q] = src[i * n + q];
-                    }
-                }
-                const int slot = s % OP_STAGES;
-                if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_OP_EMPTY + slot), ((s / OP_STAGES) & 1) ^ 1,
-                                                            abort_flag, p)))
-                    break;
-                expand_w_stage(si, n, buf, smem + SMEM_OP + slot * OP_STAGE_BYTES + OP_A_BYTES, row);
-                fence_proxy_async();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(bar(BAR_OP_FULL + slot));
-                // The packed slot goes back to the TMA producer only after its words have
-                // been consumed by the expansion above: releasing it right after the
-                // shared-memory loads let the next TMA copy land before those loads had
-                // read the slot (an intermittent wrong 32-row block of weights).
-                if (si.kind == 0 || half == 1) {
-                    if (lane == 0) mbar_arrive(bar(BAR_W_EMPTY + wslot));
-                    ++ci;
-                }
-            }
         }
     } else {
         // ---------------------------------------------------- drains + epilogue
@@ -719,6 +851,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
         }
     }
 
+
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -749,6 +882,27 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
+// The swizzle the converters expect for packed rows of n-bit codes.
+CUtensorMapSwizzle packed_swizzle(int n) {
+    if (n == 2) return CU_TENSOR_MAP_SWIZZLE_32B;
+    if (n == 4) return CU_TENSOR_MAP_SWIZZLE_64B;
+    if (n == 8) return CU_TENSOR_MAP_SWIZZLE_128B;
+    return CU_TENSOR_MAP_SWIZZLE_NONE;
+}
+
+// 2-D map over packed rows [rows][row_bytes] with a box of one 128-code chunk
+// (16*n bytes) by 128 rows.
+bool encode_packed(EncodeTiledFn enc, CUtensorMap* map, const uint8_t* base, int64_t row_bytes, int64_t rows,
+                   int n) {
+    cuuint64_t dims[2] = {(cuuint64_t)row_bytes, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
+    cuuint32_t box[2] = {(cuuint32_t)(16 * n), 128u};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, packed_swizzle(n), CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Per-group planning: operand kind, K-stages and exact accumulation segments.
 bool plan_group(const GroupGeom& G, Group& out) {
     out.bits_a = G.bits_a;
@@ -772,6 +926,9 @@ bool plan_group(const GroupGeom& G, Group& out) {
     out.w_offset = out.kind == 0 ? (1 << (G.bits_w - 1)) : 0;
     out.acc_scale = out.kind == 0 ? 262144.0f : 1.0f;   // 2^18
     out.inv_levels = (float)(1.0 / ((double)la * (double)(1 << (G.bits_w - 1))));
+    out.a_bytes = 128 * 16 * G.bits_a;
+    out.w_bytes = 128 * 16 * G.bits_w;
+    out.copy_bytes = 4;
     return true;
 }
 
@@ -822,18 +979,32 @@ cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st)
     p.g[1].chunk_base = geo.g[0].pw / 128;
     p.total_chunks = geo.g[0].pw / 128 + geo.g[1].pw / 128;
 
+    // Activation chunks come by TMA when every chunk of a plain GEMM row starts
+    // on a 16-byte boundary and holds data (128-code padding); else by gather.
+    bool a_tma = !a.conv && (geo.a_row_bytes % 16 == 0) && ((uintptr_t)a.Ap % 16 == 0);
+    for (int g = 0; g < 2; ++g) {
+        const GroupGeom& G = geo.g[g];
+        if (G.pw == 0) continue;
+        if (G.pa != G.pw || G.a_off % 16 != 0) a_tma = false;
+        // widest cp.async copy that keeps every block aligned
+        const int blk = 4 * G.bits_a;
+        for (int w = 16; w >= 4; w /= 2) {
+            if (blk % w == 0 && G.a_off % w == 0 && geo.a_row_bytes % w == 0 && (uintptr_t)a.Ap % w == 0) {
+                p.g[g].copy_bytes = w;
+                break;
+            }
+        }
+    }
+    p.a_tma = a_tma ? 1 : 0;
+
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;
     for (int g = 0; g < 2; ++g) {
-        const int box_x = 16 * (geo.g[g].pw > 0 ? geo.g[g].bits_w : 1);
-        cuuint64_t dims[2] = {(cuuint64_t)geo.w_row_bytes, (cuuint64_t)a.N};
-        cuuint64_t strides[1] = {(cuuint64_t)geo.w_row_bytes};
-        cuuint32_t box[2] = {(cuuint32_t)box_x, (cuuint32_t)BN};
-        cuuint32_t estr[2] = {1, 1};
-        CUresult r = enc(&p.tmw[g], CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(a.Wp), dims, strides, box,
-                         estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                         CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-        if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+        if (geo.g[g].pw == 0) continue;
+        if (!encode_packed(enc, &p.tmw[g], a.Wp, geo.w_row_bytes, a.N, geo.g[g].bits_w))
+            return cudaErrorInvalidValue;
+        if (a_tma && !encode_packed(enc, &p.tma[g], a.Ap, geo.a_row_bytes, a.M, geo.g[g].bits_a))
+            return cudaErrorInvalidValue;
     }
     static bool attr_done[64] = {};
     int dev = 0;
