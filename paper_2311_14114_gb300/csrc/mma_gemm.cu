@@ -31,15 +31,20 @@
 // TMA 32/64/128-byte swizzle so the converters read them without bank
 // conflicts.
 //
-// CTA = 128x128 output tile, 14 warps:
-//   warp 0      producer: ring space, TMA copies, cp.async gathers
-//   warp 1      MMA issuer (one thread) + TMEM owner
-//   warps 2-5   convert the 128 activation rows of each K-stage
-//   warps 6-9   convert the 128 weight rows
-//   warps 10-13 segment drains and the epilogue (tcgen05.ld -> fp32 -> fp16)
+// CTA = 128x128 output tile, 17 warps:
+//   warp 0      MMA issuer (one thread) + TMEM owner
+//   warps 1-4   producers: ring space and TMA copies (warp 1, lane 0); in
+//               gather mode every producer thread also copies one activation
+//               row of each chunk with cp.async
+//   warps 5-8   convert the 128 activation rows of each K-stage
+//   warps 9-12  convert the 128 weight rows
+//   warps 13-16 segment drains and the epilogue (tcgen05.ld -> fp32 -> fp16)
 // A K-stage is 128 bytes of MMA operand per row (128 E4M3 codes or 64 fp16
 // codes) in the 128-byte-swizzled K-major layout the MMA descriptors read;
 // an E4M3 chunk is one stage, an fp16 chunk two.
+//
+// Converters run one specialised loop per precision group (bit width and
+// operand kind fixed at compile time), so the inner loop has no dispatch.
 //
 // Every wait is bounded; a wait that runs out records an error bit in the
 // device error word, raises a CTA-wide abort flag and the CTA winds down
@@ -64,9 +69,10 @@ constexpr int OP_B_BYTES = BN * ROW_BYTES;           // 16 KB
 constexpr int OP_STAGE_BYTES = OP_A_BYTES + OP_B_BYTES;
 constexpr int PK_BYTES = 96 * 1024;                  // packed chunk ring
 constexpr int PK_SLOTS = 16;                         // chunks in flight at most
-constexpr int NUM_WARPS = 14;
+constexpr int NUM_WARPS = 17;
 constexpr int NUM_THREADS = NUM_WARPS * 32;
-constexpr int WARP_PROD = 0, WARP_MMA = 1, WARP_CVA = 2, WARP_CVW = 6, WARP_EPI = 10;
+constexpr int WARP_MMA = 0, WARP_PROD = 1, WARP_CVA = 5, WARP_CVW = 9, WARP_EPI = 13;
+constexpr int NUM_PROD_THREADS = 128;
 
 constexpr int SMEM_OP = 0;
 constexpr int SMEM_PK = SMEM_OP + OP_STAGES * OP_STAGE_BYTES;
@@ -233,40 +239,32 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-#define SONIQ_R32(r)                                                                                   \
-    "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),   \
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),      \
-        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),    \
-        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),    \
-        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-#define SONIQ_W32(r)                                                                                   \
-    "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), \
-        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), \
-        "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), \
-        "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
 
-// 32 consecutive TMEM columns of this thread's lane.  The load and its wait
-// sit in one asm statement: the destination registers are undefined until
-// tcgen05.wait::ld, so no instruction may read them in between.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+#define SONIQ_R16(r)                                                                                   \
+    "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),   \
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+#define SONIQ_W16(r)                                                                                   \
+    "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), \
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+
+// 16 consecutive TMEM columns of this thread's lane (load + wait in one statement).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
         "tcgen05.wait::ld.sync.aligned;"
-        : SONIQ_R32(r)
+        : SONIQ_R16(r)
         : "r"(taddr)
         : "memory");
 }
 
-// Likewise the store keeps reading its source registers until tcgen05.wait::st.
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
     asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
-        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n\t"
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n\t"
         "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
-        SONIQ_W32(r)
+        SONIQ_W16(r)
         : "memory");
 }
+
 
 // cp.async copies of 4, 8 or 16 bytes; src_bytes = 0 zero-fills the destination.
 __device__ __forceinline__ void cp_async(uint32_t dst, const void* src, int bytes, uint32_t src_bytes) {
@@ -283,13 +281,6 @@ __device__ __forceinline__ void cp_async_arrive(uint32_t bar) {
     asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
 }
 
-// XOR applied to the 16-byte chunk index of a packed row of n-bit codes
-// (16*n bytes per 128 codes): the TMA 32/64/128-byte swizzle for n = 2/4/8,
-// none otherwise.  Address bits [4, 4+k) are XORed with bits [7, 7+k).
-__device__ __forceinline__ uint32_t pk_xor(int n, uint32_t row) {
-    return (n == 2 || n == 4 || n == 8) ? ((row * (uint32_t)n) >> 3) & (uint32_t)(n - 1) : 0u;
-}
-
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
     uint4 v;
     asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
@@ -300,32 +291,20 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, ui
     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
+// XOR applied to the 16-byte chunk index of a packed row of n-bit codes
+// (16*n bytes per 128 codes): the TMA 32/64/128-byte swizzle for n = 2/4/8,
+// none otherwise.  Address bits [4, 4+k) are XORed with bits [7, 7+k).
+__device__ __forceinline__ uint32_t pk_xor(int n, uint32_t row) {
+    return (n == 2 || n == 4 || n == 8) ? ((row * (uint32_t)n) >> 3) & (uint32_t)(n - 1) : 0u;
+}
+
 // Byte offset of 16-byte chunk `chunk` of operand row `row` in the MMA tile
 // (128-byte swizzle: 8-row x 128-byte atoms).
 __device__ __forceinline__ uint32_t sw128_off(uint32_t row, uint32_t chunk) {
     return row * 128u + ((chunk ^ (row & 7u)) << 4);
 }
 
-// ---- stage and chunk bookkeeping --------------------------------------------
-
-struct StageInfo {
-    int g;       // group
-    int ls;      // stage index inside the group
-    int kind;
-    int half;    // fp16 stages: which half of the chunk
-    bool chunk_first, chunk_last;
-};
-
-__device__ __forceinline__ StageInfo stage_info(const Params& p, int s) {
-    StageInfo si;
-    si.g = s < p.g[0].n_stages ? 0 : 1;
-    si.ls = si.g ? s - p.g[0].n_stages : s;
-    si.kind = p.g[si.g].kind;
-    si.half = si.kind == 0 ? 0 : (si.ls & 1);
-    si.chunk_first = si.half == 0;
-    si.chunk_last = si.kind == 0 || si.half == 1;
-    return si;
-}
+// ---- chunk bookkeeping ---------------------------------------------------------
 
 __device__ __forceinline__ int chunk_group(const Params& p, int ci) { return ci < p.g[1].chunk_base ? 0 : 1; }
 
@@ -344,7 +323,7 @@ __device__ __forceinline__ uint32_t ring_next(const Params& p, int ci, uint32_t 
 
 // ---- conversion of packed codes into the MMA operand tile ---------------------
 
-// Reads this row's packed words of one chunk (n 16-byte pieces, swizzled).
+// This row's packed words of one chunk (n 16-byte pieces, swizzled).
 template <int N>
 __device__ __forceinline__ void read_chunk(uint32_t row_base, uint32_t xr, uint32_t* w) {
 #pragma unroll
@@ -401,110 +380,134 @@ __device__ __forceinline__ void cvt_f16(const uint32_t* w, int half, uint32_t ti
     }
 }
 
-// ---- activation gather (implicit GEMM / unaligned rows) -----------------------
-
-// Per-row state of the gather: output pixel coordinates of the 4 rows a lane owns.
-struct GatherRows {
-    int64_t base[4];   // GEMM: the row index m; conv: img * H (input row base)
-    int pp[4], qq[4];  // conv: output pixel coordinates
-    bool valid[4];
+struct CvtCtx {
+    uint32_t smem;        // shared-memory address of the aligned base
+    uint32_t pk_base;
+    uint32_t bar0;
+    volatile int* abort_flag;
+    int warp, lane;
+    uint32_t row;
+    int ci;               // next chunk
+    int s;                // next operand stage
+    uint32_t off;         // ring offset of chunk ci
 };
 
-// Issues the cp.async copies of chunk (g, c) for the 4 rows of this lane into
-// the ring slot at `slot` (swizzled like the TMA tiles).  Block kb of the
-// group's weight K range holds tap kb / cpt, channel block kb % cpt; taps
-// beyond R*S and pixels outside the image are zero-filled.
-__device__ __forceinline__ void gather_chunk(const Params& p, const GatherRows& gr, int lane, int g, int c,
-                                             uint32_t slot) {
+// Converts all chunks of group g for this row: per chunk, waits for its packed
+// slot, reads this row's words once, fills 1 (E4M3) or 2 (fp16) operand
+// stages, and hands the slot back only after its words are consumed.
+template <int N, int KIND, bool A_SIDE>
+__device__ __forceinline__ bool convert_group(const Params& p, CvtCtx& cx, int g, int32_t* rowsum_s) {
+    const Group& G = p.g[g];
+    const int nchunks = G.pw / 128;
+    const uint32_t xr = pk_xor(N, cx.row);
+    const uint32_t row_off = (A_SIDE ? 0u : (uint32_t)G.a_bytes) + cx.row * 16u * (uint32_t)N;
+    uint32_t rsum = 0;
+    for (int c = 0; c < nchunks; ++c) {
+        const int ci = cx.ci;
+        if (!__all_sync(0xffffffffu, wait_bounded(cx.bar0 + 8u * (BAR_PK_FULL + ci % PK_SLOTS),
+                                                    (ci / PK_SLOTS) & 1, cx.abort_flag, p)))
+            return false;
+        uint32_t w[4 * N];
+        read_chunk<N>(cx.pk_base + cx.off + row_off, xr, w);
+#pragma unroll
+        for (int h = 0; h < (KIND == 0 ? 1 : 2); ++h) {
+            const int s = cx.s;
+            const int slot = s % OP_STAGES;
+            if (!__all_sync(0xffffffffu, wait_bounded(cx.bar0 + 8u * (BAR_OP_EMPTY + slot),
+                                                        ((s / OP_STAGES) & 1) ^ 1, cx.abort_flag, p)))
+                return false;
+            const uint32_t tile = cx.smem + SMEM_OP + slot * OP_STAGE_BYTES + (A_SIDE ? 0 : OP_A_BYTES);
+            if constexpr (KIND == 0) rsum += cvt_e4m3<N, A_SIDE>(w, tile, cx.row);
+            else cvt_f16<N, A_SIDE>(w, h, tile, cx.row);
+            fence_proxy_async();
+            __syncwarp();
+            const bool drop = (p.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) && s == 0 && cx.warp == WARP_CVA;
+            if (cx.lane == 0 && !drop) mbar_arrive(cx.bar0 + 8u * (BAR_OP_FULL + slot));
+            cx.s = s + 1;
+        }
+        if (cx.lane == 0) mbar_arrive(cx.bar0 + 8u * (BAR_PK_EMPTY + ci % PK_SLOTS));
+        cx.off = ring_next(p, ci, cx.off);
+        cx.ci = ci + 1;
+    }
+    if (A_SIDE) rowsum_s[g * BM + cx.row] = (int32_t)rsum;
+    return true;
+}
+
+template <bool A_SIDE>
+__device__ __forceinline__ bool convert_group_n(const Params& p, CvtCtx& cx, int g, int32_t* rowsum_s) {
+    const Group& G = p.g[g];
+    const int n = A_SIDE ? G.bits_a : G.bits_w;
+    if (G.kind == 0) {
+        switch (n) {
+            case 1: return convert_group<1, 0, A_SIDE>(p, cx, g, rowsum_s);
+            case 2: return convert_group<2, 0, A_SIDE>(p, cx, g, rowsum_s);
+            case 3: return convert_group<3, 0, A_SIDE>(p, cx, g, rowsum_s);
+            default: return convert_group<4, 0, A_SIDE>(p, cx, g, rowsum_s);
+        }
+    }
+    switch (n) {
+        case 1: return convert_group<1, 1, A_SIDE>(p, cx, g, rowsum_s);
+        case 2: return convert_group<2, 1, A_SIDE>(p, cx, g, rowsum_s);
+        case 3: return convert_group<3, 1, A_SIDE>(p, cx, g, rowsum_s);
+        case 4: return convert_group<4, 1, A_SIDE>(p, cx, g, rowsum_s);
+        case 5: return convert_group<5, 1, A_SIDE>(p, cx, g, rowsum_s);
+        case 6: return convert_group<6, 1, A_SIDE>(p, cx, g, rowsum_s);
+        case 7: return convert_group<7, 1, A_SIDE>(p, cx, g, rowsum_s);
+        default: return convert_group<8, 1, A_SIDE>(p, cx, g, rowsum_s);
+    }
+}
+
+// ---- activation gather (implicit GEMM / unaligned rows) -----------------------
+
+// One producer thread copies one activation row of each chunk.  Block kb of a
+// group's weight K range holds tap kb / cpt and channel block kb % cpt; the
+// thread walks blocks in order, so tap, channel block and the tap's filter
+// offsets advance by counting instead of division.
+struct Gather {
+    int64_t base;      // GEMM: row m; conv: img * H
+    int pp, qq;        // conv: output pixel
+    bool valid;        // row < M
+    int tap, cb, r, s; // position of the next block in its group
+};
+
+__device__ __forceinline__ void gather_chunk(const Params& p, Gather& gt, uint32_t row, int g, uint32_t slot) {
     const Group& G = p.g[g];
     const int n = G.bits_a;
     const int cpt = G.pa >> 5;
     const int taps = p.conv ? p.R * p.S : 1;
     const int bw = G.copy_bytes;
-    const int blk_bytes = 4 * n;
-    const int row_bytes = 16 * n;
-#pragma unroll
+    const int blk = 4 * n;
+    const uint32_t xr = pk_xor(n, row);
+    const uint32_t dst_row = slot + row * 16u * (uint32_t)n;
+#pragma unroll 1
     for (int i = 0; i < 4; ++i) {
-        const int kb = 4 * c + i;
-        const int tap = cpt > 0 ? kb / cpt : taps;
-        const int cb = kb - tap * cpt;
-        const int r = tap / p.S, s = tap - r * p.S;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const uint32_t row = (uint32_t)(lane + 32 * k);
-            const uint8_t* src = p.Ap;   // any valid address when zero-filling
-            uint32_t nbytes = 0;
-            if (gr.valid[k] && tap < taps) {
-                if (!p.conv) {
-                    src = p.Ap + gr.base[k] * p.a_row_bytes + G.a_off + cb * blk_bytes;
+        const uint8_t* src = p.Ap;   // any valid address when zero-filling
+        uint32_t nbytes = 0;
+        if (gt.valid && gt.tap < taps) {
+            if (!p.conv) {
+                src = p.Ap + gt.base * p.a_row_bytes + G.a_off + gt.cb * blk;
+                nbytes = (uint32_t)bw;
+            } else {
+                const int h = gt.pp * p.sh - p.ph + gt.r, w = gt.qq * p.sw - p.pw + gt.s;
+                if (h >= 0 && h < p.H && w >= 0 && w < p.W) {
+                    src = p.Ap + ((gt.base + h) * p.W + w) * p.a_row_bytes + G.a_off + gt.cb * blk;
                     nbytes = (uint32_t)bw;
-                } else {
-                    const int h = gr.pp[k] * p.sh - p.ph + r, w = gr.qq[k] * p.sw - p.pw + s;
-                    if (h >= 0 && h < p.H && w >= 0 && w < p.W) {
-                        src = p.Ap + ((gr.base[k] + h) * p.W + w) * p.a_row_bytes + G.a_off + cb * blk_bytes;
-                        nbytes = (uint32_t)bw;
-                    }
                 }
             }
-            const uint32_t xr = pk_xor(n, row);
-            for (int b = 0; b < blk_bytes; b += bw) {
-                const int byte = i * blk_bytes + b;   // within the row's 16*n bytes
-                const uint32_t dst = slot + row * row_bytes + ((((uint32_t)byte >> 4) ^ xr) << 4) + (byte & 15);
-                cp_async(dst, nbytes ? (const void*)(src + b) : (const void*)p.Ap, bw, nbytes);
+        }
+        for (int b = 0; b < blk; b += bw) {
+            const int byte = i * blk + b;
+            const uint32_t dst = dst_row + ((((uint32_t)byte >> 4) ^ xr) << 4) + (uint32_t)(byte & 15);
+            cp_async(dst, nbytes ? (const void*)(src + b) : (const void*)p.Ap, bw, nbytes);
+        }
+        if (++gt.cb == cpt) {
+            gt.cb = 0;
+            ++gt.tap;
+            if (++gt.s == p.S) {
+                gt.s = 0;
+                ++gt.r;
             }
         }
-    }
-}
-
-// ---- converter: one packed chunk of one row -> one or two MMA stages ---------------
-
-struct CvtCtx {
-    uint32_t smem;        // shared-memory address of the aligned base
-    uint32_t bar0;
-    volatile int* abort_flag;
-    int warp, lane;
-    uint32_t row;
-};
-
-// Waits for each operand stage of chunk ci (1 for E4M3, 2 for fp16), converts
-// this row into it and signals the MMA.  Returns false when the CTA aborts.
-template <int N, bool A_SIDE>
-__device__ __forceinline__ bool convert_chunk(const Params& p, const CvtCtx& cx, uint32_t row_base, int s0,
-                                              int nst, int kind, uint32_t& rsum) {
-    uint32_t w[4 * N];
-    read_chunk<N>(row_base, pk_xor(N, cx.row), w);
-    for (int h = 0; h < nst; ++h) {
-        const int s = s0 + h;
-        const int slot = s % OP_STAGES;
-        if (!__all_sync(0xffffffffu, wait_bounded(cx.bar0 + 8u * (BAR_OP_EMPTY + slot), ((s / OP_STAGES) & 1) ^ 1,
-                                                    cx.abort_flag, p)))
-            return false;
-        const uint32_t tile = cx.smem + SMEM_OP + slot * OP_STAGE_BYTES + (A_SIDE ? 0 : OP_A_BYTES);
-        if (kind == 0) {
-            if constexpr (N <= 4) rsum += cvt_e4m3<N, A_SIDE>(w, tile, cx.row);
-        } else {
-            cvt_f16<N, A_SIDE>(w, h, tile, cx.row);
-        }
-        fence_proxy_async();
-        __syncwarp();
-        const bool drop = (p.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) && s == 0 && cx.warp == WARP_CVA;
-        if (cx.lane == 0 && !drop) mbar_arrive(cx.bar0 + 8u * (BAR_OP_FULL + slot));
-    }
-    return true;
-}
-
-template <bool A_SIDE>
-__device__ __forceinline__ bool convert_chunk_n(int n, const Params& p, const CvtCtx& cx, uint32_t row_base,
-                                                int s0, int nst, int kind, uint32_t& rsum) {
-    switch (n) {
-        case 1: return convert_chunk<1, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
-        case 2: return convert_chunk<2, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
-        case 3: return convert_chunk<3, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
-        case 4: return convert_chunk<4, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
-        case 5: return convert_chunk<5, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
-        case 6: return convert_chunk<6, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
-        case 7: return convert_chunk<7, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
-        default: return convert_chunk<8, A_SIDE>(p, cx, row_base, s0, nst, kind, rsum);
     }
 }
 
@@ -517,7 +520,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
     const int64_t m0 = (int64_t)blockIdx.y * BM;
     const int n0 = blockIdx.x * BN;
 
-    uint32_t bar0 = smem_u32(smem + SMEM_BAR);
+    const uint32_t bar0 = smem_u32(smem + SMEM_BAR);
     auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + SMEM_MISC);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + SMEM_MISC + 4);
@@ -527,8 +530,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < PK_SLOTS; ++i) {
-            // TMA arrival (+ the 32 gather lanes of the producer warp)
-            mbar_init(bar(BAR_PK_FULL + i), p.a_tma ? 1 : 33);
+            // the TMA arrival, plus one cp.async arrival per producer thread when gathering
+            mbar_init(bar(BAR_PK_FULL + i), p.a_tma ? 1 : 1 + NUM_PROD_THREADS);
             mbar_init(bar(BAR_PK_EMPTY + i), 8);
         }
         for (int i = 0; i < OP_STAGES; ++i) {
@@ -564,95 +567,95 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    if (warp == WARP_PROD) {
-        // ------------------------------------------------------------- producer
-        GatherRows gr;
-        if (!p.a_tma) {
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int64_t m = m0 + lane + 32 * k;
-                gr.valid[k] = m < p.M;
-                gr.base[k] = m;
-                gr.pp[k] = gr.qq[k] = 0;
-                if (p.conv && gr.valid[k]) {
-                    const int64_t pq = (int64_t)p.P * p.Q;
-                    const int64_t img = m / pq;
-                    const int rem = (int)(m - img * pq);
-                    gr.pp[k] = rem / p.Q;
-                    gr.qq[k] = rem - gr.pp[k] * p.Q;
-                    gr.base[k] = img * p.H;
+    if (warp >= WARP_PROD && warp < WARP_CVA) {
+        // ------------------------------------------------------------ producers
+        const uint32_t prow = threadIdx.x - WARP_PROD * 32;     // activation row this thread gathers
+        const bool lead = prow == 0;                           // issues the TMA copies
+        if (p.a_tma && warp != WARP_PROD) goto done;           // TMA brings both operands
+        {
+            Gather gt;
+            gt.valid = m0 + prow < p.M;
+            gt.base = m0 + prow;
+            gt.pp = gt.qq = 0;
+            if (p.conv && gt.valid) {
+                const int64_t pq = (int64_t)p.P * p.Q;
+                const int64_t img = (m0 + prow) / pq;
+                const int rem = (int)(m0 + prow - img * pq);
+                gt.pp = rem / p.Q;
+                gt.qq = rem - gt.pp * p.Q;
+                gt.base = img * p.H;
+            }
+            // Ring bookkeeping (identical in every producer thread): chunks
+            // rel..ci-1 are in flight; `tail` is the offset of chunk rel, `off`
+            // that of chunk ci and `head` the end of chunk ci-1.
+            int rel = 0, issued = 0;
+            uint32_t off = 0, tail = 0, head = 0;
+            bool ok = true;
+            for (int ci = 0; ci < p.total_chunks && ok; ++ci) {
+                const int g = chunk_group(p, ci);
+                const Group& G = p.g[g];
+                const int c = ci - G.chunk_base;
+                if (c == 0) gt.tap = gt.cb = gt.r = gt.s = 0;
+                const uint32_t sz = (uint32_t)(G.a_bytes + G.w_bytes);
+                const int b = ci % PK_SLOTS;
+                while (rel < ci) {
+                    // is [off, off + sz) clear of the chunks in flight, and is a barrier pair free?
+                    bool fits;
+                    if (ci - rel >= PK_SLOTS) fits = false;
+                    else if (off == head) fits = head > tail || head + sz <= tail;   // tail == head: ring full
+                    else fits = head > tail && sz <= tail;                           // wrapped to offset 0
+                    if (fits) break;
+                    if (!wait_bounded(bar(BAR_PK_EMPTY + rel % PK_SLOTS), (rel / PK_SLOTS) & 1, abort_flag, p)) {
+                        ok = false;
+                        break;
+                    }
+                    tail = ring_next(p, rel, tail);
+                    ++rel;
+                }
+                if (!ok) break;
+                const uint32_t slot = pk_base + off;
+                if (lead) {
+                    mbar_arrive_expect_tx(bar(BAR_PK_FULL + b), (uint32_t)(G.w_bytes + (p.a_tma ? G.a_bytes : 0)));
+                    tma_load_2d(slot + G.a_bytes, &p.tmw[g], G.w_off + c * 16 * G.bits_w, n0, bar(BAR_PK_FULL + b));
+                    if (p.a_tma)
+                        tma_load_2d(slot, &p.tma[g], G.a_off + c * 16 * G.bits_a, (int)m0, bar(BAR_PK_FULL + b));
+                }
+                if (!p.a_tma) {
+                    gather_chunk(p, gt, prow, g, slot);
+                    cp_async_arrive(bar(BAR_PK_FULL + b));
+                }
+                head = off + sz;
+                off = ring_next(p, ci, off);
+                ++issued;
+            }
+            // copies still in flight must land before the CTA's memory is released
+            if (lead) {
+                for (int ci = issued - PK_SLOTS < 0 ? 0 : issued - PK_SLOTS; ci < issued; ++ci) {
+                    volatile int no_abort = 0;
+                    wait_bounded(bar(BAR_PK_FULL + ci % PK_SLOTS), (ci / PK_SLOTS) & 1, &no_abort, p);
                 }
             }
+            asm volatile("cp.async.wait_all;" ::: "memory");
         }
-        // Ring bookkeeping (identical on all lanes): chunks rel..ci-1 are in
-        // flight; `tail` is the offset of chunk rel, `off` that of chunk ci and
-        // `head` the end of chunk ci-1 before the wrap decision.
-        int rel = 0;
-        int issued = 0;
-        uint32_t off = 0, tail = 0, head = 0;
-        bool ok = true;
-        for (int ci = 0; ci < p.total_chunks && ok; ++ci) {
-            const int g = chunk_group(p, ci);
-            const Group& G = p.g[g];
-            const int c = ci - G.chunk_base;
-            const uint32_t sz = (uint32_t)(G.a_bytes + G.w_bytes);
-            const int b = ci % PK_SLOTS;
-            while (rel < ci) {
-                // is [off, off + sz) clear of the chunks in flight, and is a barrier pair free?
-                bool fits;
-                if (ci - rel >= PK_SLOTS) fits = false;
-                else if (off == head) fits = head > tail || head + sz <= tail;   // tail == head: ring full
-                else fits = head > tail && sz <= tail;                           // wrapped to offset 0
-                if (fits) break;
-                if (!__all_sync(0xffffffffu,
-                                wait_bounded(bar(BAR_PK_EMPTY + rel % PK_SLOTS), (rel / PK_SLOTS) & 1, abort_flag, p))) {
-                    ok = false;
-                    break;
-                }
-                tail = ring_next(p, rel, tail);
-                ++rel;
-            }
-            if (!ok) break;
-            const uint32_t slot = pk_base + off;
-            if (lane == 0) {
-                mbar_arrive_expect_tx(bar(BAR_PK_FULL + b), (uint32_t)(G.w_bytes + (p.a_tma ? G.a_bytes : 0)));
-                tma_load_2d(slot + G.a_bytes, &p.tmw[g], G.w_off + c * 16 * G.bits_w, n0, bar(BAR_PK_FULL + b));
-                if (p.a_tma)
-                    tma_load_2d(slot, &p.tma[g], G.a_off + c * 16 * G.bits_a, (int)m0, bar(BAR_PK_FULL + b));
-            }
-            if (!p.a_tma) {
-                gather_chunk(p, gr, lane, g, c, slot);
-                cp_async_arrive(bar(BAR_PK_FULL + b));
-            }
-            head = off + sz;
-            off = ring_next(p, ci, off);
-            ++issued;
-        }
-        // copies still in flight must land before the CTA's memory is released
-        if (lane == 0) {
-            for (int ci = issued - PK_SLOTS < 0 ? 0 : issued - PK_SLOTS; ci < issued; ++ci) {
-                volatile int no_abort = 0;
-                wait_bounded(bar(BAR_PK_FULL + ci % PK_SLOTS), (ci / PK_SLOTS) & 1, &no_abort, p);
-            }
-        }
-        asm volatile("cp.async.wait_all;" ::: "memory");
+    done:;
     } else if (warp == WARP_MMA) {
         // ------------------------------------------------------------------ MMA
         if (lane == 0) {
             bool ok = true;
             for (int s = 0; s < p.total_stages && ok; ++s) {
-                const StageInfo si = stage_info(p, s);
-                const Group& G = p.g[si.g];
+                const int g = s < p.g[0].n_stages ? 0 : 1;
+                const Group& G = p.g[g];
+                const int ls = g ? s - p.g[0].n_stages : s;
                 const int slot = s % OP_STAGES;
                 uint32_t col;
                 bool first;
                 bool seg_end = false;
                 int seg = 0;
-                if (si.g == p.seg_group) {
-                    seg = si.ls / G.seg_stages;
-                    const int in_seg = si.ls - seg * G.seg_stages;
+                if (g == p.seg_group) {
+                    seg = ls / G.seg_stages;
+                    const int in_seg = ls - seg * G.seg_stages;
                     first = in_seg == 0;
-                    seg_end = in_seg == G.seg_stages - 1 || si.ls == G.n_stages - 1;
+                    seg_end = in_seg == G.seg_stages - 1 || ls == G.n_stages - 1;
                     col = (uint32_t)(BN + (seg & 1) * BN);
                     if (first && seg >= 2) {
                         if (!wait_bounded(bar(BAR_SLOT_FREE + (seg & 1)), ((seg >> 1) - 1) & 1, abort_flag, p)) {
@@ -662,8 +665,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                         tc_fence_after();
                     }
                 } else {
-                    first = si.ls == 0;
-                    col = (uint32_t)p.acc_col[si.g];
+                    first = ls == 0;
+                    col = (uint32_t)p.acc_col[g];
                 }
                 if (!wait_bounded(bar(BAR_OP_FULL + slot), (s / OP_STAGES) & 1, abort_flag, p)) {
                     ok = false;
@@ -676,7 +679,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                 for (int k = 0; k < 4; ++k) {
                     const uint64_t ad = sw128_desc(a_addr + 32 * k), bd = sw128_desc(b_addr + 32 * k);
                     const uint32_t acc = (first && k == 0) ? 0u : 1u;
-                    if (si.kind == 0) mma_f8(tmem_base + col, ad, bd, acc);
+                    if (G.kind == 0) mma_f8(tmem_base + col, ad, bd, acc);
                     else mma_f16(tmem_base + col, ad, bd, acc);
                 }
                 mma_commit(bar(BAR_OP_EMPTY + slot));
@@ -691,36 +694,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
     } else if (warp < WARP_EPI) {
         // ----------------------------------------------------------- converters
         const bool a_side = warp < WARP_CVW;
-        CvtCtx cx{smem_u32(smem), bar0, abort_flag, warp, lane,
-                  (uint32_t)(threadIdx.x - (a_side ? WARP_CVA : WARP_CVW) * 32)};
-        uint32_t rsum = 0;
-        uint32_t off = 0;
-        int s0 = 0;
-        for (int ci = 0; ci < p.total_chunks; ++ci) {
-            const int g = chunk_group(p, ci);
-            const Group& G = p.g[g];
-            const int nst = G.kind == 0 ? 1 : 2;
-            if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_PK_FULL + ci % PK_SLOTS), (ci / PK_SLOTS) & 1,
-                                                        abort_flag, p)))
-                break;
-            bool ok;
-            if (a_side) {
-                const uint32_t rb = pk_base + off + cx.row * 16u * (uint32_t)G.bits_a;
-                ok = convert_chunk_n<true>(G.bits_a, p, cx, rb, s0, nst, G.kind, rsum);
-                if (ci == G.chunk_base + G.pw / 128 - 1) {   // last chunk of the group
-                    rowsum_s[g * BM + cx.row] = (int32_t)rsum;
-                    rsum = 0;
-                }
-            } else {
-                const uint32_t rb = pk_base + off + G.a_bytes + cx.row * 16u * (uint32_t)G.bits_w;
-                uint32_t unused = 0;
-                ok = convert_chunk_n<false>(G.bits_w, p, cx, rb, s0, nst, G.kind, unused);
-            }
+        CvtCtx cx{smem_u32(smem), pk_base, bar0, abort_flag, warp, lane,
+                  (uint32_t)(threadIdx.x - (a_side ? WARP_CVA : WARP_CVW) * 32), 0, 0, 0u};
+        for (int g = 0; g < 2; ++g) {
+            if (p.g[g].pw == 0) continue;
+            const bool ok = a_side ? convert_group_n<true>(p, cx, g, rowsum_s)
+                                   : convert_group_n<false>(p, cx, g, rowsum_s);
             if (!ok) break;
-            // the slot goes back to the producer only after its words are consumed
-            if (lane == 0) mbar_arrive(bar(BAR_PK_EMPTY + ci % PK_SLOTS));
-            off = ring_next(p, ci, off);
-            s0 += nst;
         }
         if (a_side) {
             __syncwarp();
@@ -743,16 +723,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                 tc_fence_after();
                 const uint32_t ring_col = BN + (i & 1) * BN;
 #pragma unroll 1
-                for (int cc = 0; cc < BN / 32; ++cc) {
-                    uint32_t v[32], s[32];
-                    tmem_ld32(lane_base + ring_col + cc * 32, v);
-                    if (i > 0) tmem_ld32(lane_base + sum_col + cc * 32, s);
+                for (int cc = 0; cc < BN / 16; ++cc) {
+                    uint32_t v[16], s[16];
+                    tmem_ld16(lane_base + ring_col + cc * 16, v);
+                    if (i > 0) tmem_ld16(lane_base + sum_col + cc * 16, s);
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
+                    for (int j = 0; j < 16; ++j) {
                         const int32_t x = __float2int_rn(__uint_as_float(v[j]) * p.g[gs].acc_scale);
                         s[j] = (uint32_t)((i > 0 ? (int32_t)s[j] : 0) + x);
                     }
-                    tmem_st32(lane_base + sum_col + cc * 32, s);
+                    tmem_st16(lane_base + sum_col + cc * 16, s);
                 }
                 tc_fence_before();
                 __syncwarp();
@@ -773,76 +753,77 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
 #pragma unroll
             for (int g = 0; g < 2; ++g) corr[g] = p.g[g].w_offset * rowsum_s[g * BM + row];
 #pragma unroll 1
-            for (int cc = 0; cc < BN / 32; ++cc) {
-                int32_t acc[2][32];
+            for (int cc = 0; cc < BN / 16; ++cc) {
+                int32_t acc[2][16];
 #pragma unroll
                 for (int g = 0; g < 2; ++g) {
-                    uint32_t v[32];
+                    uint32_t v[16];
                     if (p.g[g].n_stages == 0) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) acc[g][j] = 0;
+                        for (int j = 0; j < 16; ++j) acc[g][j] = 0;
                         continue;
                     }
                     if (g == gs) {
-                        tmem_ld32(lane_base + 3 * BN + cc * 32, v);
+                        tmem_ld16(lane_base + 3 * BN + cc * 16, v);
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) acc[g][j] = (int32_t)v[j] - corr[g];
+                        for (int j = 0; j < 16; ++j) acc[g][j] = (int32_t)v[j] - corr[g];
                     } else {
-                        tmem_ld32(lane_base + p.acc_col[g] + cc * 32, v);
+                        tmem_ld16(lane_base + p.acc_col[g] + cc * 16, v);
 #pragma unroll
-                        for (int j = 0; j < 32; ++j)
+                        for (int j = 0; j < 16; ++j)
                             acc[g][j] = __float2int_rn(__uint_as_float(v[j]) * p.g[g].acc_scale) - corr[g];
                     }
                 }
-                const int nb = n0 + cc * 32;
+                const int nb = n0 + cc * 16;
                 if (m < p.M) {
                     if (p.acc_dbg != nullptr) {
 #pragma unroll
                         for (int g = 0; g < 2; ++g) {
                             int32_t* dst = p.acc_dbg + ((int64_t)g * p.M + m) * p.N;
 #pragma unroll
-                            for (int j = 0; j < 32; ++j)
+                            for (int j = 0; j < 16; ++j)
                                 if (nb + j < p.N) dst[nb + j] = acc[g][j];
                         }
                     }
-                    float y[32];
+                    float y[16];
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int c = cc * 32 + j;
+                    for (int j = 0; j < 16; ++j) {
+                        const int c = cc * 16 + j;
                         y[j] = fmaf(sa[1] * sw_s[BN + c], (float)acc[1][j], sa[0] * sw_s[c] * (float)acc[0][j]);
                     }
+                    const bool vec = nb + 16 <= p.N && (p.N & 7) == 0;
                     if (p.out_bf16) {
                         __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.Y) + m * p.N;
-                        if (nb + 32 <= p.N && (p.N & 7) == 0) {
+                        if (vec) {
 #pragma unroll
-                            for (int v8 = 0; v8 < 4; ++v8) {
-                                uint32_t w[4];
+                            for (int v8 = 0; v8 < 2; ++v8) {
+                                uint32_t wv[4];
 #pragma unroll
                                 for (int e = 0; e < 4; ++e) {
-                                    __nv_bfloat162 h = __floats2bfloat162_rn(y[v8 * 8 + 2 * e], y[v8 * 8 + 2 * e + 1]);
-                                    w[e] = *reinterpret_cast<uint32_t*>(&h);
+                                    __nv_bfloat162 h2 = __floats2bfloat162_rn(y[v8 * 8 + 2 * e], y[v8 * 8 + 2 * e + 1]);
+                                    wv[e] = *reinterpret_cast<uint32_t*>(&h2);
                                 }
-                                *reinterpret_cast<uint4*>(dst + nb + v8 * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+                                *reinterpret_cast<uint4*>(dst + nb + v8 * 8) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
                             }
                         } else {
-                            for (int j = 0; j < 32; ++j)
+                            for (int j = 0; j < 16; ++j)
                                 if (nb + j < p.N) dst[nb + j] = __float2bfloat16_rn(y[j]);
                         }
                     } else {
                         __half* dst = reinterpret_cast<__half*>(p.Y) + m * p.N;
-                        if (nb + 32 <= p.N && (p.N & 7) == 0) {
+                        if (vec) {
 #pragma unroll
-                            for (int v8 = 0; v8 < 4; ++v8) {
-                                uint32_t w[4];
+                            for (int v8 = 0; v8 < 2; ++v8) {
+                                uint32_t wv[4];
 #pragma unroll
                                 for (int e = 0; e < 4; ++e) {
-                                    __half2 h = __floats2half2_rn(y[v8 * 8 + 2 * e], y[v8 * 8 + 2 * e + 1]);
-                                    w[e] = *reinterpret_cast<uint32_t*>(&h);
+                                    __half2 h2 = __floats2half2_rn(y[v8 * 8 + 2 * e], y[v8 * 8 + 2 * e + 1]);
+                                    wv[e] = *reinterpret_cast<uint32_t*>(&h2);
                                 }
-                                *reinterpret_cast<uint4*>(dst + nb + v8 * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+                                *reinterpret_cast<uint4*>(dst + nb + v8 * 8) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
                             }
                         } else {
-                            for (int j = 0; j < 32; ++j)
+                            for (int j = 0; j < 16; ++j)
                                 if (nb + j < p.N) dst[nb + j] = __float2half_rn(y[j]);
                         }
                     }
@@ -850,7 +831,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
             }
         }
     }
-
 
     tc_fence_before();
     __syncthreads();
@@ -958,7 +938,9 @@ cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st)
     p.N = a.N;
     p.a_row_bytes = geo.a_row_bytes;
     p.conv = a.conv;
-    p.H = a.H; p.W = a.W; p.P = a.P; p.Q = a.Q; p.R = a.R; p.S = a.S;
+    p.H = a.H; p.W = a.W; p.P = a.P; p.Q = a.Q;
+    p.R = a.conv ? a.R : 1;
+    p.S = a.conv ? a.S : 1;
     p.sh = a.sh; p.sw = a.sw; p.ph = a.ph; p.pw = a.pw;
     p.s_a_per_row = a.s_a_per_row;
     p.out_bf16 = a.out_bf16;
