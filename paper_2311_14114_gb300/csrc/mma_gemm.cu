@@ -14,7 +14,10 @@
 //     binade), so activations need no conversion at all; weights are made
 //     unsigned by flipping the sign bit (j + 2^(n-1)) and the epilogue
 //     subtracts 2^(n-1) * R_g[m] with R_g the activation row sums;
-//   * wider groups use kind::f16 with fp16 operands (exact for |x| <= 2048).
+//   * wider groups use kind::f16 with fp16 operands (exact for |x| <= 2048);
+//     activations are centred (u - 2^(n-1)), which halves the worst-case
+//     product, and the epilogue adds back 2^(n-1) * C_g[n] with C_g the
+//     weight column sums.
 // Products accumulate in fp32 TMEM.  A partial sum is an exact integer while
 // its magnitude stays <= 2^24; the host splits a group's K range into
 // segments short enough for the worst case, and the epilogue warps drain each
@@ -69,6 +72,7 @@ constexpr int OP_B_BYTES = BN * ROW_BYTES;           // 16 KB
 constexpr int OP_STAGE_BYTES = OP_A_BYTES + OP_B_BYTES;
 constexpr int PK_BYTES = 96 * 1024;                  // packed chunk ring
 constexpr int PK_SLOTS = 16;                         // chunks in flight at most
+constexpr int A_TMEM_COL = 256;                      // activation stages in TMEM (32 columns each)
 constexpr int NUM_WARPS = 17;
 constexpr int NUM_THREADS = NUM_WARPS * 32;
 constexpr int WARP_MMA = 0, WARP_PROD = 1, WARP_CVA = 5, WARP_CVW = 9, WARP_EPI = 13;
@@ -80,10 +84,11 @@ constexpr int SMEM_BAR = SMEM_PK + PK_BYTES;
 constexpr int BAR_PK_FULL = 0, BAR_PK_EMPTY = 16, BAR_OP_FULL = 32, BAR_OP_EMPTY = 35,
               BAR_SEG_FULL = 38, BAR_SLOT_FREE = 40, BAR_ACC_FULL = 42, BAR_ROWSUM = 43,
               BAR_TEARDOWN = 44, NUM_BARS = 45;
-constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;         // tmem base, abort flag
+constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;         // tmem base, abort flag, a zero word
 constexpr int SMEM_ROWSUM = (SMEM_MISC + 16 + 15) & ~15;   // int32 [2][128]
 constexpr int SMEM_SW = SMEM_ROWSUM + 2 * BM * 4;          // fp32 [2][128]
-constexpr int SMEM_TOTAL = SMEM_SW + 2 * BN * 4;
+constexpr int SMEM_CS = SMEM_SW + 2 * BN * 4;              // int32 [2][128] weight column sums
+constexpr int SMEM_TOTAL = SMEM_CS + 2 * BN * 4;
 constexpr int SMEM_ALLOC = SMEM_TOTAL + 1024;              // slack for 1024-byte alignment
 
 struct Group {
@@ -95,7 +100,8 @@ struct Group {
     int32_t n_stages;      // K-stages
     int32_t seg_stages;    // K-stages per exact accumulation segment
     int32_t n_seg;
-    int32_t w_offset;      // 2^(nw-1) for kind 0, else 0
+    int32_t w_offset;      // kind 0: weights carry +2^(nw-1) (offset binary), else 0
+    int32_t a_offset;      // kind 1: activations carry -2^(na-1) (centred), else 0
     int32_t chunk_base;    // index of the group's first 128-code chunk
     int32_t a_bytes;       // packed activation bytes of one chunk (128 rows)
     int32_t w_bytes;       // packed weight bytes of one chunk (128 rows)
@@ -125,6 +131,7 @@ struct Params {
     uint32_t flags;
     int32_t seg_group;     // group accumulated in drained segments, or -1
     int32_t tmem_cols;     // 256 or 512
+    int32_t a_in_tmem;     // 1: activation stages live in TMEM columns A_TMEM_COL.. (no segments)
     int32_t acc_col[2];    // TMEM column of each group's accumulator (non-segmented)
     int32_t total_stages;
     int32_t total_chunks;
@@ -169,19 +176,38 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait: gives up when the CTA is aborting or after timeout_ns; on a
-// timeout it records the error and raises the abort flag.
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+// The CTA-wide abort flag lives in shared memory; it is read and written
+// with explicit shared-space volatile accesses.
+__device__ __forceinline__ int abort_raised(uint32_t flag) {
+    int v;
+    asm volatile("ld.volatile.shared.u32 %0, [%1];" : "=r"(v) : "r"(flag) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void raise_abort(uint32_t flag) {
+    asm volatile("st.volatile.shared.u32 [%0], %1;" ::"r"(flag), "r"(1) : "memory");
+}
+
+// Bounded wait: polls the barrier tightly and only every 64 polls looks at the
+// abort flag and the clock, so a completed phase is seen within one poll.
+// Gives up when the CTA is aborting or after timeout_ns; on a timeout it
+// records the error and raises the abort flag.
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint32_t abort_flag,
                                              const Params& p) {
     if (mbar_try_wait(bar, parity)) return true;
-    const long long t0 = globaltimer();
-    while (true) {
+    long long t0 = 0;
+    for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (globaltimer() - t0 > p.timeout_ns) {
-            *abort_flag = 1;
-            atomicOr(p.err, 1u);
-            return false;
+        if ((it & 63u) == 0u) {
+            if (abort_raised(abort_flag)) return false;
+            const long long t = globaltimer();
+            if (t0 == 0) {
+                t0 = t;
+            } else if (t - t0 > p.timeout_ns) {
+                raise_abort(abort_flag);
+                atomicOr(p.err, 1u);
+                return false;
+            }
         }
     }
 }
@@ -225,6 +251,21 @@ __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t a, uint64_t b,
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(a), "l"(b), "r"(IDESC), "r"(acc));
+}
+
+// A operand from TMEM (columns of this stage), B from shared memory.
+__device__ __forceinline__ void mma_f8_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(IDESC), "r"(acc));
+}
+
+__device__ __forceinline__ void mma_f16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(IDESC), "r"(acc));
 }
 
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
@@ -306,18 +347,30 @@ __device__ __forceinline__ uint32_t sw128_off(uint32_t row, uint32_t chunk) {
 
 // ---- chunk bookkeeping ---------------------------------------------------------
 
-__device__ __forceinline__ int chunk_group(const Params& p, int ci) { return ci < p.g[1].chunk_base ? 0 : 1; }
+// Chunk sizes of the packed ring, held in registers (hot loops never index the
+// parameter block with a runtime value).
+struct RingGeo {
+    int n0;              // chunks of group 0
+    int total;           // chunks of both groups
+    uint32_t sz0, sz1;   // slot bytes of a chunk of group 0 / group 1
+};
 
-__device__ __forceinline__ uint32_t chunk_size(const Params& p, int ci) {
-    const Group& G = p.g[chunk_group(p, ci)];
-    return (uint32_t)(G.a_bytes + G.w_bytes);
+__device__ __forceinline__ RingGeo ring_geo(const Params& p) {
+    RingGeo r;
+    r.n0 = p.g[1].chunk_base;
+    r.total = p.total_chunks;
+    r.sz0 = (uint32_t)(p.g[0].a_bytes + p.g[0].w_bytes);
+    r.sz1 = (uint32_t)(p.g[1].a_bytes + p.g[1].w_bytes);
+    return r;
 }
+
+__device__ __forceinline__ uint32_t chunk_size(const RingGeo& r, int ci) { return ci < r.n0 ? r.sz0 : r.sz1; }
 
 // Ring offset of chunk ci+1 from that of chunk ci: slots follow each other and
 // wrap to 0 when the next one would not fit.
-__device__ __forceinline__ uint32_t ring_next(const Params& p, int ci, uint32_t off) {
-    uint32_t nxt = off + chunk_size(p, ci);
-    if (ci + 1 < p.total_chunks && nxt + chunk_size(p, ci + 1) > (uint32_t)PK_BYTES) nxt = 0;
+__device__ __forceinline__ uint32_t ring_next(const RingGeo& r, int ci, uint32_t off) {
+    uint32_t nxt = off + chunk_size(r, ci);
+    if (ci + 1 < r.total && nxt + chunk_size(r, ci + 1) > (uint32_t)PK_BYTES) nxt = 0;
     return nxt;
 }
 
@@ -338,53 +391,76 @@ __device__ __forceinline__ void read_chunk(uint32_t row_base, uint32_t xr, uint3
 
 // E4M3 stage: 4 blocks of 32 codes -> 128 bytes.  Activations: the byte is the
 // code; weights: sign bit flipped (offset binary).  Returns the code sum.
+// Conversions write one stage row (128 bytes) as 32 words `out`, natural K
+// order: 16-byte piece c of the row is out[4c .. 4c+3].
 template <int N, bool A_SIDE>
-__device__ __forceinline__ uint32_t cvt_e4m3(const uint32_t* w, uint32_t tile, uint32_t row) {
+__device__ __forceinline__ uint32_t cvt_e4m3(const uint32_t* w, uint32_t* out) {
     uint32_t rsum = 0;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        uint32_t o[8];
+        uint32_t* o = out + 8 * i;
         block_to_bytes<N>(w + i * N, o);
 #pragma unroll
         for (int t = 0; t < 8; ++t) {
             if constexpr (A_SIDE) rsum = __dp4a(o[t], 0x01010101u, rsum);
             else o[t] ^= 0x01010101u << (N - 1);
         }
-        sts128(tile + sw128_off(row, 2 * i), o[0], o[1], o[2], o[3]);
-        sts128(tile + sw128_off(row, 2 * i + 1), o[4], o[5], o[6], o[7]);
     }
     return rsum;
 }
 
 // fp16 stage: blocks 2h, 2h+1 of the chunk -> 64 fp16 values (128 bytes).
 // Activations: 1024 + u - 1024; weights: 1024 + (j + 2^(n-1)) - (1024 + 2^(n-1)).
+// Both sides subtract 1024 + 2^(n-1): activations become u - 2^(n-1) (centred),
+// weights j.  Weights also return the sum of their offset-binary codes.
 template <int N, bool A_SIDE>
-__device__ __forceinline__ void cvt_f16(const uint32_t* w, int half, uint32_t tile, uint32_t row) {
-    const __half2 bias = __half2half2(
-        __ushort_as_half((unsigned short)(A_SIDE ? 0x6400u : (0x6400u + (1u << (N - 1))))));
+__device__ __forceinline__ uint32_t cvt_f16(const uint32_t* w, int half, uint32_t* out) {
+    const __half2 bias = __half2half2(__ushort_as_half((unsigned short)(0x6400u + (1u << (N - 1)))));
+    uint32_t csum = 0;
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
         uint32_t o[8];
         block_to_bytes<N>(w + (2 * half + i) * N, o);
-        uint32_t h[16];
+        uint32_t* h = out + 16 * i;
 #pragma unroll
         for (int t = 0; t < 8; ++t) {
             uint32_t lo, hi;
-            bytes_to_magic_half2(A_SIDE ? o[t] : (o[t] ^ (0x01010101u << (N - 1))), lo, hi);
+            const uint32_t x = A_SIDE ? o[t] : (o[t] ^ (0x01010101u << (N - 1)));
+            if constexpr (!A_SIDE) csum = __dp4a(x, 0x01010101u, csum);
+            bytes_to_magic_half2(x, lo, hi);
             h[2 * t] = half2_sub(lo, bias);
             h[2 * t + 1] = half2_sub(hi, bias);
         }
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-            sts128(tile + sw128_off(row, 4 * i + c), h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
     }
+    return csum;
+}
+
+// A stage row into the 128-byte-swizzled shared-memory operand tile.
+__device__ __forceinline__ void store_stage_smem(const uint32_t* out, uint32_t tile, uint32_t row) {
+#pragma unroll
+    for (int c = 0; c < 8; ++c) sts128(tile + sw128_off(row, c), out[4 * c], out[4 * c + 1], out[4 * c + 2], out[4 * c + 3]);
+}
+
+// A stage row into TMEM: this thread's lane, 32 consecutive columns.
+__device__ __forceinline__ void store_stage_tmem(const uint32_t* out, uint32_t taddr) {
+    uint32_t lo[16], hi[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        lo[j] = out[j];
+        hi[j] = out[16 + j];
+    }
+    tmem_st16(taddr, lo);
+    tmem_st16(taddr + 16, hi);
 }
 
 struct CvtCtx {
+    RingGeo ring;
+    bool drop_first;      // test hook: skip the first operand arrival of this warp
     uint32_t smem;        // shared-memory address of the aligned base
+    uint32_t a_tmem;      // TMEM address (lane of this thread's row) of the activation stages, or 0
     uint32_t pk_base;
     uint32_t bar0;
-    volatile int* abort_flag;
+    uint32_t abort_flag;
     int warp, lane;
     uint32_t row;
     int ci;               // next chunk
@@ -396,7 +472,8 @@ struct CvtCtx {
 // slot, reads this row's words once, fills 1 (E4M3) or 2 (fp16) operand
 // stages, and hands the slot back only after its words are consumed.
 template <int N, int KIND, bool A_SIDE>
-__device__ __forceinline__ bool convert_group(const Params& p, CvtCtx& cx, int g, int32_t* rowsum_s) {
+__device__ __forceinline__ bool convert_group(const Params& p, CvtCtx& cx, int g, int32_t* rowsum_s,
+                                              int32_t* colsum_s) {
     const Group& G = p.g[g];
     const int nchunks = G.pw / 128;
     const uint32_t xr = pk_xor(N, cx.row);
@@ -416,44 +493,58 @@ __device__ __forceinline__ bool convert_group(const Params& p, CvtCtx& cx, int g
             if (!__all_sync(0xffffffffu, wait_bounded(cx.bar0 + 8u * (BAR_OP_EMPTY + slot),
                                                         ((s / OP_STAGES) & 1) ^ 1, cx.abort_flag, p)))
                 return false;
-            const uint32_t tile = cx.smem + SMEM_OP + slot * OP_STAGE_BYTES + (A_SIDE ? 0 : OP_A_BYTES);
-            if constexpr (KIND == 0) rsum += cvt_e4m3<N, A_SIDE>(w, tile, cx.row);
-            else cvt_f16<N, A_SIDE>(w, h, tile, cx.row);
-            fence_proxy_async();
+            uint32_t out[32];
+            if constexpr (KIND == 0) rsum += cvt_e4m3<N, A_SIDE>(w, out);
+            else rsum += cvt_f16<N, A_SIDE>(w, h, out);
+            if (A_SIDE && cx.a_tmem) {
+                // after the MMA that read this stage, before the MMA that will
+                tc_fence_after();
+                store_stage_tmem(out, cx.a_tmem + (uint32_t)(slot * 32));
+                tc_fence_before();
+            } else {
+                store_stage_smem(out, cx.smem + SMEM_OP + slot * OP_STAGE_BYTES + (A_SIDE ? 0 : OP_A_BYTES), cx.row);
+                fence_proxy_async();
+            }
             __syncwarp();
-            const bool drop = (p.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) && s == 0 && cx.warp == WARP_CVA;
+            const bool drop = cx.drop_first && s == 0;
             if (cx.lane == 0 && !drop) mbar_arrive(cx.bar0 + 8u * (BAR_OP_FULL + slot));
             cx.s = s + 1;
         }
         if (cx.lane == 0) mbar_arrive(cx.bar0 + 8u * (BAR_PK_EMPTY + ci % PK_SLOTS));
-        cx.off = ring_next(p, ci, cx.off);
+        cx.off = ring_next(cx.ring, ci, cx.off);
         cx.ci = ci + 1;
     }
-    if (A_SIDE) rowsum_s[g * BM + cx.row] = (int32_t)rsum;
+    if constexpr (A_SIDE) {
+        if constexpr (KIND == 0) rowsum_s[g * BM + cx.row] = (int32_t)rsum;   // sum of activation codes
+    } else {
+        // sum of the weight codes j over the group's K range (offset binary removed)
+        if constexpr (KIND == 1) colsum_s[g * BN + cx.row] = (int32_t)rsum - (1 << (N - 1)) * G.pw;
+    }
     return true;
 }
 
 template <bool A_SIDE>
-__device__ __forceinline__ bool convert_group_n(const Params& p, CvtCtx& cx, int g, int32_t* rowsum_s) {
+__device__ __forceinline__ bool convert_group_n(const Params& p, CvtCtx& cx, int g, int32_t* rowsum_s,
+                                                int32_t* colsum_s) {
     const Group& G = p.g[g];
     const int n = A_SIDE ? G.bits_a : G.bits_w;
     if (G.kind == 0) {
         switch (n) {
-            case 1: return convert_group<1, 0, A_SIDE>(p, cx, g, rowsum_s);
-            case 2: return convert_group<2, 0, A_SIDE>(p, cx, g, rowsum_s);
-            case 3: return convert_group<3, 0, A_SIDE>(p, cx, g, rowsum_s);
-            default: return convert_group<4, 0, A_SIDE>(p, cx, g, rowsum_s);
+            case 1: return convert_group<1, 0, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+            case 2: return convert_group<2, 0, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+            case 3: return convert_group<3, 0, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+            default: return convert_group<4, 0, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
         }
     }
     switch (n) {
-        case 1: return convert_group<1, 1, A_SIDE>(p, cx, g, rowsum_s);
-        case 2: return convert_group<2, 1, A_SIDE>(p, cx, g, rowsum_s);
-        case 3: return convert_group<3, 1, A_SIDE>(p, cx, g, rowsum_s);
-        case 4: return convert_group<4, 1, A_SIDE>(p, cx, g, rowsum_s);
-        case 5: return convert_group<5, 1, A_SIDE>(p, cx, g, rowsum_s);
-        case 6: return convert_group<6, 1, A_SIDE>(p, cx, g, rowsum_s);
-        case 7: return convert_group<7, 1, A_SIDE>(p, cx, g, rowsum_s);
-        default: return convert_group<8, 1, A_SIDE>(p, cx, g, rowsum_s);
+        case 1: return convert_group<1, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+        case 2: return convert_group<2, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+        case 3: return convert_group<3, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+        case 4: return convert_group<4, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+        case 5: return convert_group<5, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+        case 6: return convert_group<6, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+        case 7: return convert_group<7, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
+        default: return convert_group<8, 1, A_SIDE>(p, cx, g, rowsum_s, colsum_s);
     }
 }
 
@@ -470,12 +561,19 @@ struct Gather {
     int tap, cb, r, s; // position of the next block in its group
 };
 
-__device__ __forceinline__ void gather_chunk(const Params& p, Gather& gt, uint32_t row, int g, uint32_t slot) {
-    const Group& G = p.g[g];
-    const int n = G.bits_a;
-    const int cpt = G.pa >> 5;
+struct GatherGroup {
+    int n;       // activation bits
+    int cpt;     // 32-code blocks per tap
+    int bw;      // cp.async width
+    int a_off;   // byte offset of the group in a packed activation row
+};
+
+__device__ __forceinline__ void gather_chunk(const Params& p, const GatherGroup& gg, Gather& gt, uint32_t row,
+                                             uint32_t slot) {
+    const int n = gg.n;
+    const int cpt = gg.cpt;
     const int taps = p.conv ? p.R * p.S : 1;
-    const int bw = G.copy_bytes;
+    const int bw = gg.bw;
     const int blk = 4 * n;
     const uint32_t xr = pk_xor(n, row);
     const uint32_t dst_row = slot + row * 16u * (uint32_t)n;
@@ -485,12 +583,12 @@ __device__ __forceinline__ void gather_chunk(const Params& p, Gather& gt, uint32
         uint32_t nbytes = 0;
         if (gt.valid && gt.tap < taps) {
             if (!p.conv) {
-                src = p.Ap + gt.base * p.a_row_bytes + G.a_off + gt.cb * blk;
+                src = p.Ap + gt.base * p.a_row_bytes + gg.a_off + gt.cb * blk;
                 nbytes = (uint32_t)bw;
             } else {
                 const int h = gt.pp * p.sh - p.ph + gt.r, w = gt.qq * p.sw - p.pw + gt.s;
                 if (h >= 0 && h < p.H && w >= 0 && w < p.W) {
-                    src = p.Ap + ((gt.base + h) * p.W + w) * p.a_row_bytes + G.a_off + gt.cb * blk;
+                    src = p.Ap + ((gt.base + h) * p.W + w) * p.a_row_bytes + gg.a_off + gt.cb * blk;
                     nbytes = (uint32_t)bw;
                 }
             }
@@ -523,9 +621,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
     const uint32_t bar0 = smem_u32(smem + SMEM_BAR);
     auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + SMEM_MISC);
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + SMEM_MISC + 4);
+    const uint32_t abort_flag = smem_u32(smem + SMEM_MISC + 4);
+    const uint32_t no_abort = smem_u32(smem + SMEM_MISC + 8);   // stays 0: waits that must run to completion
     int32_t* rowsum_s = reinterpret_cast<int32_t*>(smem + SMEM_ROWSUM);
     float* sw_s = reinterpret_cast<float*>(smem + SMEM_SW);
+    int32_t* colsum_s = reinterpret_cast<int32_t*>(smem + SMEM_CS);
     const uint32_t pk_base = smem_u32(smem + SMEM_PK);
 
     if (threadIdx.x == 0) {
@@ -543,9 +643,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
             mbar_init(bar(BAR_SLOT_FREE + i), 4);
         }
         mbar_init(bar(BAR_ACC_FULL), 1);
-        mbar_init(bar(BAR_ROWSUM), 4);
+        mbar_init(bar(BAR_ROWSUM), 8);
         mbar_init(bar(BAR_TEARDOWN), 1);
-        *abort_flag = 0;
+        asm volatile("st.volatile.shared.u32 [%0], %1;" ::"r"(abort_flag), "r"(0) : "memory");
+        asm volatile("st.volatile.shared.u32 [%0], %1;" ::"r"(no_abort), "r"(0) : "memory");
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == WARP_MMA) {
@@ -588,51 +689,57 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
             // Ring bookkeeping (identical in every producer thread): chunks
             // rel..ci-1 are in flight; `tail` is the offset of chunk rel, `off`
             // that of chunk ci and `head` the end of chunk ci-1.
-            int rel = 0, issued = 0;
+            const RingGeo ring = ring_geo(p);
+            const bool a_tma = p.a_tma != 0;
+            int rel = 0, issued = 0, ci = 0;
             uint32_t off = 0, tail = 0, head = 0;
             bool ok = true;
-            for (int ci = 0; ci < p.total_chunks && ok; ++ci) {
-                const int g = chunk_group(p, ci);
-                const Group& G = p.g[g];
-                const int c = ci - G.chunk_base;
-                if (c == 0) gt.tap = gt.cb = gt.r = gt.s = 0;
-                const uint32_t sz = (uint32_t)(G.a_bytes + G.w_bytes);
-                const int b = ci % PK_SLOTS;
-                while (rel < ci) {
-                    // is [off, off + sz) clear of the chunks in flight, and is a barrier pair free?
-                    bool fits;
-                    if (ci - rel >= PK_SLOTS) fits = false;
-                    else if (off == head) fits = head > tail || head + sz <= tail;   // tail == head: ring full
-                    else fits = head > tail && sz <= tail;                           // wrapped to offset 0
-                    if (fits) break;
-                    if (!wait_bounded(bar(BAR_PK_EMPTY + rel % PK_SLOTS), (rel / PK_SLOTS) & 1, abort_flag, p)) {
-                        ok = false;
-                        break;
+#pragma unroll 1
+            for (int g = 0; g < 2; ++g) {
+                const GatherGroup gg{p.g[g].bits_a, p.g[g].pa >> 5, p.g[g].copy_bytes, p.g[g].a_off};
+                const int nch = p.g[g].pw / 128;
+                const uint32_t a_bytes = (uint32_t)p.g[g].a_bytes, w_bytes = (uint32_t)p.g[g].w_bytes;
+                const uint32_t sz = a_bytes + w_bytes;
+                const uint32_t tx = w_bytes + (a_tma ? a_bytes : 0u);
+                const int w_x0 = p.g[g].w_off, w_dx = 16 * p.g[g].bits_w;
+                const int a_x0 = p.g[g].a_off, a_dx = 16 * p.g[g].bits_a;
+                gt.tap = gt.cb = gt.r = gt.s = 0;
+                for (int c = 0; c < nch && ok; ++c, ++ci) {
+                    const int b = ci % PK_SLOTS;
+                    while (rel < ci) {
+                        // is [off, off + sz) clear of the chunks in flight, and is a barrier pair free?
+                        bool fits;
+                        if (ci - rel >= PK_SLOTS) fits = false;
+                        else if (off == head) fits = head > tail || head + sz <= tail;   // tail == head: ring full
+                        else fits = head > tail && sz <= tail;                           // wrapped to offset 0
+                        if (fits) break;
+                        if (!wait_bounded(bar(BAR_PK_EMPTY + rel % PK_SLOTS), (rel / PK_SLOTS) & 1, abort_flag, p)) {
+                            ok = false;
+                            break;
+                        }
+                        tail = ring_next(ring, rel, tail);
+                        ++rel;
                     }
-                    tail = ring_next(p, rel, tail);
-                    ++rel;
+                    if (!ok) break;
+                    const uint32_t slot = pk_base + off;
+                    if (lead) {
+                        mbar_arrive_expect_tx(bar(BAR_PK_FULL + b), tx);
+                        tma_load_2d(slot + a_bytes, &p.tmw[g], w_x0 + c * w_dx, n0, bar(BAR_PK_FULL + b));
+                        if (a_tma) tma_load_2d(slot, &p.tma[g], a_x0 + c * a_dx, (int)m0, bar(BAR_PK_FULL + b));
+                    }
+                    if (!a_tma) {
+                        gather_chunk(p, gg, gt, prow, slot);
+                        cp_async_arrive(bar(BAR_PK_FULL + b));
+                    }
+                    head = off + sz;
+                    off = ring_next(ring, ci, off);
+                    ++issued;
                 }
-                if (!ok) break;
-                const uint32_t slot = pk_base + off;
-                if (lead) {
-                    mbar_arrive_expect_tx(bar(BAR_PK_FULL + b), (uint32_t)(G.w_bytes + (p.a_tma ? G.a_bytes : 0)));
-                    tma_load_2d(slot + G.a_bytes, &p.tmw[g], G.w_off + c * 16 * G.bits_w, n0, bar(BAR_PK_FULL + b));
-                    if (p.a_tma)
-                        tma_load_2d(slot, &p.tma[g], G.a_off + c * 16 * G.bits_a, (int)m0, bar(BAR_PK_FULL + b));
-                }
-                if (!p.a_tma) {
-                    gather_chunk(p, gt, prow, g, slot);
-                    cp_async_arrive(bar(BAR_PK_FULL + b));
-                }
-                head = off + sz;
-                off = ring_next(p, ci, off);
-                ++issued;
             }
             // copies still in flight must land before the CTA's memory is released
             if (lead) {
                 for (int ci = issued - PK_SLOTS < 0 ? 0 : issued - PK_SLOTS; ci < issued; ++ci) {
-                    volatile int no_abort = 0;
-                    wait_bounded(bar(BAR_PK_FULL + ci % PK_SLOTS), (ci / PK_SLOTS) & 1, &no_abort, p);
+                    wait_bounded(bar(BAR_PK_FULL + ci % PK_SLOTS), (ci / PK_SLOTS) & 1, no_abort, p);
                 }
             }
             asm volatile("cp.async.wait_all;" ::: "memory");
@@ -642,70 +749,99 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
         // ------------------------------------------------------------------ MMA
         if (lane == 0) {
             bool ok = true;
-            for (int s = 0; s < p.total_stages && ok; ++s) {
-                const int g = s < p.g[0].n_stages ? 0 : 1;
-                const Group& G = p.g[g];
-                const int ls = g ? s - p.g[0].n_stages : s;
-                const int slot = s % OP_STAGES;
-                uint32_t col;
-                bool first;
-                bool seg_end = false;
-                int seg = 0;
-                if (g == p.seg_group) {
-                    seg = ls / G.seg_stages;
-                    const int in_seg = ls - seg * G.seg_stages;
-                    first = in_seg == 0;
-                    seg_end = in_seg == G.seg_stages - 1 || ls == G.n_stages - 1;
-                    col = (uint32_t)(BN + (seg & 1) * BN);
-                    if (first && seg >= 2) {
-                        if (!wait_bounded(bar(BAR_SLOT_FREE + (seg & 1)), ((seg >> 1) - 1) & 1, abort_flag, p)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                    }
-                } else {
-                    first = ls == 0;
-                    col = (uint32_t)p.acc_col[g];
-                }
-                if (!wait_bounded(bar(BAR_OP_FULL + slot), (s / OP_STAGES) & 1, abort_flag, p)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t a_addr = smem_u32(smem + SMEM_OP + slot * OP_STAGE_BYTES);
-                const uint32_t b_addr = a_addr + OP_A_BYTES;
+            const bool a_in_tmem = p.a_in_tmem != 0;
+            const int seg_group = p.seg_group;
+            int slot = 0;
+            uint32_t phase = 0;
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    const uint64_t ad = sw128_desc(a_addr + 32 * k), bd = sw128_desc(b_addr + 32 * k);
-                    const uint32_t acc = (first && k == 0) ? 0u : 1u;
-                    if (G.kind == 0) mma_f8(tmem_base + col, ad, bd, acc);
-                    else mma_f16(tmem_base + col, ad, bd, acc);
+            for (int g = 0; g < 2; ++g) {
+                const int nst = p.g[g].n_stages;
+                const bool f8 = p.g[g].kind == 0;
+                const bool segmented = seg_group == g;
+                const int seg_stages = p.g[g].seg_stages;
+                const uint32_t acc_col = (uint32_t)p.acc_col[g];
+                int seg = 0, in_seg = 0;
+                for (int ls = 0; ls < nst && ok; ++ls) {
+                    uint32_t col;
+                    bool first, seg_end = false;
+                    if (segmented) {
+                        first = in_seg == 0;
+                        seg_end = in_seg == seg_stages - 1 || ls == nst - 1;
+                        col = (uint32_t)(BN + (seg & 1) * BN);
+                        if (first && seg >= 2) {
+                            if (!wait_bounded(bar(BAR_SLOT_FREE + (seg & 1)), ((seg >> 1) - 1) & 1, abort_flag, p)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                        }
+                    } else {
+                        first = ls == 0;
+                        col = acc_col;
+                    }
+                    if (!wait_bounded(bar(BAR_OP_FULL + slot), phase, abort_flag, p)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_addr = smem_u32(smem + SMEM_OP + slot * OP_STAGE_BYTES);
+                    const uint32_t b_addr = a_addr + OP_A_BYTES;
+                    if (a_in_tmem) {
+                        // 8 TMEM columns (32 bytes of K per row) per MMA
+                        const uint32_t a_t = tmem_base + (uint32_t)(A_TMEM_COL + slot * 32);
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const uint64_t bd = sw128_desc(b_addr + 32 * k);
+                            const uint32_t acc = (first && k == 0) ? 0u : 1u;
+                            if (f8) mma_f8_ta(tmem_base + col, a_t + 8 * k, bd, acc);
+                            else mma_f16_ta(tmem_base + col, a_t + 8 * k, bd, acc);
+                        }
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const uint64_t ad = sw128_desc(a_addr + 32 * k), bd = sw128_desc(b_addr + 32 * k);
+                            const uint32_t acc = (first && k == 0) ? 0u : 1u;
+                            if (f8) mma_f8(tmem_base + col, ad, bd, acc);
+                            else mma_f16(tmem_base + col, ad, bd, acc);
+                        }
+                    }
+                    mma_commit(bar(BAR_OP_EMPTY + slot));
+                    if (seg_end) mma_commit(bar(BAR_SEG_FULL + (seg & 1)));
+                    if (segmented && ++in_seg == seg_stages) {
+                        in_seg = 0;
+                        ++seg;
+                    }
+                    if (++slot == OP_STAGES) {
+                        slot = 0;
+                        phase ^= 1u;
+                    }
                 }
-                mma_commit(bar(BAR_OP_EMPTY + slot));
-                if (seg_end) mma_commit(bar(BAR_SEG_FULL + (seg & 1)));
             }
             if (ok) mma_commit(bar(BAR_ACC_FULL));
             // all issued MMAs complete before TMEM and shared memory are released
             mma_commit(bar(BAR_TEARDOWN));
-            volatile int no_abort = 0;
-            wait_bounded(bar(BAR_TEARDOWN), 0, &no_abort, p);
+            wait_bounded(bar(BAR_TEARDOWN), 0, no_abort, p);
         }
     } else if (warp < WARP_EPI) {
         // ----------------------------------------------------------- converters
         const bool a_side = warp < WARP_CVW;
-        CvtCtx cx{smem_u32(smem), pk_base, bar0, abort_flag, warp, lane,
-                  (uint32_t)(threadIdx.x - (a_side ? WARP_CVA : WARP_CVW) * 32), 0, 0, 0u};
+        // activation rows follow the warp's TMEM lane quadrant (warp % 4)
+        const uint32_t row = a_side ? (uint32_t)((warp & 3) * 32 + lane)
+                                    : (uint32_t)(threadIdx.x - WARP_CVW * 32);
+        const uint32_t a_tmem = (a_side && p.a_in_tmem)
+                                    ? tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)A_TMEM_COL
+                                    : 0u;
+        CvtCtx cx{ring_geo(p), (p.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) != 0 && warp == WARP_CVA,
+                  smem_u32(smem), a_tmem, pk_base, bar0, abort_flag, warp, lane, row, 0, 0, 0u};
+#pragma unroll 1
         for (int g = 0; g < 2; ++g) {
             if (p.g[g].pw == 0) continue;
-            const bool ok = a_side ? convert_group_n<true>(p, cx, g, rowsum_s)
-                                   : convert_group_n<false>(p, cx, g, rowsum_s);
+            const bool ok = a_side ? convert_group_n<true>(p, cx, g, rowsum_s, colsum_s)
+                                   : convert_group_n<false>(p, cx, g, rowsum_s, colsum_s);
             if (!ok) break;
         }
-        if (a_side) {
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(BAR_ROWSUM));
-        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar(BAR_ROWSUM));   // row and column sums are in shared memory
     } else {
         // ---------------------------------------------------- drains + epilogue
         const int quad = warp & 3;                 // TMEM lanes 32*quad .. +31
@@ -715,7 +851,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
         const int gs = p.seg_group;
         if (gs >= 0) {
             const uint32_t sum_col = 3 * BN;
-            for (int i = 0; i < p.g[gs].n_seg && ok; ++i) {
+            const int n_seg = gs == 0 ? p.g[0].n_seg : p.g[1].n_seg;
+            const float seg_scale = gs == 0 ? p.g[0].acc_scale : p.g[1].acc_scale;
+            for (int i = 0; i < n_seg && ok; ++i) {
                 if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_SEG_FULL + (i & 1)), (i >> 1) & 1, abort_flag, p))) {
                     ok = false;
                     break;
@@ -729,7 +867,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                     if (i > 0) tmem_ld16(lane_base + sum_col + cc * 16, s);
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        const int32_t x = __float2int_rn(__uint_as_float(v[j]) * p.g[gs].acc_scale);
+                        const int32_t x = __float2int_rn(__uint_as_float(v[j]) * seg_scale);
                         s[j] = (uint32_t)((i > 0 ? (int32_t)s[j] : 0) + x);
                     }
                     tmem_st16(lane_base + sum_col + cc * 16, s);
@@ -749,9 +887,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
 #pragma unroll
             for (int g = 0; g < 2; ++g)
                 sa[g] = m < p.M ? (p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g)) : 0.0f;
-            int32_t corr[2];
+            int32_t corr[2];   // kind 0: the weight offset times this row's activation code sum
 #pragma unroll
-            for (int g = 0; g < 2; ++g) corr[g] = p.g[g].w_offset * rowsum_s[g * BM + row];
+            for (int g = 0; g < 2; ++g) corr[g] = p.g[g].w_offset ? p.g[g].w_offset * rowsum_s[g * BM + row] : 0;
 #pragma unroll 1
             for (int cc = 0; cc < BN / 16; ++cc) {
                 int32_t acc[2][16];
@@ -772,6 +910,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
 #pragma unroll
                         for (int j = 0; j < 16; ++j)
                             acc[g][j] = __float2int_rn(__uint_as_float(v[j]) * p.g[g].acc_scale) - corr[g];
+                    }
+                    if (p.g[g].a_offset) {   // kind 1: undo the centring of the activations
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) acc[g][j] += p.g[g].a_offset * colsum_s[g * BN + cc * 16 + j];
                     }
                 }
                 const int nb = n0 + cc * 16;
@@ -894,9 +1036,11 @@ bool plan_group(const GroupGeom& G, Group& out) {
     out.kind = (G.bits_a <= 4 && G.bits_w <= 4) ? 0 : 1;
     const int codes_per_stage = out.kind == 0 ? 128 : 64;
     out.n_stages = G.pw / codes_per_stage;
-    // worst-case |product|: offset-binary weights for E4M3, signed for fp16
+    // worst-case |product|: offset-binary weights for E4M3; centred activations
+    // times signed weights for fp16
     const int64_t la = (1 << G.bits_a) - 1;
-    const int64_t maxprod = out.kind == 0 ? la * ((1 << G.bits_w) - 1) : la * (1 << (G.bits_w - 1));
+    const int64_t maxprod = out.kind == 0 ? la * ((1 << G.bits_w) - 1)
+                                          : (int64_t(1) << (G.bits_a - 1)) * (int64_t(1) << (G.bits_w - 1));
     const int64_t seg_codes = maxprod > 0 ? (int64_t(1) << 24) / maxprod : (int64_t(1) << 24);
     int64_t seg_stages = seg_codes / codes_per_stage;
     if (seg_stages < 1) return false;
@@ -904,6 +1048,7 @@ bool plan_group(const GroupGeom& G, Group& out) {
     out.seg_stages = (int32_t)seg_stages;
     out.n_seg = out.n_stages > 0 ? (int32_t)((out.n_stages + seg_stages - 1) / seg_stages) : 0;
     out.w_offset = out.kind == 0 ? (1 << (G.bits_w - 1)) : 0;
+    out.a_offset = out.kind == 1 ? (1 << (G.bits_a - 1)) : 0;
     out.acc_scale = out.kind == 0 ? 262144.0f : 1.0f;   // 2^18
     out.inv_levels = (float)(1.0 / ((double)la * (double)(1 << (G.bits_w - 1))));
     out.a_bytes = 128 * 16 * G.bits_a;
@@ -948,7 +1093,9 @@ cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st)
     p.timeout_ns = 2000000000LL;
     p.seg_group = p.g[0].n_seg > 1 ? 0 : (p.g[1].n_seg > 1 ? 1 : -1);
     if (p.seg_group < 0) {
-        p.tmem_cols = 256;
+        // accumulators in columns 0..255, activation stages in 256..351
+        p.tmem_cols = 512;
+        p.a_in_tmem = 1;
         p.acc_col[0] = 0;
         p.acc_col[1] = BN;
     } else {
