@@ -713,7 +713,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                         else if (off == head) fits = head > tail || head + sz <= tail;   // tail == head: ring full
                         else fits = head > tail && sz <= tail;                           // wrapped to offset 0
                         if (fits) break;
-                        if (!wait_bounded(bar(BAR_PK_EMPTY + rel % PK_SLOTS), (rel / PK_SLOTS) & 1, abort_flag, p)) {
+                        // warp-uniform, so that the lanes stay converged for the gather
+                        if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_PK_EMPTY + rel % PK_SLOTS), (rel / PK_SLOTS) & 1,
+                                                                  abort_flag, p))) {
                             ok = false;
                             break;
                         }
@@ -727,6 +729,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                         tma_load_2d(slot + a_bytes, &p.tmw[g], w_x0 + c * w_dx, n0, bar(BAR_PK_FULL + b));
                         if (a_tma) tma_load_2d(slot, &p.tma[g], a_x0 + c * a_dx, (int)m0, bar(BAR_PK_FULL + b));
                     }
+                    // reconverge after the lead's copies: a diverged warp issues the gather twice
+                    __syncwarp();
                     if (!a_tma) {
                         gather_chunk(p, gg, gt, prow, slot);
                         cp_async_arrive(bar(BAR_PK_FULL + b));
