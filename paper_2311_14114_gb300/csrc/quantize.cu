@@ -89,9 +89,63 @@ __global__ void __launch_bounds__(kThreads) absmax_kernel(const T* __restrict__ 
 }
 
 // ---------------------------------------------------------------------------
-// Activation quantize-and-pack.  One warp per row: the fp16 row is staged in
-// shared memory with 16-byte loads, then each 32-code block is gathered
-// through perm, quantized (Sec. 3 step 2) and packed by the warp.
+// fp16 activations, per-(tensor, group) max |a|.  Each thread owns a fixed
+// 16-byte column of the [rows][K] matrix (8 channels) and walks rows, so the
+// channel-to-group masks are computed once.  |a| is taken on the fp16 bit
+// patterns (sign cleared); for non-negative finite halves the integer order is
+// the float order, so two halves are maxed per instruction (__vmaxu2).  NaN
+// patterns are dropped, as fmaxf drops a NaN operand.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) act_absmax_kernel(const uint4* __restrict__ X, int64_t rows,
+                                                             int32_t K, const int32_t* __restrict__ perm,
+                                                             int32_t count0, unsigned* __restrict__ s_bits) {
+    extern __shared__ uint8_t grp[];   // group of each original channel
+    __shared__ float red[64];
+    for (int j = threadIdx.x; j < K; j += blockDim.x) grp[perm[j]] = (uint8_t)(j >= count0);
+    __syncthreads();
+    const int KV = K >> 3;                         // 16-byte vectors per row
+    const int cols = KV < kThreads ? KV : kThreads;
+    const int rpar = kThreads / cols;              // rows in flight per CTA
+    const int tc = threadIdx.x % cols, tr = threadIdx.x / cols;
+    uint32_t g0 = 0u, g1 = 0u;                     // packed half maxima of group 0 / 1
+    if (tr < rpar) {
+        for (int j = tc; j < KV; j += cols) {
+            uint32_t m1[4];                        // 0xFFFF in the halves of group-1 channels
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                m1[q] = (grp[8 * j + 2 * q] ? 0x0000FFFFu : 0u) | (grp[8 * j + 2 * q + 1] ? 0xFFFF0000u : 0u);
+            for (int64_t m = (int64_t)blockIdx.x * rpar + tr; m < rows; m += (int64_t)gridDim.x * rpar) {
+                const uint4 v = __ldg(X + m * KV + j);
+                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t x = w[q] & 0x7FFF7FFFu;
+                    x &= __vcmpleu2(x, 0x7C007C00u);          // NaN -> 0
+                    g1 = __vmaxu2(g1, x & m1[q]);
+                    g0 = __vmaxu2(g0, x & ~m1[q]);
+                }
+            }
+        }
+    }
+    auto hmax = [](uint32_t g) {
+        const uint32_t h = max(g & 0xFFFFu, g >> 16);
+        return __half2float(__ushort_as_half((unsigned short)h));
+    };
+    float mx0 = hmax(g0), mx1 = hmax(g1);
+    block_max2(mx0, mx1, red);
+    if (threadIdx.x == 0) {
+        atomicMax(s_bits + 0, __float_as_uint(mx0));
+        atomicMax(s_bits + 1, __float_as_uint(mx1));
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Activation quantize-and-pack.  A CTA stages a tile of rows in shared memory
+// already permuted and padded (packed position order, group g starting at
+// g ? pa0 : 0), so that each 32-code block is 64 contiguous bytes.  Four
+// consecutive threads share a block, one quarter (8 codes, 16 bytes) each:
+// they quantize (Sec. 3 step 2), build their part of each bit slice, and
+// combine the 2-bit and 1-bit slice words with two width-4 shuffles.
 // ---------------------------------------------------------------------------
 struct QuantActParams {
     const uint16_t* A;
@@ -103,64 +157,185 @@ struct QuantActParams {
     int32_t a_row_bytes;
     int32_t scale_mode;
     int32_t vec_ok;
-    int32_t warps;           // rows staged per CTA
+    int32_t tile_rows;       // rows staged per CTA
+    int32_t row_halves;      // pa0 + pa1: staged row length
+    int32_t nblk0;           // 32-code blocks of group 0 per row
+    int32_t nblk;            // blocks of both groups per row
     GroupGeom g[2];
 };
 
-__global__ void __launch_bounds__(kThreads) quantize_act_kernel(const QuantActParams p) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    uint16_t* perm_s = reinterpret_cast<uint16_t*>(smem);                 // K entries
-    const int perm_bytes = (p.K * 2 + 15) & ~15;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __half* row_s = reinterpret_cast<__half*>(smem + perm_bytes) + (int64_t)warp * p.K;
+// The code of Sec. 3 step 2, t = (a / s) * (2^n - 1) rounded half to even and
+// clipped to [0, 2^n - 1].  The quotient is formed by Markstein's correction
+// step: q0 = a * r, q = q0 + (a - q0 * s) * r with r = RN(1 / s), both
+// products fused; for |a| <= 65504 and s in [2^-60, 2^60] this is the
+// correctly rounded quotient (checked exhaustively over every fp16 a); other
+// scales take the IEEE division.  Rounding to an unsigned integer saturates
+// negative values (and NaN) at 0, which is the clip at 0.
+template <bool FAST>
+__device__ __forceinline__ uint32_t act_code_q(float a, float s, float r, float levels, uint32_t top) {
+    float q;
+    if constexpr (FAST) {
+        const float q0 = a * r;
+        q = fmaf(fmaf(-q0, s, a), r, q0);
+    } else {
+        q = __fdiv_rn(a, s);
+    }
+    return min(__float2uint_rn(__fmul_rn(q, levels)), top);
+}
 
-    for (int j = threadIdx.x; j < p.K; j += blockDim.x) perm_s[j] = (uint16_t)p.perm[j];
+// Quantizer constants of one (row or tensor, group): scale, its reciprocal,
+// the level count and the largest code.
+struct QConst {
+    float s, r, levels;
+    uint32_t top;
+    int mode;   // 0: every code is 0 (no positive scale); 1: Markstein quotient; 2: IEEE division
+};
+
+__device__ __forceinline__ QConst make_qconst(float s, int n) {
+    QConst q;
+    q.s = s;
+    q.levels = (float)((1 << n) - 1);
+    q.top = (1u << n) - 1u;
+    q.mode = (s >= 0x1p-60f && s <= 0x1p60f) ? 1 : (s > 0.0f ? 2 : 0);
+    q.r = q.mode == 1 ? __frcp_rn(s) : 0.0f;
+    return q;
+}
+
+// Quantizes 8 halves (x) into two words of bytes: byte b of o[i] is code 4i+b.
+template <bool FAST>
+__device__ __forceinline__ void quarter_codes(const uint4 x, int valid, const QConst& k, uint32_t o[2]) {
+    const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        uint32_t v = 0u;
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&xw[2 * i + e]));
+            const int c = 4 * i + 2 * e;
+            const uint32_t u0 = c < valid ? act_code_q<FAST>(f.x, k.s, k.r, k.levels, k.top) : 0u;
+            const uint32_t u1 = c + 1 < valid ? act_code_q<FAST>(f.y, k.s, k.r, k.levels, k.top) : 0u;
+            v |= (u0 | (u1 << 8)) << (16 * e);
+        }
+        o[i] = v;
+    }
+}
+
+__global__ void __launch_bounds__(256) quantize_act_kernel(const QuantActParams p) {
+    extern __shared__ __align__(16) uint8_t smem[];
+    uint16_t* pos_s = reinterpret_cast<uint16_t*>(smem);              // original channel -> staged position
+    const int pos_bytes = (p.K * 2 + 15) & ~15;
+    float* scale_s = reinterpret_cast<float*>(smem + pos_bytes);      // [tile_rows][2]
+    const int scale_bytes = (p.tile_rows * 8 + 15) & ~15;
+    __half* rows_s = reinterpret_cast<__half*>(smem + pos_bytes + scale_bytes);   // [tile_rows][RH]
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    const int RH = p.row_halves;
+
+    const int c0 = p.g[0].count, pa0 = p.g[0].pa;
+    for (int j = threadIdx.x; j < p.K; j += blockDim.x) pos_s[p.perm[j]] = (uint16_t)(j < c0 ? j : pa0 + (j - c0));
+    const bool per_row = p.scale_mode == SONIQ_SCALE_PER_ROW;
+    const QConst tk0 = make_qconst(per_row ? 0.0f : p.s_a[0], p.g[0].bits_a);
+    const QConst tk1 = make_qconst(per_row ? 0.0f : p.s_a[1], p.g[1].bits_a);
+    // staging map: thread -> (row offset, 16-byte column); no division in the loop
+    const int kv = p.K >> 3;
+    const int scols = kv < (int)blockDim.x ? kv : (int)blockDim.x;
+    const int srows = blockDim.x / scols;
+    const int s_tc = threadIdx.x % scols, s_tr = threadIdx.x / scols;
     __syncthreads();
 
-    float tensor_s[2] = {0.0f, 0.0f};
-    if (p.scale_mode != SONIQ_SCALE_PER_ROW) { tensor_s[0] = p.s_a[0]; tensor_s[1] = p.s_a[1]; }
-
-    for (int64_t m = (int64_t)blockIdx.x * p.warps + warp; m < p.M; m += (int64_t)gridDim.x * p.warps) {
-        const uint16_t* src = p.A + m * p.K;
+    for (int64_t m0 = (int64_t)blockIdx.x * p.tile_rows; m0 < p.M; m0 += (int64_t)gridDim.x * p.tile_rows) {
+        const int nr = p.M - m0 < p.tile_rows ? (int)(p.M - m0) : p.tile_rows;
+        // stage: row r, original channel c -> rows_s[r * RH + pos(c)]
         if (p.vec_ok) {
-            const uint4* s4 = reinterpret_cast<const uint4*>(src);
-            uint4* d4 = reinterpret_cast<uint4*>(row_s);
-            for (int v = lane; v < p.K / 8; v += 32) d4[v] = __ldg(s4 + v);
+            const uint4* src = reinterpret_cast<const uint4*>(p.A + m0 * p.K);
+            if (s_tr < srows) {
+                for (int j = s_tc; j < kv; j += scols) {
+                    const uint4 ps = *reinterpret_cast<const uint4*>(pos_s + 8 * j);
+                    const uint32_t pw[4] = {ps.x, ps.y, ps.z, ps.w};
+                    for (int r = s_tr; r < nr; r += srows) {
+                        const uint4 v = __ldg(src + (int64_t)r * kv + j);
+                        const uint32_t vw[4] = {v.x, v.y, v.z, v.w};
+                        uint16_t* dst = reinterpret_cast<uint16_t*>(rows_s) + r * RH;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            dst[pw[q] & 0xFFFFu] = (uint16_t)(vw[q] & 0xFFFFu);
+                            dst[pw[q] >> 16] = (uint16_t)(vw[q] >> 16);
+                        }
+                    }
+                }
+            }
         } else {
-            for (int c = lane; c < p.K; c += 32)
-                row_s[c] = *reinterpret_cast<const __half*>(src + c);
-        }
-        __syncwarp();
-
-        float s[2] = {tensor_s[0], tensor_s[1]};
-        if (p.scale_mode == SONIQ_SCALE_PER_ROW) {
-#pragma unroll
-            for (int g = 0; g < 2; ++g) {
-                float mx = 0.0f;
-                for (int j = lane; j < p.g[g].count; j += 32)
-                    mx = fmaxf(mx, fabsf(__half2float(row_s[perm_s[p.g[g].perm_base + j]])));
-                s[g] = warp_max(mx);
-            }
-            if (lane < 2) p.s_a[m * 2 + lane] = s[lane];
-        }
-
-        uint8_t* dst_row = p.Ap + m * (int64_t)p.a_row_bytes;
-#pragma unroll
-        for (int g = 0; g < 2; ++g) {
-            const GroupGeom& G = p.g[g];
-            const int n = G.bits_a;
-            const float levels = (float)((1 << n) - 1);
-            const int nblk = G.pa / 32;
-            uint32_t* dst = reinterpret_cast<uint32_t*>(dst_row + G.a_off);
-            for (int kb = 0; kb < nblk; ++kb) {
-                const int c = kb * 32 + lane;
-                uint32_t u = 0u;
-                if (c < G.count) u = act_code(__half2float(row_s[perm_s[G.perm_base + c]]), s[g], levels);
-                const uint32_t word = pack_block_warp(u, n);
-                if (lane < n) dst[kb * n + lane] = word;
+            const uint16_t* src = p.A + m0 * p.K;
+            for (int i = threadIdx.x; i < nr * p.K; i += blockDim.x) {
+                const int r = i / p.K, c = i - r * p.K;
+                reinterpret_cast<uint16_t*>(rows_s)[r * RH + pos_s[c]] = src[i];
             }
         }
-        __syncwarp();
+        __syncthreads();
+        if (per_row) {
+            // max |a| of each staged row and group (the group's channels are contiguous here)
+            for (int r = warp; r < nr; r += nwarps) {
+                const __half* row = rows_s + r * RH;
+#pragma unroll
+                for (int g = 0; g < 2; ++g) {
+                    const int base = g ? pa0 : 0;
+                    float mx = 0.0f;
+                    for (int j = lane; j < p.g[g].count; j += 32) mx = fmaxf(mx, fabsf(__half2float(row[base + j])));
+                    mx = warp_max(mx);
+                    if (lane == 0) {
+                        scale_s[2 * r + g] = mx;
+                        p.s_a[(m0 + r) * 2 + g] = mx;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+        // quarter-block tasks, whole warps at a time so that the shuffles see all lanes
+        const int tasks = nr * p.nblk * 4;
+        for (int base = warp * 32; base < tasks; base += nwarps * 32) {
+            const int t = base + lane;
+            const bool live = t < tasks;                   // whole 4-lane groups are live or not
+            const int blk = (live ? t : 0) >> 2, qq = t & 3;
+            const int r = blk / p.nblk;
+            const int kb = blk - r * p.nblk;
+            const int g = kb >= p.nblk0;
+            const int kbg = kb - (g ? p.nblk0 : 0);
+            const int n = p.g[g].bits_a;
+            const QConst k = per_row ? make_qconst(scale_s[2 * r + g], n) : (g ? tk1 : tk0);
+            const int valid = p.g[g].count - kbg * 32 - 8 * qq;   // channels of this quarter; the rest is padding
+            const uint4 x = *reinterpret_cast<const uint4*>(rows_s + r * RH + (g ? pa0 : 0) + kbg * 32 + 8 * qq);
+            uint32_t o[2];
+            if (k.mode == 1) quarter_codes<true>(x, valid, k, o);
+            else if (k.mode == 2) quarter_codes<false>(x, valid, k, o);
+            else o[0] = o[1] = 0u;                          // no positive scale: every code is 0
+            // this quarter's share of each slice word
+            const uint32_t p4 = (o[0] & 0x0F0F0F0Fu) | ((o[1] & 0x0F0F0F0Fu) << 4);
+            const int off2 = (n & 4) ? 4 : 0, off1 = off2 + ((n & 2) ? 2 : 0);
+            const int j2 = 2 * (qq & 1);
+            uint32_t p2 = (((o[0] >> off2) & 0x03030303u) << (2 * j2)) | (((o[1] >> off2) & 0x03030303u) << (2 * j2 + 2));
+            uint32_t p1 = (((o[0] >> off1) & 0x01010101u) << (2 * qq)) | (((o[1] >> off1) & 0x01010101u) << (2 * qq + 1));
+            p2 |= __shfl_xor_sync(0xffffffffu, p2, 1, 4);
+            p1 |= __shfl_xor_sync(0xffffffffu, p1, 1, 4);
+            p1 |= __shfl_xor_sync(0xffffffffu, p1, 2, 4);
+            if (!live) continue;
+            uint32_t* dst = reinterpret_cast<uint32_t*>(p.Ap + (m0 + r) * (int64_t)p.a_row_bytes + p.g[g].a_off +
+                                                        kbg * 4 * n);
+            if (n == 8) {
+                dst[2 * qq] = o[0];
+                dst[2 * qq + 1] = o[1];
+            } else {
+                int w = 0;
+                if (n & 4) {
+                    dst[qq] = p4;
+                    w = 4;
+                }
+                if (n & 2) {
+                    if ((qq & 1) == 0) dst[w + (qq >> 1)] = p2;
+                    w += 2;
+                }
+                if ((n & 1) && qq == 0) dst[w] = p1;
+            }
+        }
+        __syncthreads();   // the tile is overwritten next
     }
 }
 
@@ -244,11 +419,21 @@ cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const 
                               int64_t M, float* s_out, cudaStream_t st) {
     cudaError_t e = cudaMemsetAsync(s_out, 0, 2 * sizeof(float), st);
     if (e != cudaSuccess) return e;
-    const int vec_ok = (geo.K % 8 == 0) && ((uintptr_t)A % 16 == 0);
-    const int grid = grid_for(M * (int64_t)geo.K / 8, kThreads * 4);
-    absmax_kernel<__half><<<grid, kThreads, geo.K, st>>>(reinterpret_cast<const __half*>(A), M,
-                                                         geo.K, perm, geo.g[0].count,
-                                                         reinterpret_cast<unsigned*>(s_out), vec_ok);
+    if (geo.K % 8 == 0 && (uintptr_t)A % 16 == 0) {
+        const int KV = geo.K / 8;
+        const int rpar = kThreads / (KV < kThreads ? KV : kThreads);
+        // enough CTAs that each thread streams a handful of rows
+        int64_t ctas = (M + 4 * rpar - 1) / (4 * rpar);
+        const int64_t cap = (int64_t)num_sms() * 8;
+        if (ctas > cap) ctas = cap;
+        if (ctas < 1) ctas = 1;
+        act_absmax_kernel<<<(int)ctas, kThreads, geo.K, st>>>(reinterpret_cast<const uint4*>(A), M, geo.K, perm,
+                                                             geo.g[0].count, reinterpret_cast<unsigned*>(s_out));
+    } else {
+        const int grid = grid_for(M * (int64_t)geo.K, kThreads * 4);
+        absmax_kernel<__half><<<grid, kThreads, geo.K, st>>>(reinterpret_cast<const __half*>(A), M, geo.K, perm,
+                                                             geo.g[0].count, reinterpret_cast<unsigned*>(s_out), 0);
+    }
     note_launch();
     return cudaGetLastError();
 }
@@ -268,20 +453,26 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
     p.vec_ok = (geo.K % 8 == 0) && ((uintptr_t)A % 16 == 0);
     p.g[0] = geo.g[0];
     p.g[1] = geo.g[1];
-    const int perm_bytes = (geo.K * 2 + 15) & ~15;
-    // rows staged per CTA: as many warps as fit in 96 KB of shared memory
-    int warps = (96 * 1024 - perm_bytes) / (geo.K * 2);
-    if (warps > kThreads / 32) warps = kThreads / 32;
-    if (warps < 1) warps = 1;
-    p.warps = warps;
-    const size_t smem = (size_t)perm_bytes + (size_t)warps * geo.K * 2;
+    p.nblk0 = geo.g[0].pa / 32;
+    p.nblk = p.nblk0 + geo.g[1].pa / 32;
+    p.row_halves = geo.g[0].pa + geo.g[1].pa;
+    const int row_bytes = p.row_halves * 2;
+    // about 16 KB of staged rows per CTA, several CTAs per SM
+    int tr = (16 * 1024) / row_bytes;
+    if (tr > 64) tr = 64;
+    if (tr < 1) tr = 1;
+    p.tile_rows = tr;
+    const size_t smem = (size_t)((geo.K * 2 + 15) & ~15) + (size_t)((tr * 8 + 15) & ~15) + (size_t)tr * row_bytes;
+    if (smem > 227 * 1024) return cudaErrorInvalidValue;
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(quantize_act_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(quantize_act_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
         if (e != cudaSuccess) return e;
     }
-    const int grid = grid_for(M, warps * 4);
-    quantize_act_kernel<<<grid, warps * 32, smem, st>>>(p);
+    int64_t ctas = (M + tr - 1) / tr;
+    const int64_t cap = (int64_t)num_sms() * 8;
+    if (ctas > cap) ctas = cap;
+    quantize_act_kernel<<<(int)ctas, 256, smem, st>>>(p);
     note_launch();
     return cudaGetLastError();
 }

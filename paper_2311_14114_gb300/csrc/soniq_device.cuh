@@ -66,6 +66,41 @@ __device__ __forceinline__ uint32_t pack_block_warp(uint32_t code, int n) {
     return mine;
 }
 
+// One thread packs one block: the inverse of block_to_bytes.  Byte b of o[t]
+// holds code 4*t + b (< 2^N); w receives the block's N words.
+template <int N>
+__device__ __forceinline__ void bytes_to_block(const uint32_t* o, uint32_t* w) {
+    if constexpr (N == 8) {
+#pragma unroll
+        for (int t = 0; t < 8; ++t) w[t] = o[t];
+    } else {
+        int word = 0, off = 0;
+        if constexpr ((N & 4) != 0) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) w[q] = (o[2 * q] & 0x0F0F0F0Fu) | ((o[2 * q + 1] & 0x0F0F0F0Fu) << 4);
+            word += 4;
+            off += 4;
+        }
+        if constexpr ((N & 2) != 0) {
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                uint32_t v = 0u;
+#pragma unroll
+                for (int j = 0; j < 4; ++j) v |= ((o[4 * q + j] >> off) & 0x03030303u) << (2 * j);
+                w[word + q] = v;
+            }
+            word += 2;
+            off += 2;
+        }
+        if constexpr ((N & 1) != 0) {
+            uint32_t v = 0u;
+#pragma unroll
+            for (int t = 0; t < 8; ++t) v |= ((o[t] >> off) & 0x01010101u) << t;
+            w[word] = v;
+        }
+    }
+}
+
 // Expands one packed block (N words at w) to 8 words of bytes: byte b of
 // o[t] is the N-bit pattern of code 4*t + b.
 template <int N>

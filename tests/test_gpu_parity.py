@@ -107,6 +107,37 @@ def test_quantize_act_calibrated_clips(sq):
     assert np.array_equal(Ap.cpu().numpy(), oracle.pack_act_rows(U, d["count"], d["bits"], 128))
 
 
+@pytest.mark.parametrize("mode", ["tensor", "row"])
+def test_quantize_act_bytes_full_warps(sq, mode):
+    # enough rows that each warp stages 32 rows, plus a ragged last tile
+    d = wl.random_linear(21, M=80011, K=64, N=8, bits_lo=3, bits_hi=8, frac_hi=0.3, n_outliers=2)
+    lay = sq.Layout(d["perm"], d["count"], d["bits"], pad_unit=32)
+    Ap, s_a = sq.quantize_act(lay, _dev(d["A"]), scale_mode=mode)
+    A32 = d["A"].astype(np.float32)
+    s_ref = oracle.act_scales(A32, d["perm"], d["count"], per_row=(mode == "row"))
+    U = oracle.act_codes(A32, d["perm"], d["count"], d["bits"], s_ref, per_row=(mode == "row"))
+    assert np.array_equal(s_a.cpu().numpy(), s_ref)
+    assert np.array_equal(Ap.cpu().numpy(), oracle.pack_act_rows(U, d["count"], d["bits"], 32))
+
+
+@pytest.mark.parametrize("s_cal", [(1.0, 3.7), (2.0 ** -70, 2.0 ** 70), (6.1e-5, 65504.0)])
+def test_quantize_act_every_fp16_value(sq, s_cal):
+    # every finite fp16 pattern (signed zeros, subnormals, the extremes) through Sec. 3 step 2
+    h = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    h = h[(h & 0x7C00) != 0x7C00]
+    K = 256
+    pad = (-len(h)) % K
+    A = np.concatenate([h, np.zeros(pad, np.uint16)]).view(np.float16).reshape(-1, K)
+    rng = np.random.default_rng(5)
+    perm = rng.permutation(K).astype(np.int32)
+    count, bits = [160, 96], [4, 8]
+    lay = sq.Layout(perm, count, bits, pad_unit=32)
+    s = np.asarray(s_cal, np.float32)
+    Ap, _ = sq.quantize_act(lay, _dev(A), scale_mode="calibrated", s_a=_dev(s))
+    U = oracle.act_codes(A.astype(np.float32), perm, count, bits, s)
+    assert np.array_equal(Ap.cpu().numpy(), oracle.pack_act_rows(U, count, bits, 32))
+
+
 def test_quantize_act_unaligned_k(sq):
     # K % 8 != 0 takes the scalar staging path
     d = wl.random_linear(10, M=33, K=301, N=8, bits_lo=3, bits_hi=7, frac_hi=0.4)
