@@ -83,7 +83,7 @@ constexpr int SMEM_PK = SMEM_OP + OP_STAGES * OP_STAGE_BYTES;
 constexpr int SMEM_BAR = SMEM_PK + PK_BYTES;
 constexpr int BAR_PK_FULL = 0, BAR_PK_EMPTY = 16, BAR_OP_FULL = 32, BAR_OP_EMPTY = 35,
               BAR_SEG_FULL = 38, BAR_SLOT_FREE = 40, BAR_ACC_FULL = 42, BAR_ROWSUM = 43,
-              BAR_TEARDOWN = 44, NUM_BARS = 45;
+              BAR_TEARDOWN = 44, BAR_HALO = 45, NUM_BARS = 46;
 constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;         // tmem base, abort flag, a zero word
 constexpr int SMEM_ROWSUM = (SMEM_MISC + 16 + 15) & ~15;   // int32 [2][128]
 constexpr int SMEM_SW = SMEM_ROWSUM + 2 * BM * 4;          // fp32 [2][128]
@@ -125,6 +125,11 @@ struct Params {
     int32_t a_row_bytes;
     int32_t conv;
     int32_t a_tma;         // 1: activation chunks by TMA, 0: cp.async gather
+    int32_t a_halo;        // conv: 1 = each CTA loads its input rows once (the halo) and the
+                           // activation converters read every tap from it; 0 = per-chunk gather
+    int32_t halo_stride;   // bytes per halo pixel in shared memory (an odd multiple of 16)
+    int32_t halo_copy;     // cp.async width of the halo load (4, 8 or 16)
+    int32_t ring_cap;      // bytes of the packed ring; the halo follows it
     int32_t H, W, P, Q, R, S, sh, sw, ph, pw;
     int32_t s_a_per_row;
     int32_t out_bf16;
@@ -328,6 +333,12 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
     return v;
 }
 
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
 __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
@@ -353,6 +364,7 @@ struct RingGeo {
     int n0;              // chunks of group 0
     int total;           // chunks of both groups
     uint32_t sz0, sz1;   // slot bytes of a chunk of group 0 / group 1
+    uint32_t cap;        // ring bytes
 };
 
 __device__ __forceinline__ RingGeo ring_geo(const Params& p) {
@@ -361,6 +373,7 @@ __device__ __forceinline__ RingGeo ring_geo(const Params& p) {
     r.total = p.total_chunks;
     r.sz0 = (uint32_t)(p.g[0].a_bytes + p.g[0].w_bytes);
     r.sz1 = (uint32_t)(p.g[1].a_bytes + p.g[1].w_bytes);
+    r.cap = (uint32_t)p.ring_cap;
     return r;
 }
 
@@ -370,7 +383,7 @@ __device__ __forceinline__ uint32_t chunk_size(const RingGeo& r, int ci) { retur
 // wrap to 0 when the next one would not fit.
 __device__ __forceinline__ uint32_t ring_next(const RingGeo& r, int ci, uint32_t off) {
     uint32_t nxt = off + chunk_size(r, ci);
-    if (ci + 1 < r.total && nxt + chunk_size(r, ci + 1) > (uint32_t)PK_BYTES) nxt = 0;
+    if (ci + 1 < r.total && nxt + chunk_size(r, ci + 1) > r.cap) nxt = 0;
     return nxt;
 }
 
@@ -453,6 +466,82 @@ __device__ __forceinline__ void store_stage_tmem(const uint32_t* out, uint32_t t
     tmem_st16(taddr + 16, hi);
 }
 
+// ---- the input halo of an implicit-GEMM tile -----------------------------------
+
+// The output pixels m0 .. m0 + BM - 1 read input rows from the first one's
+// first tap row to the last one's last tap row: one contiguous range of
+// pixels [first, end) of the NHWC input (whole rows, images in between).
+__device__ __forceinline__ int64_t halo_first(const Params& p, int64_t m0) {
+    const int64_t pq = (int64_t)p.P * p.Q;
+    const int64_t img = m0 / pq;
+    const int pp = (int)((m0 - img * pq) / p.Q);
+    int h = pp * p.sh - p.ph;
+    if (h < 0) h = 0;
+    return (img * p.H + h) * p.W;
+}
+
+__device__ __forceinline__ int64_t halo_end(const Params& p, int64_t m0) {
+    const int64_t pq = (int64_t)p.P * p.Q;
+    const int64_t m_last = (m0 + BM < p.M ? m0 + BM : p.M) - 1;
+    const int64_t img = m_last / pq;
+    const int pp = (int)((m_last - img * pq) / p.Q);
+    int h = pp * p.sh - p.ph + p.R - 1;
+    if (h > p.H - 1) h = p.H - 1;
+    return (img * p.H + h) * p.W + p.W;
+}
+
+// Where an activation converter thread reads its row's codes in the halo.
+struct HaloRow {
+    uint32_t base;         // shared address of the halo
+    int64_t first;         // first input pixel held
+    int64_t img_h;         // img * H of this output pixel
+    int hp, wq;            // p * sh - ph, q * sw - pw
+    bool valid;            // row < M
+    int tap, cb, r, s;     // position of the next block in its group
+};
+
+// This row's 4 blocks of the next chunk (n words each, block i at w[n*i]),
+// read from the halo; taps outside the image read code 0.
+template <int N>
+__device__ __forceinline__ void read_halo(const Params& p, const Group& G, HaloRow& hr, uint32_t* w) {
+    const int taps = p.R * p.S;
+    const int cpt = G.pa >> 5;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int h = hr.hp + hr.r, x = hr.wq + hr.s;
+        const bool in = hr.valid && hr.tap < taps && h >= 0 && h < p.H && x >= 0 && x < p.W;
+        if (in) {
+            const int64_t local = (hr.img_h + h) * p.W + x - hr.first;
+            const uint32_t a = hr.base + (uint32_t)local * (uint32_t)p.halo_stride + (uint32_t)G.a_off +
+                               (uint32_t)(hr.cb * 4 * N);
+            if (N % 4 == 0 && (a & 15u) == 0) {
+#pragma unroll
+                for (int j = 0; j < (N & ~3); j += 4) {
+                    const uint4 v = lds128(a + 4 * j);
+                    w[N * i + j] = v.x;
+                    w[N * i + j + 1] = v.y;
+                    w[N * i + j + 2] = v.z;
+                    w[N * i + j + 3] = v.w;
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < N; ++j) w[N * i + j] = lds32(a + 4 * j);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < N; ++j) w[N * i + j] = 0u;
+        }
+        if (++hr.cb == cpt) {
+            hr.cb = 0;
+            ++hr.tap;
+            if (++hr.s == p.S) {
+                hr.s = 0;
+                ++hr.r;
+            }
+        }
+    }
+}
+
 struct CvtCtx {
     RingGeo ring;
     bool drop_first;      // test hook: skip the first operand arrival of this warp
@@ -466,6 +555,8 @@ struct CvtCtx {
     int ci;               // next chunk
     int s;                // next operand stage
     uint32_t off;         // ring offset of chunk ci
+    bool halo;            // activation side: read taps from the halo
+    HaloRow hr;
 };
 
 // Converts all chunks of group g for this row: per chunk, waits for its packed
@@ -478,6 +569,7 @@ __device__ __forceinline__ bool convert_group(const Params& p, CvtCtx& cx, int g
     const int nchunks = G.pw / 128;
     const uint32_t xr = pk_xor(N, cx.row);
     const uint32_t row_off = (A_SIDE ? 0u : (uint32_t)G.a_bytes) + cx.row * 16u * (uint32_t)N;
+    if (A_SIDE && cx.halo) cx.hr.tap = cx.hr.cb = cx.hr.r = cx.hr.s = 0;
     uint32_t rsum = 0;
     for (int c = 0; c < nchunks; ++c) {
         const int ci = cx.ci;
@@ -485,7 +577,8 @@ __device__ __forceinline__ bool convert_group(const Params& p, CvtCtx& cx, int g
                                                     (ci / PK_SLOTS) & 1, cx.abort_flag, p)))
             return false;
         uint32_t w[4 * N];
-        read_chunk<N>(cx.pk_base + cx.off + row_off, xr, w);
+        if (A_SIDE && cx.halo) read_halo<N>(p, G, cx.hr, w);
+        else read_chunk<N>(cx.pk_base + cx.off + row_off, xr, w);
 #pragma unroll
         for (int h = 0; h < (KIND == 0 ? 1 : 2); ++h) {
             const int s = cx.s;
@@ -550,15 +643,18 @@ __device__ __forceinline__ bool convert_group_n(const Params& p, CvtCtx& cx, int
 
 // ---- activation gather (implicit GEMM / unaligned rows) -----------------------
 
-// One producer thread copies one activation row of each chunk.  Block kb of a
-// group's weight K range holds tap kb / cpt and channel block kb % cpt; the
-// thread walks blocks in order, so tap, channel block and the tap's filter
-// offsets advance by counting instead of division.
+// Producer thread t copies block slot i = t & 3 of every chunk for the four
+// rows (t >> 2) + 32 k, k = 0..3.  The four threads of a row copy its four
+// blocks, which lie side by side in global memory when they share a tap, so a
+// warp's copy instruction touches 8 rows instead of 32.  Block kb of a group's
+// weight K range holds tap kb / cpt and channel block kb % cpt; slot i of
+// chunk c is block 4c + i, so tap, channel block and the tap's filter offsets
+// advance by counting.
 struct Gather {
-    int64_t base;      // GEMM: row m; conv: img * H
-    int pp, qq;        // conv: output pixel
-    bool valid;        // row < M
-    int tap, cb, r, s; // position of the next block in its group
+    int64_t base[4];   // GEMM: row m; conv: img * H
+    int pp[4], qq[4];  // conv: output pixel
+    uint32_t valid;    // bit k: row k is < M
+    int tap, cb, r, s; // position of this thread's block slot in the next chunk
 };
 
 struct GatherGroup {
@@ -568,43 +664,57 @@ struct GatherGroup {
     int a_off;   // byte offset of the group in a packed activation row
 };
 
-__device__ __forceinline__ void gather_chunk(const Params& p, const GatherGroup& gg, Gather& gt, uint32_t row,
+__device__ __forceinline__ void gather_start_group(Gather& gt, int slot_i, int cpt, int S) {
+    gt.tap = slot_i / cpt;
+    gt.cb = slot_i - gt.tap * cpt;
+    gt.r = gt.tap / S;
+    gt.s = gt.tap - gt.r * S;
+}
+
+__device__ __forceinline__ void gather_advance(Gather& gt, int cpt, int S) {
+    gt.cb += 4;
+    while (gt.cb >= cpt) {
+        gt.cb -= cpt;
+        ++gt.tap;
+        if (++gt.s == S) {
+            gt.s = 0;
+            ++gt.r;
+        }
+    }
+}
+
+__device__ __forceinline__ void gather_chunk(const Params& p, const GatherGroup& gg, const Gather& gt, uint32_t t,
                                              uint32_t slot) {
     const int n = gg.n;
-    const int cpt = gg.cpt;
-    const int taps = p.conv ? p.R * p.S : 1;
     const int bw = gg.bw;
     const int blk = 4 * n;
-    const uint32_t xr = pk_xor(n, row);
-    const uint32_t dst_row = slot + row * 16u * (uint32_t)n;
-#pragma unroll 1
-    for (int i = 0; i < 4; ++i) {
+    const int taps = p.conv ? p.R * p.S : 1;
+    const int i = (int)(t & 3u);
+    const bool in_k = gt.tap < taps;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t row = (t >> 2) + 32u * (uint32_t)k;
         const uint8_t* src = p.Ap;   // any valid address when zero-filling
         uint32_t nbytes = 0;
-        if (gt.valid && gt.tap < taps) {
+        if (((gt.valid >> k) & 1u) && in_k) {
             if (!p.conv) {
-                src = p.Ap + gt.base * p.a_row_bytes + gg.a_off + gt.cb * blk;
+                src = p.Ap + gt.base[k] * p.a_row_bytes + gg.a_off + gt.cb * blk;
                 nbytes = (uint32_t)bw;
             } else {
-                const int h = gt.pp * p.sh - p.ph + gt.r, w = gt.qq * p.sw - p.pw + gt.s;
+                const int h = gt.pp[k] * p.sh - p.ph + gt.r, w = gt.qq[k] * p.sw - p.pw + gt.s;
                 if (h >= 0 && h < p.H && w >= 0 && w < p.W) {
-                    src = p.Ap + ((gt.base + h) * p.W + w) * p.a_row_bytes + gg.a_off + gt.cb * blk;
+                    src = p.Ap + ((gt.base[k] + h) * p.W + w) * p.a_row_bytes + gg.a_off + gt.cb * blk;
                     nbytes = (uint32_t)bw;
                 }
             }
         }
+        const uint32_t xr = pk_xor(n, row);
+        const uint32_t dst_row = slot + row * 16u * (uint32_t)n;
+#pragma unroll 1
         for (int b = 0; b < blk; b += bw) {
             const int byte = i * blk + b;
             const uint32_t dst = dst_row + ((((uint32_t)byte >> 4) ^ xr) << 4) + (uint32_t)(byte & 15);
             cp_async(dst, nbytes ? (const void*)(src + b) : (const void*)p.Ap, bw, nbytes);
-        }
-        if (++gt.cb == cpt) {
-            gt.cb = 0;
-            ++gt.tap;
-            if (++gt.s == p.S) {
-                gt.s = 0;
-                ++gt.r;
-            }
         }
     }
 }
@@ -631,7 +741,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
     if (threadIdx.x == 0) {
         for (int i = 0; i < PK_SLOTS; ++i) {
             // the TMA arrival, plus one cp.async arrival per producer thread when gathering
-            mbar_init(bar(BAR_PK_FULL + i), p.a_tma ? 1 : 1 + NUM_PROD_THREADS);
+            mbar_init(bar(BAR_PK_FULL + i), (p.a_tma || p.a_halo) ? 1 : 1 + NUM_PROD_THREADS);
             mbar_init(bar(BAR_PK_EMPTY + i), 8);
         }
         for (int i = 0; i < OP_STAGES; ++i) {
@@ -645,6 +755,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
         mbar_init(bar(BAR_ACC_FULL), 1);
         mbar_init(bar(BAR_ROWSUM), 8);
         mbar_init(bar(BAR_TEARDOWN), 1);
+        mbar_init(bar(BAR_HALO), NUM_PROD_THREADS);   // one cp.async arrival per producer thread
         asm volatile("st.volatile.shared.u32 [%0], %1;" ::"r"(abort_flag), "r"(0) : "memory");
         asm volatile("st.volatile.shared.u32 [%0], %1;" ::"r"(no_abort), "r"(0) : "memory");
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -670,27 +781,55 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
 
     if (warp >= WARP_PROD && warp < WARP_CVA) {
         // ------------------------------------------------------------ producers
-        const uint32_t prow = threadIdx.x - WARP_PROD * 32;     // activation row this thread gathers
+        const uint32_t prow = threadIdx.x - WARP_PROD * 32;     // producer thread index (see Gather)
         const bool lead = prow == 0;                           // issues the TMA copies
+        if (p.a_halo) {
+            // the tile's input rows, once: pixel first + i of the range goes to halo row i
+            const int64_t first = halo_first(p, m0);
+            const int64_t cnt = halo_end(p, m0) - first;
+            const int cw = p.halo_copy;
+            const int per_px = p.a_row_bytes / cw;
+            const uint32_t hbase = pk_base + (uint32_t)p.ring_cap;
+            const int total = cnt > 0 ? (int)cnt * per_px : 0;
+            for (int i = (int)prow; i < total; i += NUM_PROD_THREADS) {
+                const int px = i / per_px;
+                const int piece = i - px * per_px;
+                cp_async(hbase + (uint32_t)px * (uint32_t)p.halo_stride + (uint32_t)(piece * cw),
+                         p.Ap + (first + px) * p.a_row_bytes + piece * cw, cw, (uint32_t)cw);
+            }
+            cp_async_arrive(bar(BAR_HALO));
+            if (warp != WARP_PROD) {
+                asm volatile("cp.async.wait_all;" ::: "memory");
+                goto done;
+            }
+        }
         if (p.a_tma && warp != WARP_PROD) goto done;           // TMA brings both operands
         {
             Gather gt;
-            gt.valid = m0 + prow < p.M;
-            gt.base = m0 + prow;
-            gt.pp = gt.qq = 0;
-            if (p.conv && gt.valid) {
-                const int64_t pq = (int64_t)p.P * p.Q;
-                const int64_t img = (m0 + prow) / pq;
-                const int rem = (int)(m0 + prow - img * pq);
-                gt.pp = rem / p.Q;
-                gt.qq = rem - gt.pp * p.Q;
-                gt.base = img * p.H;
+            gt.valid = 0u;
+            const int64_t pq = (int64_t)p.P * p.Q;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int64_t m = m0 + (prow >> 2) + 32 * k;
+                gt.base[k] = m;
+                gt.pp[k] = gt.qq[k] = 0;
+                if (m < p.M) {
+                    gt.valid |= 1u << k;
+                    if (p.conv) {
+                        const int64_t img = m / pq;
+                        const int rem = (int)(m - img * pq);
+                        gt.pp[k] = rem / p.Q;
+                        gt.qq[k] = rem - gt.pp[k] * p.Q;
+                        gt.base[k] = img * p.H;
+                    }
+                }
             }
             // Ring bookkeeping (identical in every producer thread): chunks
             // rel..ci-1 are in flight; `tail` is the offset of chunk rel, `off`
             // that of chunk ci and `head` the end of chunk ci-1.
             const RingGeo ring = ring_geo(p);
             const bool a_tma = p.a_tma != 0;
+            const bool a_gather = !a_tma && !p.a_halo;             // per-chunk activation gather
             int rel = 0, issued = 0, ci = 0;
             uint32_t off = 0, tail = 0, head = 0;
             bool ok = true;
@@ -703,7 +842,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                 const uint32_t tx = w_bytes + (a_tma ? a_bytes : 0u);
                 const int w_x0 = p.g[g].w_off, w_dx = 16 * p.g[g].bits_w;
                 const int a_x0 = p.g[g].a_off, a_dx = 16 * p.g[g].bits_a;
-                gt.tap = gt.cb = gt.r = gt.s = 0;
+                if (gg.cpt > 0) gather_start_group(gt, (int)(prow & 3u), gg.cpt, p.S);
                 for (int c = 0; c < nch && ok; ++c, ++ci) {
                     const int b = ci % PK_SLOTS;
                     while (rel < ci) {
@@ -731,9 +870,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                     }
                     // reconverge after the lead's copies: a diverged warp issues the gather twice
                     __syncwarp();
-                    if (!a_tma) {
+                    if (a_gather) {
                         gather_chunk(p, gg, gt, prow, slot);
                         cp_async_arrive(bar(BAR_PK_FULL + b));
+                        gather_advance(gt, gg.cpt, p.S);
                     }
                     head = off + sz;
                     off = ring_next(ring, ci, off);
@@ -837,8 +977,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                                     : 0u;
         CvtCtx cx{ring_geo(p), (p.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) != 0 && warp == WARP_CVA,
                   smem_u32(smem), a_tmem, pk_base, bar0, abort_flag, warp, lane, row, 0, 0, 0u};
+        cx.halo = a_side && p.a_halo;
+        bool halo_ok = true;
+        if (cx.halo) {
+            const int64_t m = m0 + row;
+            const int64_t pq = (int64_t)p.P * p.Q;
+            const int64_t img = m / pq;
+            const int rem = (int)(m - img * pq);
+            const int pp = rem / p.Q, qq = rem - (rem / p.Q) * p.Q;
+            cx.hr.base = pk_base + (uint32_t)p.ring_cap;
+            cx.hr.first = halo_first(p, m0);
+            cx.hr.img_h = img * p.H;
+            cx.hr.hp = pp * p.sh - p.ph;
+            cx.hr.wq = qq * p.sw - p.pw;
+            cx.hr.valid = m < p.M;
+            halo_ok = __all_sync(0xffffffffu, wait_bounded(bar(BAR_HALO), 0, abort_flag, p));
+        }
 #pragma unroll 1
-        for (int g = 0; g < 2; ++g) {
+        for (int g = 0; g < 2 && halo_ok; ++g) {
             if (p.g[g].pw == 0) continue;
             const bool ok = a_side ? convert_group_n<true>(p, cx, g, rowsum_s, colsum_s)
                                    : convert_group_n<false>(p, cx, g, rowsum_s, colsum_s);
@@ -1029,6 +1185,26 @@ bool encode_packed(EncodeTiledFn enc, CUtensorMap* map, const uint8_t* base, int
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Host copies of halo_first / halo_end (same arithmetic).
+int64_t host_halo_first(const Params& p, int64_t m0) {
+    const int64_t pq = (int64_t)p.P * p.Q;
+    const int64_t img = m0 / pq;
+    const int pp = (int)((m0 - img * pq) / p.Q);
+    int h = pp * p.sh - p.ph;
+    if (h < 0) h = 0;
+    return (img * p.H + h) * p.W;
+}
+
+int64_t host_halo_end(const Params& p, int64_t m0) {
+    const int64_t pq = (int64_t)p.P * p.Q;
+    const int64_t m_last = (m0 + BM < p.M ? m0 + BM : p.M) - 1;
+    const int64_t img = m_last / pq;
+    const int pp = (int)((m_last - img * pq) / p.Q);
+    int h = pp * p.sh - p.ph + p.R - 1;
+    if (h > p.H - 1) h = p.H - 1;
+    return (img * p.H + h) * p.W + p.W;
+}
+
 // Per-group planning: operand kind, K-stages and exact accumulation segments.
 bool plan_group(const GroupGeom& G, Group& out) {
     out.bits_a = G.bits_a;
@@ -1129,6 +1305,34 @@ cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st)
         }
     }
     p.a_tma = a_tma ? 1 : 0;
+
+    // Convolution: load each tile's input rows once (the halo) when they fit
+    // beside a ring of at least three weight chunks.
+    p.ring_cap = PK_BYTES;
+    if (a.conv) {
+        const int64_t rb = geo.a_row_bytes;
+        const uintptr_t ap = (uintptr_t)a.Ap;
+        const int cw = (rb % 16 == 0 && ap % 16 == 0) ? 16 : (rb % 8 == 0 && ap % 8 == 0) ? 8
+                                                      : (rb % 4 == 0 && ap % 4 == 0) ? 4 : 0;
+        int64_t stride = (rb + 15) / 16 * 16;
+        if ((stride / 16) % 2 == 0) stride += 16;   // odd number of 16-byte units: no bank conflicts
+        int64_t max_cnt = 0;
+        for (int64_t m0 = 0; m0 < a.M; m0 += BM) {
+            const int64_t c = host_halo_end(p, m0) - host_halo_first(p, m0);
+            if (c > max_cnt) max_cnt = c;
+        }
+        int64_t w_chunk = 0;
+        for (int g = 0; g < 2; ++g)
+            if (geo.g[g].pw > 0 && p.g[g].w_bytes > w_chunk) w_chunk = p.g[g].w_bytes;
+        const int64_t ring = (PK_BYTES - max_cnt * stride) / 1024 * 1024;
+        if (cw > 0 && max_cnt > 0 && ring >= 3 * w_chunk) {
+            p.a_halo = 1;
+            p.halo_stride = (int32_t)stride;
+            p.halo_copy = cw;
+            p.ring_cap = (int32_t)ring;
+            p.g[0].a_bytes = p.g[1].a_bytes = 0;   // activation codes no longer travel in the ring
+        }
+    }
 
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;

@@ -322,6 +322,21 @@ def test_conv_1x1_and_5x5_pad128(sq):
         check_conv(sq, spec, pad_unit=128, what=f"conv {R}x{R}")
 
 
+def test_conv_wide_rows_gather_path(sq):
+    # 128-pixel tiles of a 200-pixel-wide image need ~800 input pixels of 256+ bytes: more
+    # than the shared-memory halo holds, so the kernel gathers each chunk's rows instead
+    spec = wl.ConvSpec("t", batch=1, H=6, W=200, C=256, C_out=32, R=3, S=3, stride=(1, 1),
+                       pad=(1, 1), bits_lo=6, bits_hi=8, frac_hi=0.5, seed=11)
+    check_conv(sq, spec, what="conv wide rows")
+
+
+def test_conv_tiles_span_many_images(sq):
+    # 5x5 images: a 128-pixel tile covers parts of six images (halo over whole images)
+    spec = wl.ConvSpec("t", batch=13, H=5, W=5, C=96, C_out=24, R=3, S=3, stride=(1, 1),
+                       pad=(1, 1), bits_lo=2, bits_hi=7, frac_hi=0.4, seed=12)
+    check_conv(sq, spec, what="conv small images")
+
+
 # ---------------------------------------------------------------------------
 # full-size workloads (sampled outputs where the oracle would be slow)
 # ---------------------------------------------------------------------------
