@@ -303,6 +303,18 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         : "memory");
 }
 
+// Two 16-column loads (one per accumulator) and one wait, in one statement so
+// that no register is read before the wait.
+__device__ __forceinline__ void tmem_ld16x2(uint32_t ta, uint32_t tb, uint32_t (&a)[16], uint32_t (&b)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%32];\n\t"
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%33];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : SONIQ_R16(a), SONIQ_R16(b)
+        : "r"(ta), "r"(tb)
+        : "memory");
+}
+
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
     asm volatile(
         "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n\t"
@@ -454,16 +466,20 @@ __device__ __forceinline__ void store_stage_smem(const uint32_t* out, uint32_t t
     for (int c = 0; c < 8; ++c) sts128(tile + sw128_off(row, c), out[4 * c], out[4 * c + 1], out[4 * c + 2], out[4 * c + 3]);
 }
 
-// A stage row into TMEM: this thread's lane, 32 consecutive columns.
+// A stage row into TMEM: this thread's lane, 32 consecutive columns; two
+// stores, then one wait for both.
 __device__ __forceinline__ void store_stage_tmem(const uint32_t* out, uint32_t taddr) {
-    uint32_t lo[16], hi[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-        lo[j] = out[j];
-        hi[j] = out[16 + j];
-    }
-    tmem_st16(taddr, lo);
-    tmem_st16(taddr + 16, hi);
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(out[0]), "r"(out[1]), "r"(out[2]), "r"(out[3]), "r"(out[4]), "r"(out[5]), "r"(out[6]), "r"(out[7]),
+        "r"(out[8]), "r"(out[9]), "r"(out[10]), "r"(out[11]), "r"(out[12]), "r"(out[13]), "r"(out[14]), "r"(out[15])
+        : "memory");
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n\t"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(taddr + 16),
+        "r"(out[16]), "r"(out[17]), "r"(out[18]), "r"(out[19]), "r"(out[20]), "r"(out[21]), "r"(out[22]), "r"(out[23]),
+        "r"(out[24]), "r"(out[25]), "r"(out[26]), "r"(out[27]), "r"(out[28]), "r"(out[29]), "r"(out[30]), "r"(out[31])
+        : "memory");
 }
 
 // ---- the input halo of an implicit-GEMM tile -----------------------------------
@@ -491,14 +507,21 @@ __device__ __forceinline__ int64_t halo_end(const Params& p, int64_t m0) {
 }
 
 // Where an activation converter thread reads its row's codes in the halo.
+// For tap (r, s) the input pixel is pix0 + r * W + s (halo-local index);
+// bit r of mr / bit s of ms says whether that row / column is in the image.
 struct HaloRow {
-    uint32_t base;         // shared address of the halo
-    int64_t first;         // first input pixel held
-    int64_t img_h;         // img * H of this output pixel
-    int hp, wq;            // p * sh - ph, q * sw - pw
-    bool valid;            // row < M
+    uint32_t base;         // shared address of the halo plus the group's byte offset
+    int32_t pix0;          // halo-local index of tap (0, 0) (may be negative)
+    uint32_t mr, ms;       // in-image masks over filter rows / columns (0 for rows >= M)
     int tap, cb, r, s;     // position of the next block in its group
+    uint32_t addr;         // shared address of the current tap's pixel (valid when in)
+    bool in;               // the current tap reads real codes
 };
+
+__device__ __forceinline__ void halo_tap(const Params& p, HaloRow& hr, int taps) {
+    hr.in = hr.tap < taps && ((hr.mr >> hr.r) & 1u) && ((hr.ms >> hr.s) & 1u);
+    hr.addr = hr.base + (uint32_t)(hr.pix0 + hr.r * p.W + hr.s) * (uint32_t)p.halo_stride;
+}
 
 // This row's 4 blocks of the next chunk (n words each, block i at w[n*i]),
 // read from the halo; taps outside the image read code 0.
@@ -506,15 +529,12 @@ template <int N>
 __device__ __forceinline__ void read_halo(const Params& p, const Group& G, HaloRow& hr, uint32_t* w) {
     const int taps = p.R * p.S;
     const int cpt = G.pa >> 5;
+    const bool vec = N % 4 == 0 && ((hr.base + (uint32_t)G.a_off) & 15u) == 0;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int h = hr.hp + hr.r, x = hr.wq + hr.s;
-        const bool in = hr.valid && hr.tap < taps && h >= 0 && h < p.H && x >= 0 && x < p.W;
-        if (in) {
-            const int64_t local = (hr.img_h + h) * p.W + x - hr.first;
-            const uint32_t a = hr.base + (uint32_t)local * (uint32_t)p.halo_stride + (uint32_t)G.a_off +
-                               (uint32_t)(hr.cb * 4 * N);
-            if (N % 4 == 0 && (a & 15u) == 0) {
+        const uint32_t a = hr.addr + (uint32_t)G.a_off + (uint32_t)(hr.cb * 4 * N);
+        if (hr.in) {
+            if (vec) {
 #pragma unroll
                 for (int j = 0; j < (N & ~3); j += 4) {
                     const uint4 v = lds128(a + 4 * j);
@@ -538,6 +558,7 @@ __device__ __forceinline__ void read_halo(const Params& p, const Group& G, HaloR
                 hr.s = 0;
                 ++hr.r;
             }
+            halo_tap(p, hr, taps);
         }
     }
 }
@@ -569,11 +590,16 @@ __device__ __forceinline__ bool convert_group(const Params& p, CvtCtx& cx, int g
     const int nchunks = G.pw / 128;
     const uint32_t xr = pk_xor(N, cx.row);
     const uint32_t row_off = (A_SIDE ? 0u : (uint32_t)G.a_bytes) + cx.row * 16u * (uint32_t)N;
-    if (A_SIDE && cx.halo) cx.hr.tap = cx.hr.cb = cx.hr.r = cx.hr.s = 0;
+    if (A_SIDE && cx.halo) {
+        cx.hr.tap = cx.hr.cb = cx.hr.r = cx.hr.s = 0;
+        halo_tap(p, cx.hr, p.R * p.S);
+    }
     uint32_t rsum = 0;
     for (int c = 0; c < nchunks; ++c) {
         const int ci = cx.ci;
-        if (!__all_sync(0xffffffffu, wait_bounded(cx.bar0 + 8u * (BAR_PK_FULL + ci % PK_SLOTS),
+        // the halo side reads no ring data: it only hands the slot back
+        if (!(A_SIDE && cx.halo) &&
+            !__all_sync(0xffffffffu, wait_bounded(cx.bar0 + 8u * (BAR_PK_FULL + ci % PK_SLOTS),
                                                     (ci / PK_SLOTS) & 1, cx.abort_flag, p)))
             return false;
         uint32_t w[4 * N];
@@ -985,12 +1011,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
             const int64_t img = m / pq;
             const int rem = (int)(m - img * pq);
             const int pp = rem / p.Q, qq = rem - (rem / p.Q) * p.Q;
+            const int hp = pp * p.sh - p.ph, wq = qq * p.sw - p.pw;
             cx.hr.base = pk_base + (uint32_t)p.ring_cap;
-            cx.hr.first = halo_first(p, m0);
-            cx.hr.img_h = img * p.H;
-            cx.hr.hp = pp * p.sh - p.ph;
-            cx.hr.wq = qq * p.sw - p.pw;
-            cx.hr.valid = m < p.M;
+            cx.hr.pix0 = (int32_t)((img * p.H + hp) * p.W + wq - halo_first(p, m0));
+            cx.hr.mr = cx.hr.ms = 0u;
+            if (m < p.M) {
+                for (int t = 0; t < p.R; ++t)
+                    if (hp + t >= 0 && hp + t < p.H) cx.hr.mr |= 1u << t;
+                for (int t = 0; t < p.S; ++t)
+                    if (wq + t >= 0 && wq + t < p.W) cx.hr.ms |= 1u << t;
+            }
             halo_ok = __all_sync(0xffffffffu, wait_bounded(bar(BAR_HALO), 0, abort_flag, p));
         }
 #pragma unroll 1
@@ -1050,26 +1080,28 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
             int32_t corr[2];   // kind 0: the weight offset times this row's activation code sum
 #pragma unroll
             for (int g = 0; g < 2; ++g) corr[g] = p.g[g].w_offset ? p.g[g].w_offset * rowsum_s[g * BM + row] : 0;
+            uint32_t col[2];   // TMEM column of each group's result (the int32 sum if segmented)
+#pragma unroll
+            for (int g = 0; g < 2; ++g) col[g] = g == gs ? 3 * BN : p.acc_col[g];
 #pragma unroll 1
             for (int cc = 0; cc < BN / 16; ++cc) {
                 int32_t acc[2][16];
+                uint32_t v[2][16];
+                tmem_ld16x2(lane_base + col[0] + cc * 16, lane_base + col[1] + cc * 16, v[0], v[1]);
 #pragma unroll
                 for (int g = 0; g < 2; ++g) {
-                    uint32_t v[16];
                     if (p.g[g].n_stages == 0) {
 #pragma unroll
                         for (int j = 0; j < 16; ++j) acc[g][j] = 0;
                         continue;
                     }
                     if (g == gs) {
-                        tmem_ld16(lane_base + 3 * BN + cc * 16, v);
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) acc[g][j] = (int32_t)v[j] - corr[g];
+                        for (int j = 0; j < 16; ++j) acc[g][j] = (int32_t)v[g][j] - corr[g];
                     } else {
-                        tmem_ld16(lane_base + p.acc_col[g] + cc * 16, v);
 #pragma unroll
                         for (int j = 0; j < 16; ++j)
-                            acc[g][j] = __float2int_rn(__uint_as_float(v[j]) * p.g[g].acc_scale) - corr[g];
+                            acc[g][j] = __float2int_rn(__uint_as_float(v[g][j]) * p.g[g].acc_scale) - corr[g];
                     }
                     if (p.g[g].a_offset) {   // kind 1: undo the centring of the activations
 #pragma unroll
@@ -1325,7 +1357,7 @@ cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st)
         for (int g = 0; g < 2; ++g)
             if (geo.g[g].pw > 0 && p.g[g].w_bytes > w_chunk) w_chunk = p.g[g].w_bytes;
         const int64_t ring = (PK_BYTES - max_cnt * stride) / 1024 * 1024;
-        if (cw > 0 && max_cnt > 0 && ring >= 3 * w_chunk) {
+        if (cw > 0 && max_cnt > 0 && ring >= 3 * w_chunk && a.R <= 32 && a.S <= 32) {
             p.a_halo = 1;
             p.halo_stride = (int32_t)stride;
             p.halo_copy = cw;
