@@ -745,6 +745,34 @@ __device__ __forceinline__ void gather_chunk(const Params& p, const GatherGroup&
     }
 }
 
+// MMA issue for one group whose activation stages are in TMEM: per stage,
+// wait for the operands, 4 MMAs over the stage's 128 bytes of K, and a commit
+// that frees the stage when they complete.
+template <bool F8>
+__device__ __forceinline__ bool mma_group_ta(const Params& p, uint32_t bar0, uint32_t abort_flag, uint32_t op_base,
+                                             uint32_t tmem_base, uint32_t d, int nst, int& slot, uint32_t& phase) {
+#pragma unroll 1
+    for (int ls = 0; ls < nst; ++ls) {
+        if (!wait_bounded(bar0 + 8u * (uint32_t)(BAR_OP_FULL + slot), phase, abort_flag, p)) return false;
+        tc_fence_after();
+        const uint32_t b = op_base + (uint32_t)(slot * OP_STAGE_BYTES + OP_A_BYTES);
+        const uint32_t a = tmem_base + (uint32_t)(A_TMEM_COL + slot * 32);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint64_t bd = sw128_desc(b + 32 * k);
+            const uint32_t acc = (ls == 0 && k == 0) ? 0u : 1u;
+            if constexpr (F8) mma_f8_ta(d, a + 8 * k, bd, acc);
+            else mma_f16_ta(d, a + 8 * k, bd, acc);
+        }
+        mma_commit(bar0 + 8u * (uint32_t)(BAR_OP_EMPTY + slot));
+        if (++slot == OP_STAGES) {
+            slot = 0;
+            phase ^= 1u;
+        }
+    }
+    return true;
+}
+
 // ---- the kernel ----------------------------------------------------------------
 
 __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_constant__ Params p) {
@@ -923,6 +951,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
             const int seg_group = p.seg_group;
             int slot = 0;
             uint32_t phase = 0;
+            if (a_in_tmem && seg_group < 0) {
+                // common case: no segments, activation stages in TMEM.  One tight
+                // loop per group with the operand kind fixed (a per-MMA kind test
+                // and the segment bookkeeping cost about a third of the issue rate)
+#pragma unroll 1
+                for (int g = 0; g < 2 && ok; ++g) {
+                    const int nst = p.g[g].n_stages;
+                    const uint32_t d = tmem_base + (uint32_t)p.acc_col[g];
+                    if (p.g[g].kind == 0)
+                        ok = mma_group_ta<true>(p, bar0, abort_flag, smem_u32(smem + SMEM_OP), tmem_base, d, nst, slot, phase);
+                    else
+                        ok = mma_group_ta<false>(p, bar0, abort_flag, smem_u32(smem + SMEM_OP), tmem_base, d, nst, slot, phase);
+                }
+            } else
 #pragma unroll
             for (int g = 0; g < 2; ++g) {
                 const int nst = p.g[g].n_stages;
