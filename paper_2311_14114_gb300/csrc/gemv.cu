@@ -1,14 +1,17 @@
 // Small-M mixed-precision GEMV (M <= 16): the decode-shaped case where the
-// packed weight bytes streamed from HBM are the roofline (Sec. 2.4 C5: one
-// coalesced load per packed word).
+// packed weight bytes streamed from HBM are the roofline (Sec. 2.4 C5).
 //
 // Exact integer arithmetic on CUDA cores (Sec. 4.2: unsigned x signed
 // integer dot products):
-//   * the activation codes (M rows) are expanded once per CTA into shared
-//     memory as bytes, together with their per-group row sums R_g[m];
-//   * each warp streams RT weight rows; every lane expands packed 32-code
-//     blocks to bytes, flips the sign bit (j -> j + 2^(n-1), unsigned), and
-//     accumulates dp4a(u, j + 2^(n-1)) in uint32;
+//   * each CTA expands the activation codes (M rows) once into shared memory
+//     as bytes, with their per-group row sums R_g[m];
+//   * weight rows are contiguous in HBM, so a CTA pulls a batch of rows with
+//     bulk TMA copies into one of two shared-memory buffers while its warps
+//     work on the other (the memory system sees a few large requests per
+//     SM, not one small load per lane);
+//   * a warp takes one row at a time; lane l expands the 128-code chunks l,
+//     l+32, ... of each group to bytes, flips the sign bit (j -> j + 2^(n-1),
+//     unsigned) and accumulates dp4a(u, j + 2^(n-1)) in uint32;
 //   * Acc_g = sum - 2^(n-1) * R_g[m], exact; the fp32 epilogue applies the
 //     group scales (decode rules of Sec. 3 steps 2-3).
 #include <cuda_bf16.h>
@@ -31,63 +34,273 @@ struct GemvParams {
     int32_t a_row_bytes, w_row_bytes;
     int32_t s_a_per_row, out_bf16;
     GroupGeom g[2];
-    int32_t a_s_off[2];   // byte offset of group g's [M][pa] byte matrix in shared memory
+    int32_t a_s_off[2];   // byte offset of group g's activation bytes in shared memory
+    int32_t a_m_stride[2];// bytes per activation row of group g in shared memory
+    int32_t sum_off;      // per-row integer sums of a batch [batch_rows][2][MT]
+    int32_t scale_off;    // activation scales [16][2], then weight scales [max_batches][32][2]
+    int32_t max_batches;  // batches per CTA at most
+    int32_t bar_off;      // two mbarriers
+    int32_t buf_off;      // two weight buffers of buf_bytes
+    int32_t buf_bytes;
+    int32_t batch_rows;   // weight rows per batch (<= 32: lane = row)
+    int32_t wstride;      // bytes between weight rows in a buffer
+    unsigned* err;        // device error word (a bounded wait ran out)
+    long long timeout_ns;
 };
 
-constexpr int kThreads = 256;
+// Activation chunk c (128 codes) of a row sits at c * A_CHUNK: 16 bytes of
+// padding per chunk put the chunks of consecutive lanes on different banks.
+constexpr int A_CHUNK = 144;
 
-template <int NB>
-__device__ __forceinline__ void load_words(const uint8_t* p, uint32_t* w) {
-    const uint32_t* q = reinterpret_cast<const uint32_t*>(p);
-#pragma unroll
-    for (int i = 0; i < NB; ++i) w[i] = __ldg(q + i);
+constexpr int kThreads = 512;
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
 }
 
-// Accumulates one weight block (NW-bit codes) of RT rows against MT rows of
-// activation bytes.
-template <int NW, int MT, int RT>
-__device__ __forceinline__ void gemv_block(const GemvParams& p, const uint8_t* const* wrow,
-                                           const bool* rv, int g, int kb, const uint8_t* a_s,
-                                           uint32_t (&acc)[RT][MT]) {
-    uint32_t wb[RT][8];
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+// Mask of the top code bit in every field of a w-bit slice word: flipping it
+// turns n-bit two's complement j into offset binary j + 2^(n-1).
+__host__ __device__ constexpr uint32_t top_bit_mask(int w) {
+    return w == 8 ? 0x80808080u : w == 4 ? 0x88888888u : w == 2 ? 0xAAAAAAAAu : 0xFFFFFFFFu;
+}
+
+// sum over a block of u * (w-bit slice field), the slice's w words at `sw`:
+// shifting slice word q right by w*k and masking each byte's low w bits gives
+// the fields of codes 4t..4t+3, t = q*(8/w) + k, next to activation word a[t].
+template <int W>
+__device__ __forceinline__ uint32_t slice_dot(const uint32_t* sw, const uint32_t* a, uint32_t acc) {
+    constexpr int PER = 8 / W;
+    constexpr uint32_t MASK = W == 8 ? 0xFFFFFFFFu : W == 4 ? 0x0F0F0F0Fu : W == 2 ? 0x03030303u : 0x01010101u;
 #pragma unroll
-    for (int r = 0; r < RT; ++r) {
-        uint32_t w[NW];
-        if (rv[r]) {
-            load_words<NW>(wrow[r] + p.g[g].w_off + kb * 4 * NW, w);
-        } else {
+    for (int q = 0; q < W; ++q)
 #pragma unroll
-            for (int i = 0; i < NW; ++i) w[i] = 0u;
-        }
-        block_to_bytes<NW>(w, wb[r]);
+        for (int k = 0; k < PER; ++k) acc = __dp4a((sw[q] >> (W * k)) & MASK, a[q * PER + k], acc);
+    return acc;
+}
+
+// One 128-code chunk (4 blocks, 16*NW bytes, in shared memory) of one weight
+// row against MT rows of activation bytes (chunk-padded layout, `astride`
+// bytes per row): acc[m] += sum over the chunk of u * (j + 2^(n-1)).  The
+// slices of the packed codes are used directly (weights are never expanded
+// to bytes); the slice holding the top code bit is flipped to offset binary.
+template <int NW, int MT>
+__device__ __forceinline__ void gemv_chunk(uint32_t wsrc, uint32_t a_s, int astride, int M, uint32_t (&acc)[MT]) {
+    uint32_t w[4 * NW];
+#pragma unroll
+    for (int q = 0; q < NW; ++q) {
+        const uint4 v = lds128(wsrc + 16 * q);
+        w[4 * q] = v.x;
+        w[4 * q + 1] = v.y;
+        w[4 * q + 2] = v.z;
+        w[4 * q + 3] = v.w;
+    }
+    // slice widths, low bits first; the last slice holds the top bit
+    constexpr int W0 = NW == 8 ? 8 : (NW & 4), W1 = NW == 8 ? 0 : (NW & 2), W2 = NW == 8 ? 0 : (NW & 1);
+    constexpr int WT = W2 ? W2 : (W1 ? W1 : W0);
+    constexpr int OFF1 = W0, OFF2 = W0 + W1;
+    if constexpr (MT > 2) {
+        // several activation rows: expand each block to bytes once, reuse it per row
         const uint32_t flip = sign_flip_mask(NW);
 #pragma unroll
-        for (int t = 0; t < 8; ++t) wb[r][t] ^= flip;
+        for (int i = 0; i < 4; ++i) {
+            uint32_t wb[8];
+            block_to_bytes<NW>(w + NW * i, wb);
+#pragma unroll
+            for (int t = 0; t < 8; ++t) wb[t] ^= flip;
+#pragma unroll
+            for (int m = 0; m < MT; ++m) {
+                if (m < M) {
+                    const uint32_t aa = a_s + (uint32_t)(m * astride + i * 32);
+                    const uint4 x0 = lds128(aa), x1 = lds128(aa + 16);
+                    // two short chains per block instead of one long one
+                    uint32_t e = __dp4a(wb[0], x0.x, 0u), o = __dp4a(wb[1], x0.y, 0u);
+                    e = __dp4a(wb[2], x0.z, e);
+                    o = __dp4a(wb[3], x0.w, o);
+                    e = __dp4a(wb[4], x1.x, e);
+                    o = __dp4a(wb[5], x1.y, o);
+                    e = __dp4a(wb[6], x1.z, e);
+                    o = __dp4a(wb[7], x1.w, o);
+                    acc[m] += e + o;
+                }
+            }
+        }
+        return;
     }
-    const int pa = p.g[g].pa;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        uint32_t* blk = w + NW * i;
+        // flip the top code bit: it sits in the last slice's words
+        constexpr int FIRST_TOP = NW - WT;
+#pragma unroll
+        for (int q = FIRST_TOP; q < NW; ++q) blk[q] ^= top_bit_mask(WT);
+    }
 #pragma unroll
     for (int m = 0; m < MT; ++m) {
-        if (m < p.M) {
-            const uint4* a4 = reinterpret_cast<const uint4*>(a_s + m * pa + kb * 32);
-            const uint4 x0 = a4[0], x1 = a4[1];
-            const uint32_t a[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+        if (m < M) {
+            // independent partial sums per block and slice: short dependency chains
+            uint32_t s0[4], s1[4], s2[4];
 #pragma unroll
-            for (int r = 0; r < RT; ++r)
-#pragma unroll
-                for (int t = 0; t < 8; ++t) acc[r][m] = __dp4a(wb[r][t], a[t], acc[r][m]);
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t aa = a_s + (uint32_t)(m * astride + i * 32);
+                const uint4 x0 = lds128(aa), x1 = lds128(aa + 16);
+                const uint32_t a[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+                const uint32_t* blk = w + NW * i;
+                s0[i] = s1[i] = s2[i] = 0u;
+                if constexpr (W0 > 0) s0[i] = slice_dot<W0>(blk, a, 0u);
+                if constexpr (W1 > 0) s1[i] = slice_dot<W1 ? W1 : 1>(blk + W0, a, 0u);
+                if constexpr (W2 > 0) s2[i] = slice_dot<W2 ? W2 : 1>(blk + W0 + W1, a, 0u);
+            }
+            const uint32_t t0 = (s0[0] + s0[1]) + (s0[2] + s0[3]);
+            const uint32_t t1 = (s1[0] + s1[1]) + (s1[2] + s1[3]);
+            const uint32_t t2 = (s2[0] + s2[1]) + (s2[2] + s2[3]);
+            acc[m] += t0 + (t1 << OFF1) + (t2 << OFF2);
         }
     }
 }
 
-template <int MT, int RT>
-__global__ void __launch_bounds__(kThreads) gemv_kernel(const GemvParams p) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    int32_t* rowsum = reinterpret_cast<int32_t*>(smem);   // [2][16]
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+template <int MT>
+__device__ __forceinline__ void gemv_chunk_n(int nw, uint32_t wsrc, uint32_t a_s, int astride, int M,
+                                             uint32_t (&acc)[MT]) {
+    switch (nw) {
+        case 1: gemv_chunk<1, MT>(wsrc, a_s, astride, M, acc); break;
+        case 2: gemv_chunk<2, MT>(wsrc, a_s, astride, M, acc); break;
+        case 3: gemv_chunk<3, MT>(wsrc, a_s, astride, M, acc); break;
+        case 4: gemv_chunk<4, MT>(wsrc, a_s, astride, M, acc); break;
+        case 5: gemv_chunk<5, MT>(wsrc, a_s, astride, M, acc); break;
+        case 6: gemv_chunk<6, MT>(wsrc, a_s, astride, M, acc); break;
+        case 7: gemv_chunk<7, MT>(wsrc, a_s, astride, M, acc); break;
+        default: gemv_chunk<8, MT>(wsrc, a_s, astride, M, acc); break;
+    }
+}
+
+// Blocks kb0 .. kb0 + nb - 1 (nb < 4) of a final partial chunk, block by block.
+template <int NW, int MT>
+__device__ __forceinline__ void gemv_tail(uint32_t wgrp, uint32_t a_s, int astride, int M, int kb0, int nb,
+                                          uint32_t (&acc)[MT]) {
+    const uint32_t flip = sign_flip_mask(NW);
+    for (int kb = kb0; kb < kb0 + nb; ++kb) {
+        uint32_t w[NW], wb[8];
+#pragma unroll
+        for (int i = 0; i < NW; ++i) w[i] = lds32(wgrp + (uint32_t)(kb * 4 * NW + 4 * i));
+        block_to_bytes<NW>(w, wb);
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+            if (m < M) {
+                const uint32_t aa = a_s + (uint32_t)(m * astride + (kb >> 2) * A_CHUNK + (kb & 3) * 32);
+                const uint4 x0 = lds128(aa), x1 = lds128(aa + 16);
+                const uint32_t a[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+                for (int t = 0; t < 8; ++t) acc[m] = __dp4a(wb[t] ^ flip, a[t], acc[m]);
+            }
+        }
+    }
+}
+
+template <int MT>
+__device__ __forceinline__ void gemv_tail_n(int nw, uint32_t wgrp, uint32_t a_s, int astride, int M,
+                                            int kb0, int nb, uint32_t (&acc)[MT]) {
+    switch (nw) {
+        case 1: gemv_tail<1, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+        case 2: gemv_tail<2, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+        case 3: gemv_tail<3, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+        case 4: gemv_tail<4, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+        case 5: gemv_tail<5, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+        case 6: gemv_tail<6, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+        case 7: gemv_tail<7, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+        default: gemv_tail<8, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
+    }
+}
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ bool gemv_wait(uint32_t bar, uint32_t parity, const GemvParams& p) {
+    long long t0 = 0;
+    for (uint32_t it = 0;; ++it) {
+        uint32_t ok;
+        asm volatile("{\n\t.reg .pred q;\n\tmbarrier.try_wait.parity.shared::cta.b64 q, [%1], %2;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+                     : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+        if (ok) return true;
+        if ((it & 63u) == 63u) {
+            long long t;
+            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+            if (t0 == 0) t0 = t;
+            else if (t - t0 > p.timeout_ns) {
+                atomicOr(p.err, 1u);
+                return false;
+            }
+        }
+    }
+}
+
+// Rows [n0, n0 + nr) into buffer `buf`, one bulk copy per row (issued by the
+// lanes of warp 0) to rows `wstride` bytes apart; one transaction count on the
+// buffer's barrier, armed by lane 0 before any copy can complete.
+__device__ __forceinline__ void gemv_issue(const GemvParams& p, uint8_t* smem, int buf, int64_t n0, int nr,
+                                           int lane) {
+    const uint32_t bar = smem_addr(smem + p.bar_off + 8 * buf);
+    if (lane == 0) {
+        const uint32_t bytes = (uint32_t)nr * (uint32_t)p.w_row_bytes;
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+    }
+    __syncwarp();
+    const uint32_t dst = smem_addr(smem + p.buf_off + buf * p.buf_bytes);
+    for (int r = lane; r < nr; r += 32)
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                         dst + (uint32_t)(r * p.wstride)),
+                     "l"(p.Wp + (n0 + r) * p.w_row_bytes), "r"((uint32_t)p.w_row_bytes), "r"(bar)
+                     : "memory");
+}
+
+// A persistent grid, one CTA per SM.  Each CTA expands the activation codes
+// once, then walks batches of `batch_rows` (<= 32) weight rows, double
+// buffered.  In a batch, lane l of every warp owns row l and warp w takes
+// the 128-code chunks w, w + nwarps, ... of the row's two groups (all lanes
+// of a warp work on the same chunk, so activation reads are broadcasts);
+// the per-row sums meet in shared memory.
+template <int MT>
+__global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvParams p) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    int32_t* rowsum = reinterpret_cast<int32_t*>(smem);                       // [2][16]
+    uint32_t* sums = reinterpret_cast<uint32_t*>(smem + p.sum_off);           // [batch_rows][2][MT]
+    float* sa_s = reinterpret_cast<float*>(smem + p.scale_off);               // [16][2] activation scales
+    float* sw_all = sa_s + 32;                                                // [batches of this CTA][64] weight scales
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    const int nbatch = (p.N + p.batch_rows - 1) / p.batch_rows;
+    const int c0 = (p.g[0].pa + 127) / 128, c1 = (p.g[1].pa + 127) / 128;   // chunks per group (last may be partial)
+
+    if (threadIdx.x < 32) {
+        rowsum[threadIdx.x] = 0;
+        const int m = threadIdx.x >> 1, g = threadIdx.x & 1;
+        if (m < p.M) sa_s[threadIdx.x] = p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g);
+    }
+    for (int i = threadIdx.x; i < p.batch_rows * 2 * MT; i += blockDim.x) sums[i] = 0u;
+    // the weight scales of every batch this CTA will take, read once up front
+    for (int i = threadIdx.x; i < p.max_batches * 64; i += blockDim.x) {
+        const int k = i >> 6, j = i & 63;
+        const int64_t row = ((int64_t)blockIdx.x + (int64_t)k * gridDim.x) * p.batch_rows + (j >> 1);
+        if (j < 2 * p.batch_rows && row < p.N) sw_all[i] = __ldg(p.s_w + row * 2 + (j & 1));
+    }
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 2; ++i)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(smem + p.bar_off + 8 * i)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    // the first batch streams in while the activations expand
+    if (warp == 0 && (int)blockIdx.x < nbatch) {
+        const int64_t n0 = (int64_t)blockIdx.x * p.batch_rows;
+        gemv_issue(p, smem, 0, n0, (int)(p.N - n0 < p.batch_rows ? p.N - n0 : p.batch_rows), lane);
+    }
 
     // ---- expand the activation codes of all M rows into shared memory ----
-    if (threadIdx.x < 32) rowsum[threadIdx.x] = 0;
-    __syncthreads();
 #pragma unroll
     for (int g = 0; g < 2; ++g) {
         const GroupGeom& G = p.g[g];
@@ -103,7 +316,7 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(const GemvParams p) {
             uint32_t s = 0;
 #pragma unroll
             for (int t = 0; t < 8; ++t) s = __dp4a(o[t], 0x01010101u, s);
-            uint4* d = reinterpret_cast<uint4*>(a_s + m * G.pa + kb * 32);
+            uint4* d = reinterpret_cast<uint4*>(a_s + m * p.a_m_stride[g] + (kb >> 2) * A_CHUNK + (kb & 3) * 32);
             d[0] = make_uint4(o[0], o[1], o[2], o[3]);
             d[1] = make_uint4(o[4], o[5], o[6], o[7]);
             atomicAdd(&rowsum[g * 16 + m], (int32_t)s);
@@ -111,124 +324,140 @@ __global__ void __launch_bounds__(kThreads) gemv_kernel(const GemvParams p) {
     }
     __syncthreads();
 
-    // ---- stream weight rows ----
-    const int total_warps = gridDim.x * (blockDim.x >> 5);
-    for (int n0 = (blockIdx.x * (blockDim.x >> 5) + warp) * RT; n0 < p.N; n0 += total_warps * RT) {
-        float y[RT][MT];
-#pragma unroll
-        for (int r = 0; r < RT; ++r)
-#pragma unroll
-            for (int m = 0; m < MT; ++m) y[r][m] = 0.0f;
-        const uint8_t* wrow[RT];
-        bool rv[RT];
-#pragma unroll
-        for (int r = 0; r < RT; ++r) {
-            rv[r] = n0 + r < p.N;
-            wrow[r] = p.Wp + (int64_t)(rv[r] ? n0 + r : 0) * p.w_row_bytes;
+    bool ok = true;
+    int it = 0;
+    for (int b = blockIdx.x; b < nbatch && ok; b += gridDim.x, ++it) {
+        const int buf = it & 1;
+        const int64_t n0 = (int64_t)b * p.batch_rows;
+        const int nr = (int)(p.N - n0 < p.batch_rows ? p.N - n0 : p.batch_rows);
+        // the other buffer was released by the __syncthreads that ended the previous batch
+        if (warp == 0 && b + (int)gridDim.x < nbatch) {
+            const int64_t n1 = (int64_t)(b + gridDim.x) * p.batch_rows;
+            gemv_issue(p, smem, buf ^ 1, n1, (int)(p.N - n1 < p.batch_rows ? p.N - n1 : p.batch_rows), lane);
         }
+        ok = gemv_wait(smem_addr(smem + p.bar_off + 8 * buf), (uint32_t)((it >> 1) & 1), p);
+        if (__syncthreads_or(!ok)) break;
+        if (lane < nr) {
+            const uint32_t wrow = smem_addr(smem) + (uint32_t)(p.buf_off + buf * p.buf_bytes + lane * p.wstride);
+            uint32_t acc[2][MT];
 #pragma unroll
-        for (int g = 0; g < 2; ++g) {
-            const GroupGeom& G = p.g[g];
-            if (G.pa == 0) continue;
-            uint32_t acc[RT][MT];
+            for (int g = 0; g < 2; ++g)
 #pragma unroll
-            for (int r = 0; r < RT; ++r)
-#pragma unroll
-                for (int m = 0; m < MT; ++m) acc[r][m] = 0u;
-            const uint8_t* a_s = smem + p.a_s_off[g];
-            const int nblk = G.pa / 32;   // blocks beyond pa hold no activation codes
-            for (int kb = lane; kb < nblk; kb += 32) {
-                switch (G.bits_w) {
-                    case 1: gemv_block<1, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
-                    case 2: gemv_block<2, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
-                    case 3: gemv_block<3, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
-                    case 4: gemv_block<4, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
-                    case 5: gemv_block<5, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
-                    case 6: gemv_block<6, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
-                    case 7: gemv_block<7, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
-                    default: gemv_block<8, MT, RT>(p, wrow, rv, g, kb, a_s, acc); break;
+                for (int m = 0; m < MT; ++m) acc[g][m] = 0u;
+            for (int c = warp; c < c0 + c1; c += nwarps) {
+                const int g = c >= c0;
+                const GroupGeom& G = p.g[g];
+                const int cc = g ? c - c0 : c;
+                const uint32_t a_s = smem_addr(smem) + (uint32_t)(p.a_s_off[g] + cc * A_CHUNK);
+                const int left = G.pa - cc * 128;   // activation codes from this chunk on
+                if (left >= 128) {
+                    if (g) gemv_chunk_n<MT>(G.bits_w, wrow + G.w_off + cc * 16 * G.bits_w, a_s, p.a_m_stride[1], p.M, acc[1]);
+                    else gemv_chunk_n<MT>(G.bits_w, wrow + G.w_off + cc * 16 * G.bits_w, a_s, p.a_m_stride[0], p.M, acc[0]);
+                } else {
+                    // a final partial chunk: its blocks one by one (beyond pa the weights pair with no code)
+                    const uint32_t a0 = smem_addr(smem) + (uint32_t)p.a_s_off[g];
+                    if (g) gemv_tail_n<MT>(G.bits_w, wrow + G.w_off, a0, p.a_m_stride[1], p.M, cc * 4, left / 32, acc[1]);
+                    else gemv_tail_n<MT>(G.bits_w, wrow + G.w_off, a0, p.a_m_stride[0], p.M, cc * 4, left / 32, acc[0]);
                 }
             }
-            // warp butterfly: every lane ends with the full sums
 #pragma unroll
-            for (int r = 0; r < RT; ++r)
+            for (int g = 0; g < 2; ++g)
 #pragma unroll
-                for (int m = 0; m < MT; ++m) {
-                    uint32_t v = acc[r][m];
-#pragma unroll
-                    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                    acc[r][m] = v;
-                }
-            const int32_t off = 1 << (G.bits_w - 1);
-            const float inv = 1.0f / ((float)((1 << G.bits_a) - 1) * (float)off);
-#pragma unroll
-            for (int r = 0; r < RT; ++r) {
-                if (!rv[r]) continue;
-                const int n = n0 + r;
-                const float sw = __ldg(p.s_w + (int64_t)n * 2 + g) * inv;
-#pragma unroll
-                for (int m = 0; m < MT; ++m) {
-                    if (m < p.M) {
-                        const int32_t a = (int32_t)(acc[r][m] - (uint32_t)(off * rowsum[g * 16 + m]));
-                        const float sa = p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g);
-                        y[r][m] = fmaf(sa * sw, (float)a, y[r][m]);
-                        if (p.acc_dbg != nullptr && lane == ((r * MT + m) & 31))
-                            p.acc_dbg[((int64_t)g * p.M + m) * p.N + n] = a;
-                    }
-                }
-            }
+                for (int m = 0; m < MT; ++m)
+                    if (m < p.M && acc[g][m] != 0u) atomicAdd(&sums[(lane * 2 + g) * MT + m], acc[g][m]);
         }
+        __syncthreads();
+        // epilogue: one thread per (row, m)
+        for (int t = threadIdx.x; t < nr * p.M; t += blockDim.x) {
+            const int r = t / p.M, m = t - r * p.M;
+            const int64_t n = n0 + r;
+            float y = 0.0f;
 #pragma unroll
-        for (int r = 0; r < RT; ++r) {
-            if (!rv[r]) continue;
-#pragma unroll
-            for (int m = 0; m < MT; ++m) {
-                if (m < p.M && lane == ((r * MT + m) & 31)) {
-                    const int64_t idx = (int64_t)m * p.N + n0 + r;
-                    if (p.out_bf16) reinterpret_cast<__nv_bfloat16*>(p.Y)[idx] = __float2bfloat16_rn(y[r][m]);
-                    else reinterpret_cast<__half*>(p.Y)[idx] = __float2half_rn(y[r][m]);
-                }
+            for (int g = 0; g < 2; ++g) {
+                const GroupGeom& G = p.g[g];
+                uint32_t* sp = &sums[(r * 2 + g) * MT + m];
+                const uint32_t v = *sp;
+                *sp = 0u;
+                if (G.pa == 0) continue;
+                const int32_t off = 1 << (G.bits_w - 1);
+                const int32_t a = (int32_t)(v - (uint32_t)(off * rowsum[g * 16 + m]));
+                const float inv = 1.0f / ((float)((1 << G.bits_a) - 1) * (float)off);
+                const float sw = sw_all[it * 64 + r * 2 + g] * inv;
+                const float sa = sa_s[m * 2 + g];
+                y = g == 0 ? (sa * sw) * (float)a : fmaf(sa * sw, (float)a, y);
+                if (p.acc_dbg != nullptr) p.acc_dbg[((int64_t)g * p.M + m) * p.N + n] = a;
             }
+            const int64_t idx = (int64_t)m * p.N + n;
+            if (p.out_bf16) reinterpret_cast<__nv_bfloat16*>(p.Y)[idx] = __float2bfloat16_rn(y);
+            else reinterpret_cast<__half*>(p.Y)[idx] = __float2half_rn(y);
+        }
+        __syncthreads();   // buffer and sums are free for the next batch
+    }
+    // copies still in flight (the abandoned batch and its prefetched successor)
+    // must land before the CTA exits
+    if (threadIdx.x == 0 && !ok) {
+        const int b = (int)blockIdx.x + it * (int)gridDim.x;
+        for (int j = 0; j < 2; ++j) {
+            const int k = it + j;
+            if (b + j * (int)gridDim.x < nbatch)
+                gemv_wait(smem_addr(smem + p.bar_off + 8 * (k & 1)), (uint32_t)((k >> 1) & 1), p);
         }
     }
 }
 
-size_t gemv_smem(const LayoutGeom& geo, int64_t M, int32_t* off) {
+// Shared memory: row sums, chunk-padded activation bytes of both groups,
+// per-row sums of a batch, two barriers, two weight buffers.
+size_t gemv_smem(const LayoutGeom& geo, int64_t M, int64_t N, GemvParams* p) {
     size_t o = 128;   // row sums [2][16]
     for (int g = 0; g < 2; ++g) {
-        off[g] = (int32_t)o;
-        o += (size_t)M * geo.g[g].pa;
+        const int64_t chunks = (geo.g[g].pa + 127) / 128;
+        p->a_s_off[g] = (int32_t)o;
+        p->a_m_stride[g] = (int32_t)(chunks * A_CHUNK);
+        o += (size_t)M * chunks * A_CHUNK;
         o = (o + 15) & ~(size_t)15;
     }
-    return o;
+    // weight rows at an odd number of 16-byte units apart: lanes' 16-byte reads hit distinct banks
+    int64_t ws = geo.w_row_bytes;
+    if ((ws / 16) % 2 == 0) ws += 16;
+    p->wstride = (int32_t)ws;
+    int rows = (int)((60 * 1024) / ws);
+    if (rows > 32) rows = 32;
+    if (rows < 1) rows = 1;
+    p->batch_rows = rows;
+    p->sum_off = (int32_t)o;
+    o += (size_t)rows * 2 * 16 * 4;
+    p->scale_off = (int32_t)o;
+    const int64_t nbatch = (N + rows - 1) / rows;
+    const int64_t grid = nbatch < num_sms() ? nbatch : num_sms();
+    p->max_batches = (int32_t)((nbatch + grid - 1) / grid);
+    o += (32 + (size_t)p->max_batches * 64) * 4;
+    p->bar_off = (int32_t)o;
+    o += 16;
+    o = (o + 127) & ~(size_t)127;
+    p->buf_off = (int32_t)o;
+    p->buf_bytes = (int32_t)((rows * ws + 127) / 128 * 128);
+    return o + 2 * (size_t)p->buf_bytes;
 }
 
-template <int MT, int RT>
+template <int MT>
 cudaError_t run(const GemvParams& p, size_t smem, cudaStream_t st) {
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(gemv_kernel<MT, RT>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(gemv_kernel<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
-    int per_sm = 0;
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gemv_kernel<MT, RT>,
-                                                                   kThreads, smem);
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) return cudaErrorNotSupported;
-    const int rows_per_cta = (kThreads / 32) * RT;
-    int grid = (p.N + rows_per_cta - 1) / rows_per_cta;
-    const int cap = num_sms() * per_sm;
+    int grid = (p.N + p.batch_rows - 1) / p.batch_rows;
+    const int cap = num_sms();   // one CTA per SM (double-buffered batches)
     if (grid > cap) grid = cap;
-    gemv_kernel<MT, RT><<<grid, kThreads, smem, st>>>(p);
+    gemv_kernel<MT><<<grid, kThreads, smem, st>>>(p);
     note_launch();
     return cudaGetLastError();
 }
 
 }  // namespace
 
-bool gemv_supported(const LayoutGeom& geo, int64_t M) {
-    int32_t off[2];
-    return M >= 1 && M <= 16 && gemv_smem(geo, M, off) <= 200 * 1024;
+bool gemv_supported(const LayoutGeom& geo, int64_t M, int64_t N) {
+    GemvParams p;
+    return M >= 1 && M <= 16 && geo.w_row_bytes % 16 == 0 && gemv_smem(geo, M, N, &p) <= 220 * 1024;
 }
 
 cudaError_t launch_gemv(const LayoutGeom& geo, const GemvArgs& a, cudaStream_t st) {
@@ -247,13 +476,17 @@ cudaError_t launch_gemv(const LayoutGeom& geo, const GemvArgs& a, cudaStream_t s
     p.out_bf16 = a.out_bf16;
     p.g[0] = geo.g[0];
     p.g[1] = geo.g[1];
-    if (!gemv_supported(geo, a.M)) return cudaErrorNotSupported;
-    const size_t smem = gemv_smem(geo, a.M, p.a_s_off);
-    if (a.M == 1) return run<1, 4>(p, smem, st);
-    if (a.M <= 2) return run<2, 4>(p, smem, st);
-    if (a.M <= 4) return run<4, 4>(p, smem, st);
-    if (a.M <= 8) return run<8, 2>(p, smem, st);
-    return run<16, 2>(p, smem, st);
+    if (!gemv_supported(geo, a.M, a.N)) return cudaErrorNotSupported;
+    const size_t smem = gemv_smem(geo, a.M, a.N, &p);
+    p.err = device_error_word();
+    if (p.err == nullptr) return cudaErrorUnknown;
+    p.timeout_ns = 2000000000LL;
+    if (((uintptr_t)a.Wp & 15u) != 0) return cudaErrorNotSupported;
+    if (a.M == 1) return run<1>(p, smem, st);
+    if (a.M <= 2) return run<2>(p, smem, st);
+    if (a.M <= 4) return run<4>(p, smem, st);
+    if (a.M <= 8) return run<8>(p, smem, st);
+    return run<16>(p, smem, st);
 }
 
 }  // namespace soniq

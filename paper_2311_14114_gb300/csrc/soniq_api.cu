@@ -218,7 +218,7 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     const int per_row = scale_mode == SONIQ_SCALE_PER_ROW;
     cudaStream_t s = as_stream(stream);
     const bool want_gemv = (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= 16 && !(flags & SONIQ_FLAG_FORCE_MMA));
-    if (want_gemv && gemv_supported(geo, M)) {
+    if (want_gemv && gemv_supported(geo, M, N)) {
         GemvArgs a{Ap, Wp, s_a, s_w, Y, acc_dbg, (int32_t)M, N, per_row, out_dtype == SONIQ_OUT_BF16};
         return cuda_status(launch_gemv(geo, a, s));
     }

@@ -66,7 +66,7 @@ struct GemvArgs {
 };
 // Returns cudaErrorNotSupported if the shape does not fit the GEMV kernel.
 cudaError_t launch_gemv(const LayoutGeom& geo, const GemvArgs& a, cudaStream_t st);
-bool gemv_supported(const LayoutGeom& geo, int64_t M);
+bool gemv_supported(const LayoutGeom& geo, int64_t M, int64_t N);
 
 struct MmaArgs {
     const uint8_t* Ap;
