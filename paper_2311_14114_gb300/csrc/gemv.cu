@@ -448,6 +448,8 @@ cudaError_t run(const GemvParams& p, size_t smem, cudaStream_t st) {
     int grid = (p.N + p.batch_rows - 1) / p.batch_rows;
     const int cap = num_sms();   // one CTA per SM (double-buffered batches)
     if (grid > cap) grid = cap;
+    cudaError_t ec = prefer_max_shared((const void*)gemv_kernel<MT>);
+    if (ec != cudaSuccess) return ec;
     gemv_kernel<MT><<<grid, kThreads, smem, st>>>(p);
     note_launch();
     return cudaGetLastError();

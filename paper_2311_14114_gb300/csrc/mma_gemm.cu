@@ -1425,6 +1425,8 @@ cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st)
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
+    cudaError_t ec = prefer_max_shared((const void*)mp_mma_kernel);
+    if (ec != cudaSuccess) return ec;
     dim3 grid((unsigned)((a.N + BN - 1) / BN), (unsigned)((a.M + BM - 1) / BM));
     mp_mma_kernel<<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
     note_launch();

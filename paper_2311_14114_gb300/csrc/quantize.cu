@@ -427,6 +427,7 @@ cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const 
         const int64_t cap = (int64_t)num_sms() * 8;
         if (ctas > cap) ctas = cap;
         if (ctas < 1) ctas = 1;
+        if ((e = prefer_max_shared((const void*)act_absmax_kernel)) != cudaSuccess) return e;
         act_absmax_kernel<<<(int)ctas, kThreads, geo.K, st>>>(reinterpret_cast<const uint4*>(A), M, geo.K, perm,
                                                              geo.g[0].count, reinterpret_cast<unsigned*>(s_out));
     } else {
@@ -472,6 +473,8 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
     int64_t ctas = (M + tr - 1) / tr;
     const int64_t cap = (int64_t)num_sms() * 8;
     if (ctas > cap) ctas = cap;
+    cudaError_t ec = prefer_max_shared((const void*)quantize_act_kernel);
+    if (ec != cudaSuccess) return ec;
     quantize_act_kernel<<<(int)ctas, 256, smem, st>>>(p);
     note_launch();
     return cudaGetLastError();

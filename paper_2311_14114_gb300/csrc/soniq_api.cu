@@ -5,6 +5,10 @@
 #include <cstring>
 #include <vector>
 
+#include <mutex>
+#include <set>
+#include <utility>
+
 #include "soniq_internal.h"
 
 namespace soniq {
@@ -51,6 +55,18 @@ unsigned* device_error_word() {
 }
 
 void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+cudaError_t prefer_max_shared(const void* func) {
+    static std::mutex mu;
+    static std::set<std::pair<int, const void*>> done;
+    const int dev = current_device();
+    std::lock_guard<std::mutex> lock(mu);
+    if (done.count({dev, func})) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(func, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                         (int)cudaSharedmemCarveoutMaxShared);
+    if (e == cudaSuccess) done.insert({dev, func});
+    return e;
+}
 
 int num_sms() {
     const int dev = current_device();

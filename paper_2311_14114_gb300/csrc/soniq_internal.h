@@ -38,6 +38,10 @@ soniq_status make_geom(const soniq_layout* L, int32_t taps, LayoutGeom* geo);
 unsigned* device_error_word();
 void note_launch(int n = 1);
 int num_sms();
+// Asks for the largest shared-memory carve-out for `func` (once per device):
+// every kernel of the library then runs in one L1 / shared-memory split, so
+// consecutive calls do not make the SMs reconfigure between kernels.
+cudaError_t prefer_max_shared(const void* func);
 
 // ---- launchers (return the CUDA error of the launch) ----------------------
 
