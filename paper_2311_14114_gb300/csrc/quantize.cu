@@ -340,6 +340,285 @@ __global__ void __launch_bounds__(256) quantize_act_kernel(const QuantActParams 
 }
 
 // ---------------------------------------------------------------------------
+// Per-tensor scales in one pass over the input (a cooperative launch, all
+// CTAs resident): each CTA stages its rows in shared memory (permuted and
+// padded as above) and folds their |a| into the per-group maxima; a grid-wide
+// barrier (bounded wait) makes the global maxima visible; the CTA then
+// quantizes its staged rows, one thread per 32-code block.  The input is read
+// from HBM once instead of twice.
+// ---------------------------------------------------------------------------
+struct FusedParams {
+    const uint16_t* A;
+    uint8_t* Ap;
+    float* s_a;              // [2] out
+    unsigned* bar;           // grid barrier: [0] arrivals (0 between launches), [1] generation
+    float* part;             // [gridDim][2] per-CTA maxima (library scratch)
+    unsigned* err;           // device error word
+    const int32_t* perm;
+    int64_t M;
+    int32_t K;
+    int32_t a_row_bytes;
+    int32_t vec_ok;
+    int32_t rows_per_cta;
+    int32_t row_halves;      // pa0 + pa1
+    int32_t nblk0, nblk;
+    long long timeout_ns;
+    GroupGeom g[2];
+};
+
+template <int N>
+__device__ __forceinline__ void store_block32(const uint32_t* o, uint8_t* dst) {
+    uint32_t w[N];
+    bytes_to_block<N>(o, w);
+    if constexpr (N % 4 == 0) {
+        if ((reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+#pragma unroll
+            for (int q = 0; q < N; q += 4)
+                *reinterpret_cast<uint4*>(dst + 4 * q) = make_uint4(w[q], w[q + 1], w[q + 2], w[q + 3]);
+            return;
+        }
+    }
+    if constexpr (N % 2 == 0) {
+        if ((reinterpret_cast<uintptr_t>(dst) & 7u) == 0) {
+#pragma unroll
+            for (int q = 0; q < N; q += 2) *reinterpret_cast<uint2*>(dst + 4 * q) = make_uint2(w[q], w[q + 1]);
+            return;
+        }
+    }
+#pragma unroll
+    for (int q = 0; q < N; ++q) reinterpret_cast<uint32_t*>(dst)[q] = w[q];
+}
+
+__device__ __forceinline__ void store_block32_n(int n, const uint32_t* o, uint8_t* dst) {
+    switch (n) {
+        case 1: store_block32<1>(o, dst); break;
+        case 2: store_block32<2>(o, dst); break;
+        case 3: store_block32<3>(o, dst); break;
+        case 4: store_block32<4>(o, dst); break;
+        case 5: store_block32<5>(o, dst); break;
+        case 6: store_block32<6>(o, dst); break;
+        case 7: store_block32<7>(o, dst); break;
+        default: store_block32<8>(o, dst); break;
+    }
+}
+
+__device__ __forceinline__ uint4 lds128q(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+
+// 32 staged halves at shared address `src` (padding already zero) -> 8 words of
+// bytes, codes by the Markstein quotient (scales in [2^-60, 2^60]).
+__device__ __forceinline__ void block_codes_fast(uint32_t src, float s, float rcp, float levels, uint32_t top,
+                                                 uint32_t o[8]) {
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+        const uint4 x = lds128q(src + 16u * v);
+        const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            uint32_t word = 0u;
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&xw[2 * i + e]));
+                const uint32_t u0 = act_code_q<true>(f.x, s, rcp, levels, top);
+                const uint32_t u1 = act_code_q<true>(f.y, s, rcp, levels, top);
+                word |= (u0 | (u1 << 8)) << (16 * e);
+            }
+            o[2 * v + i] = word;
+        }
+    }
+}
+
+// 32 staged halves (codes 0..31 of a block, `valid` of them real) -> 8 words of bytes.
+template <bool FAST>
+__device__ __forceinline__ void block_codes(const __half* src, int valid, const QConst& k, uint32_t o[8]) {
+    const uint4* s4 = reinterpret_cast<const uint4*>(src);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+        uint32_t q[2];
+        quarter_codes<FAST>(s4[v], valid - 8 * v, k, q);
+        o[2 * v] = q[0];
+        o[2 * v + 1] = q[1];
+    }
+}
+
+__global__ void __launch_bounds__(1024) quantize_fused_kernel(const FusedParams p) {
+    extern __shared__ __align__(16) uint8_t smem[];
+    uint16_t* pos_s = reinterpret_cast<uint16_t*>(smem);
+    const int pos_bytes = (p.K * 2 + 15) & ~15;
+    __half* rows_s = reinterpret_cast<__half*>(smem + pos_bytes);
+    __shared__ float red[64];
+    __shared__ int abort_s;
+    const int RH = p.row_halves;
+    const int c0 = p.g[0].count, pa0 = p.g[0].pa;
+    for (int j = threadIdx.x; j < p.K; j += blockDim.x) pos_s[p.perm[j]] = (uint16_t)(j < c0 ? j : pa0 + (j - c0));
+    if (threadIdx.x == 0) abort_s = 0;
+    __syncthreads();
+
+    const int64_t m0 = (int64_t)blockIdx.x * p.rows_per_cta;
+    const int nr = m0 >= p.M ? 0 : (p.M - m0 < p.rows_per_cta ? (int)(p.M - m0) : p.rows_per_cta);
+    // ---- stage the rows; the whole tile is zeroed first so that padding slots
+    // hold code 0 and do not count in the max ----
+    {
+        uint4* z = reinterpret_cast<uint4*>(rows_s);
+        const int nz = nr * RH / 8;
+        for (int i = threadIdx.x; i < nz; i += blockDim.x) z[i] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    __syncthreads();
+    if (p.vec_ok) {
+        // thread -> (row offset, 16-byte column), fixed: no division in the loops
+        const int kv = p.K >> 3;
+        const int cols = kv < (int)blockDim.x ? kv : (int)blockDim.x;
+        const int rp = blockDim.x / cols;
+        const int tc = threadIdx.x % cols, tr = threadIdx.x / cols;
+        const uint4* src = reinterpret_cast<const uint4*>(p.A + m0 * p.K);
+        if (tr < rp) {
+            for (int j = tc; j < kv; j += cols) {
+                const uint4 ps = *reinterpret_cast<const uint4*>(pos_s + 8 * j);
+                const uint32_t pw[4] = {ps.x, ps.y, ps.z, ps.w};
+                // four rows' loads in flight before their stores
+                for (int r0 = tr; r0 < nr; r0 += 4 * rp) {
+                    uint4 v[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int r = r0 + u * rp;
+                        v[u] = r < nr ? __ldg(src + (int64_t)r * kv + j) : make_uint4(0u, 0u, 0u, 0u);
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int r = r0 + u * rp;
+                        if (r >= nr) break;
+                        const uint32_t vw[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+                        uint16_t* dst = reinterpret_cast<uint16_t*>(rows_s) + r * RH;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            dst[pw[q] & 0xFFFFu] = (uint16_t)(vw[q] & 0xFFFFu);
+                            dst[pw[q] >> 16] = (uint16_t)(vw[q] >> 16);
+                        }
+                    }
+                }
+            }
+        }
+    } else {
+        const uint16_t* src = p.A + m0 * p.K;
+        for (int i = threadIdx.x; i < nr * p.K; i += blockDim.x) {
+            const int r = i / p.K, c = i - r * p.K;
+            reinterpret_cast<uint16_t*>(rows_s)[r * RH + pos_s[c]] = src[i];
+        }
+    }
+    __syncthreads();
+    // ---- per-group max |a| over the staged rows: group 0 is [0, pa0), group 1 [pa0, RH) of
+    // each row; sign cleared, two halves per instruction, NaN dropped as fmaxf drops it ----
+    uint32_t mx0 = 0u, mx1 = 0u;
+    {
+        const int vpr = RH / 8, v0 = pa0 / 8;   // 16-byte vectors per row / in group 0
+        const int cols = vpr < (int)blockDim.x ? vpr : (int)blockDim.x;
+        const int rp = blockDim.x / cols;
+        const int tc = threadIdx.x % cols, tr = threadIdx.x / cols;
+        const uint32_t rs = (uint32_t)__cvta_generic_to_shared(rows_s);
+        if (tr < rp) {
+            for (int v = tc; v < vpr; v += cols) {
+                uint32_t m = 0u;
+                for (int r = tr; r < nr; r += rp) {
+                    const uint4 x = lds128q(rs + 16u * (uint32_t)(r * vpr + v));
+                    const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint32_t a = xw[q] & 0x7FFF7FFFu;
+                        a &= __vcmpleu2(a, 0x7C007C00u);
+                        m = __vmaxu2(m, a);
+                    }
+                }
+                if (v < v0) mx0 = __vmaxu2(mx0, m);
+                else mx1 = __vmaxu2(mx1, m);
+            }
+        }
+        mx0 = max(mx0 & 0xFFFFu, mx0 >> 16);
+        mx1 = max(mx1 & 0xFFFFu, mx1 >> 16);
+    }
+    float f0 = __half2float(__ushort_as_half((unsigned short)mx0));
+    float f1 = __half2float(__ushort_as_half((unsigned short)mx1));
+    block_max2(f0, f1, red);
+    // ---- grid barrier: every CTA's maxima are published before anyone reads them.
+    // The last CTA to arrive resets the count and advances the generation, so the
+    // barrier needs no clearing between launches ----
+    if (threadIdx.x == 0) {
+        p.part[2 * blockIdx.x + 0] = f0;
+        p.part[2 * blockIdx.x + 1] = f1;
+        const unsigned gen = *reinterpret_cast<volatile unsigned*>(p.bar + 1);
+        __threadfence();
+        if (atomicAdd(p.bar, 1u) == gridDim.x - 1) {
+            *reinterpret_cast<volatile unsigned*>(p.bar) = 0u;
+            __threadfence();
+            atomicAdd(p.bar + 1, 1u);
+        }
+        long long t0 = 0;
+        for (uint32_t it = 0;; ++it) {
+            if (*reinterpret_cast<volatile unsigned*>(p.bar + 1) != gen) break;
+            if ((it & 63u) == 63u) {
+                long long t;
+                asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+                if (t0 == 0) t0 = t;
+                else if (t - t0 > p.timeout_ns) {
+                    atomicOr(p.err, 1u);
+                    abort_s = 1;
+                    break;
+                }
+            }
+        }
+        __threadfence();
+    }
+    __syncthreads();
+    if (abort_s) return;
+    // every CTA folds all partial maxima (a few hundred floats from L2)
+    float g0 = 0.0f, g1 = 0.0f;
+    for (int i = threadIdx.x; i < (int)gridDim.x; i += blockDim.x) {
+        g0 = fmaxf(g0, __ldcg(p.part + 2 * i));
+        g1 = fmaxf(g1, __ldcg(p.part + 2 * i + 1));
+    }
+    block_max2(g0, g1, red);
+    if (blockIdx.x == 0 && threadIdx.x < 2) p.s_a[threadIdx.x] = threadIdx.x ? g1 : g0;
+    const float s0 = g0, s1 = g1;
+    const QConst k0 = make_qconst(s0, p.g[0].bits_a), k1 = make_qconst(s1, p.g[1].bits_a);
+    const bool fast = k0.mode == 1 && k1.mode == 1;   // both scales in the Markstein range
+    const uint32_t rows_a = (uint32_t)__cvta_generic_to_shared(rows_s);
+
+    // ---- quantize the staged rows: thread per (row, 32-code block) ----
+    const int tasks = nr * p.nblk;
+    int t = threadIdx.x;
+    int r = t / p.nblk, kb = t - r * p.nblk;
+    const int dr = blockDim.x / p.nblk, dk = blockDim.x - dr * p.nblk;
+    for (; t < tasks; t += blockDim.x) {
+        const int g = kb >= p.nblk0;
+        const GroupGeom& G = p.g[g];
+        const int kbg = kb - (g ? p.nblk0 : 0);
+        const QConst& k = g ? k1 : k0;
+        const int valid = G.count - kbg * 32;
+        const __half* src = rows_s + r * RH + (g ? pa0 : 0) + kbg * 32;
+        uint32_t o[8];
+        if (fast) {
+            const uint32_t sa = rows_a + 2u * (uint32_t)(r * RH + (g ? pa0 : 0) + kbg * 32);
+            if (g) block_codes_fast(sa, k1.s, k1.r, k1.levels, k1.top, o);
+            else block_codes_fast(sa, k0.s, k0.r, k0.levels, k0.top, o);
+        } else if (k.mode == 1) block_codes<true>(src, valid, k, o);
+        else if (k.mode == 2) block_codes<false>(src, valid, k, o);
+        else {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) o[q] = 0u;
+        }
+        store_block32_n(G.bits_a, o, p.Ap + (m0 + r) * (int64_t)p.a_row_bytes + G.a_off + kbg * 4 * G.bits_a);
+        r += dr;
+        kb += dk;
+        if (kb >= p.nblk) {
+            kb -= p.nblk;
+            ++r;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Weight quantize-and-pack: one CTA per output row n.  K order inside a group
 // is tap-major (position p -> tap p / pa, channel p % pa), padded with code 0.
 // ---------------------------------------------------------------------------
@@ -478,6 +757,66 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
     quantize_act_kernel<<<(int)ctas, 256, smem, st>>>(p);
     note_launch();
     return cudaGetLastError();
+}
+
+// The one-pass per-tensor path, when every CTA's rows fit in shared memory
+// next to a co-resident grid; returns cudaErrorNotSupported otherwise.
+cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
+                                  float* s_a, uint8_t* Ap, cudaStream_t st) {
+    static __thread int attr_dev = -1;
+    FusedParams p;
+    p.A = A;
+    p.Ap = Ap;
+    p.s_a = s_a;
+    p.err = device_error_word();
+    p.bar = grid_barrier_word();
+    p.part = grid_partials();
+    if (p.err == nullptr || p.bar == nullptr || p.part == nullptr) return cudaErrorNotSupported;
+    p.perm = perm;
+    p.M = M;
+    p.K = geo.K;
+    p.a_row_bytes = geo.a_row_bytes;
+    p.vec_ok = (geo.K % 8 == 0) && ((uintptr_t)A % 16 == 0);
+    p.row_halves = geo.g[0].pa + geo.g[1].pa;
+    p.nblk0 = geo.g[0].pa / 32;
+    p.nblk = p.nblk0 + geo.g[1].pa / 32;
+    p.timeout_ns = 2000000000LL;
+    p.g[0] = geo.g[0];
+    p.g[1] = geo.g[1];
+    if (p.nblk == 0) return cudaErrorNotSupported;
+    const int threads = 1024;
+    const int sms = num_sms();
+    const int64_t rpc = (M + sms - 1) / sms;
+    const size_t smem = (size_t)((geo.K * 2 + 15) & ~15) + (size_t)rpc * p.row_halves * 2;
+    if (smem > 200 * 1024) return cudaErrorNotSupported;
+    p.rows_per_cta = (int32_t)rpc;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (attr_dev != dev) {
+        cudaError_t e = cudaFuncSetAttribute(quantize_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             200 * 1024);
+        if (e != cudaSuccess) return e;
+        if ((e = prefer_max_shared((const void*)quantize_fused_kernel)) != cudaSuccess) return e;
+        attr_dev = dev;
+    }
+    int per_sm = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, quantize_fused_kernel, threads, smem);
+    if (e != cudaSuccess) return e;
+    const int64_t grid = (M + rpc - 1) / rpc;
+    if (per_sm < 1 || grid > (int64_t)per_sm * sms || grid > kMaxGridPartials) return cudaErrorNotSupported;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, quantize_fused_kernel, p);
+    if (e == cudaSuccess) note_launch();
+    return e;
 }
 
 cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, const float* W,

@@ -18,6 +18,8 @@ namespace {
 // One word per device: kernels atomically OR error bits into it when a
 // bounded wait runs out; soniq_sync_status reads and clears it.
 __device__ unsigned g_error_word;
+__device__ unsigned g_grid_barrier[2];                     // per-tensor quantize: arrivals, generation
+__device__ float g_grid_partials[2 * kMaxGridPartials];    // per-tensor quantize: per-CTA maxima
 
 std::atomic<int64_t> g_launches{0};
 
@@ -52,6 +54,30 @@ unsigned* device_error_word() {
         g_err_addr[dev] = static_cast<unsigned*>(p);
     }
     return g_err_addr[dev];
+}
+
+unsigned* grid_barrier_word() {
+    static unsigned* addr[64] = {};
+    const int dev = current_device();
+    if (dev < 0 || dev >= 64) return nullptr;
+    if (addr[dev] == nullptr) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_grid_barrier) != cudaSuccess) return nullptr;
+        addr[dev] = static_cast<unsigned*>(p);
+    }
+    return addr[dev];
+}
+
+float* grid_partials() {
+    static float* addr[64] = {};
+    const int dev = current_device();
+    if (dev < 0 || dev >= 64) return nullptr;
+    if (addr[dev] == nullptr) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_grid_partials) != cudaSuccess) return nullptr;
+        addr[dev] = static_cast<float*>(p);
+    }
+    return addr[dev];
 }
 
 void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
@@ -208,7 +234,10 @@ soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M,
     cudaStream_t s = as_stream(stream);
     const uint16_t* A16 = static_cast<const uint16_t*>(A);
     if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
-        cudaError_t e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);
+        cudaError_t e = launch_quantize_fused(geo, L->perm, A16, M, s_a, Ap, s);
+        if (e == cudaSuccess) return SONIQ_OK;
+        if (e != cudaErrorNotSupported) return cuda_status(e);
+        e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);   // two passes: rows do not fit on chip
         if (e != cudaSuccess) return cuda_status(e);
     }
     return cuda_status(launch_quantize_act(geo, L->perm, A16, M, scale_mode, s_a, Ap, s));
@@ -317,6 +346,9 @@ soniq_status soniq_sync_status(soniq_stream_t stream) {
     if (v != 0) {
         const unsigned zero = 0;
         if (cudaMemcpy(addr, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return SONIQ_ERR_CUDA;
+        // an abandoned grid barrier may have left arrivals behind: start it afresh
+        unsigned* bar = grid_barrier_word();
+        if (bar != nullptr && cudaMemset(bar, 0, 2 * sizeof(unsigned)) != cudaSuccess) return SONIQ_ERR_CUDA;
         return SONIQ_ERR_TIMEOUT;
     }
     return SONIQ_OK;

@@ -36,6 +36,13 @@ soniq_status make_geom(const soniq_layout* L, int32_t taps, LayoutGeom* geo);
 
 // Device address of the library's error word on the current device (0 on failure).
 unsigned* device_error_word();
+// Library scratch on the current device for the one-pass per-tensor quantize
+// (0 on failure): a grid barrier (arrival count, generation) and per-CTA maxima
+// [kMaxGridPartials][2].  One set per device: per-tensor activation quantize
+// calls must not run concurrently on different streams of the same device.
+constexpr int kMaxGridPartials = 1024;
+unsigned* grid_barrier_word();
+float* grid_partials();
 void note_launch(int n = 1);
 int num_sms();
 // Asks for the largest shared-memory carve-out for `func` (once per device):
@@ -50,6 +57,8 @@ cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const 
 cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
                                 int64_t M, int32_t scale_mode, float* s_a, uint8_t* Ap,
                                 cudaStream_t st);
+cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
+                                  float* s_a, uint8_t* Ap, cudaStream_t st);
 cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, const float* W,
                                  int32_t N, float* s_out, cudaStream_t st);
 cudaError_t launch_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W,
