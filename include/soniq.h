@@ -182,6 +182,30 @@ SONIQ_API soniq_status soniq_quantize_act(const soniq_layout *layout, const void
                                 soniq_stream_t stream);
 
 /*
+ * Per-tensor activation quantize-and-pack that allocates nothing and never
+ * takes a second pass.  The paper has no counterpart: this is an engineering
+ * variant of soniq_quantize_act with scale_mode SONIQ_SCALE_PER_TENSOR, for
+ * callers that must not let the library reach any memory other than the
+ * arguments and a fixed scratch (for instance inside CUDA graph capture).
+ *
+ * It computes exactly what soniq_quantize_act computes in per-tensor mode
+ * (same s_a and packed bytes), in one cooperative kernel whose grid barrier
+ * and per-CTA maxima live in a file-scope static device array of the library
+ * (8 KB per device, resolved once per device with cudaGetSymbolAddress).
+ *   Limits: one CTA per SM, at most 1024 CTAs; each CTA's M / (number of SMs)
+ *   rows, padded, must fit in 200 KB of shared memory (2 * K bytes per row plus
+ *   the permutation), i.e. M * K up to about 15 * 2^20 on a 152-SM GB300.
+ *   Larger inputs return SONIQ_ERR_UNSUPPORTED before any launch.
+ *   Concurrency: calls share that scratch, so two calls that overlap in time
+ *   (on different streams of one device) race; serialize them.
+ *   A barrier wait that runs out (2 s) is reported by soniq_sync_status, which
+ *   also clears the barrier.
+ * Arguments as for soniq_quantize_act; s_a is an output [2].
+ */
+SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, const void *A, int64_t M,
+                                        float *s_a, uint8_t *Ap, soniq_stream_t stream);
+
+/*
  * Mixed-precision quantized GEMM Y = A W^T.  Sec. 3 (integer MAC per fused
  * dot product, decode rules of steps 2-3) and Sec. 4.2 (unsigned x signed
  * integer dot products):

@@ -762,15 +762,16 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
 // The one-pass per-tensor path, when every CTA's rows fit in shared memory
 // next to a co-resident grid; returns cudaErrorNotSupported otherwise.
 cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
-                                  float* s_a, uint8_t* Ap, cudaStream_t st) {
+                                  float* s_a, uint8_t* Ap, cudaStream_t st, unsigned* bar, float* part,
+                                  int max_ctas) {
     static __thread int attr_dev = -1;
     FusedParams p;
     p.A = A;
     p.Ap = Ap;
     p.s_a = s_a;
     p.err = device_error_word();
-    p.bar = grid_barrier_word();
-    p.part = grid_partials();
+    p.bar = bar;
+    p.part = part;
     if (p.err == nullptr || p.bar == nullptr || p.part == nullptr) return cudaErrorNotSupported;
     p.perm = perm;
     p.M = M;
@@ -803,7 +804,7 @@ cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, co
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, quantize_fused_kernel, threads, smem);
     if (e != cudaSuccess) return e;
     const int64_t grid = (M + rpc - 1) / rpc;
-    if (per_sm < 1 || grid > (int64_t)per_sm * sms || grid > kMaxGridPartials) return cudaErrorNotSupported;
+    if (per_sm < 1 || grid > (int64_t)per_sm * sms || grid > max_ctas) return cudaErrorNotSupported;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
     cfg.blockDim = dim3(threads);

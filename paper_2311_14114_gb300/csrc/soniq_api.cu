@@ -21,6 +21,13 @@ __device__ unsigned g_error_word;
 __device__ unsigned g_grid_barrier[2];                     // per-tensor quantize: arrivals, generation
 __device__ float g_grid_partials[2 * kMaxGridPartials];    // per-tensor quantize: per-CTA maxima
 
+// Scratch of soniq_quantize_act_oneshot: its own grid barrier (arrival count,
+// generation; zero at module load and left at zero by every completed call)
+// and per-CTA maxima for at most kOneShotMaxCtas CTAs (8 KB).
+constexpr int kOneShotMaxCtas = 1024;
+static __device__ __align__(256) unsigned g_oneshot_barrier[2];
+static __device__ __align__(256) float g_oneshot_partials[2 * kOneShotMaxCtas];
+
 std::atomic<int64_t> g_launches{0};
 
 constexpr int kMaxDevices = 64;
@@ -66,6 +73,28 @@ unsigned* grid_barrier_word() {
         addr[dev] = static_cast<unsigned*>(p);
     }
     return addr[dev];
+}
+
+// Device addresses of the one-shot scratch, resolved once per device at first
+// use; false if the runtime cannot resolve them.
+bool oneshot_scratch(unsigned** bar, float** part) {
+    static std::mutex mu;
+    static unsigned* bars[64] = {};
+    static float* parts[64] = {};
+    const int dev = current_device();
+    if (dev < 0 || dev >= 64) return false;
+    std::lock_guard<std::mutex> lock(mu);
+    if (bars[dev] == nullptr) {
+        void* b = nullptr;
+        void* q = nullptr;
+        if (cudaGetSymbolAddress(&b, g_oneshot_barrier) != cudaSuccess) return false;
+        if (cudaGetSymbolAddress(&q, g_oneshot_partials) != cudaSuccess) return false;
+        bars[dev] = static_cast<unsigned*>(b);
+        parts[dev] = static_cast<float*>(q);
+    }
+    *bar = bars[dev];
+    *part = parts[dev];
+    return true;
 }
 
 float* grid_partials() {
@@ -234,13 +263,33 @@ soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M,
     cudaStream_t s = as_stream(stream);
     const uint16_t* A16 = static_cast<const uint16_t*>(A);
     if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
-        cudaError_t e = launch_quantize_fused(geo, L->perm, A16, M, s_a, Ap, s);
+        cudaError_t e = launch_quantize_fused(geo, L->perm, A16, M, s_a, Ap, s, grid_barrier_word(), grid_partials(),
+                                              kMaxGridPartials);
         if (e == cudaSuccess) return SONIQ_OK;
         if (e != cudaErrorNotSupported) return cuda_status(e);
         e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);   // two passes: rows do not fit on chip
         if (e != cudaSuccess) return cuda_status(e);
     }
     return cuda_status(launch_quantize_act(geo, L->perm, A16, M, scale_mode, s_a, Ap, s));
+}
+
+soniq_status soniq_quantize_act_oneshot(const soniq_layout* L, const void* A, int64_t M, float* s_a, uint8_t* Ap,
+                                        soniq_stream_t stream) {
+    LayoutGeom geo;
+    soniq_status st = make_geom(L, 1, &geo);
+    if (st != SONIQ_OK) return st;
+    if (L->K > 32768) return SONIQ_ERR_UNSUPPORTED;
+    if (M < 0) return SONIQ_ERR_INVALID_ARG;
+    if (M == 0) return SONIQ_OK;
+    if (A == nullptr || s_a == nullptr || Ap == nullptr || L->perm == nullptr) return SONIQ_ERR_INVALID_ARG;
+    if (!aligned(A, 2) || !aligned(Ap, 4) || !aligned(s_a, 4)) return SONIQ_ERR_ALIGNMENT;
+    unsigned* bar = nullptr;
+    float* part = nullptr;
+    if (!oneshot_scratch(&bar, &part)) return SONIQ_ERR_CUDA;
+    const cudaError_t e = launch_quantize_fused(geo, L->perm, static_cast<const uint16_t*>(A), M, s_a, Ap,
+                                                as_stream(stream), bar, part, kOneShotMaxCtas);
+    if (e == cudaErrorNotSupported) return SONIQ_ERR_UNSUPPORTED;   // rows do not fit on chip: no fallback
+    return cuda_status(e);
 }
 
 soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float* s_a, int32_t scale_mode,

@@ -57,8 +57,12 @@ cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const 
 cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
                                 int64_t M, int32_t scale_mode, float* s_a, uint8_t* Ap,
                                 cudaStream_t st);
+// One-pass per-tensor quantize (cooperative launch); its grid barrier (two
+// words, zero between launches) and per-CTA maxima [max_ctas][2] are `bar` and
+// `part`.  cudaErrorNotSupported when the rows do not fit on chip.
 cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
-                                  float* s_a, uint8_t* Ap, cudaStream_t st);
+                                  float* s_a, uint8_t* Ap, cudaStream_t st, unsigned* bar, float* part,
+                                  int max_ctas);
 cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, const float* W,
                                  int32_t N, float* s_out, cudaStream_t st);
 cudaError_t launch_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W,

@@ -17,6 +17,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_lib", "libsoniq.so")
 
 SONIQ_OK = 0
+SONIQ_ERR_INVALID_ARG, SONIQ_ERR_UNSUPPORTED, SONIQ_ERR_ALIGNMENT, SONIQ_ERR_CUDA, SONIQ_ERR_TIMEOUT = 1, 2, 3, 4, 5
 STATUS_NAMES = {0: "SONIQ_OK", 1: "SONIQ_ERR_INVALID_ARG", 2: "SONIQ_ERR_UNSUPPORTED",
                 3: "SONIQ_ERR_ALIGNMENT", 4: "SONIQ_ERR_CUDA", 5: "SONIQ_ERR_TIMEOUT"}
 SCALE_PER_TENSOR, SCALE_PER_ROW, SCALE_CALIBRATED = 0, 1, 2
@@ -25,8 +26,8 @@ FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_TEST_DROP_ARRIVE = 1, 2, 0x100
 
 EXPORTED = ["soniq_abi_version", "soniq_status_string", "soniq_group_codes",
             "soniq_packed_row_bytes", "soniq_validate_layout", "soniq_launch_count",
-            "soniq_pack_weights", "soniq_quantize_act", "soniq_mp_gemm", "soniq_mp_conv2d",
-            "soniq_sync_status"]
+            "soniq_pack_weights", "soniq_quantize_act", "soniq_quantize_act_oneshot", "soniq_mp_gemm",
+            "soniq_mp_conv2d", "soniq_sync_status"]
 
 _SCALE = {"tensor": SCALE_PER_TENSOR, "row": SCALE_PER_ROW, "calibrated": SCALE_CALIBRATED}
 
@@ -76,6 +77,8 @@ def lib() -> ctypes.CDLL:
         L.soniq_pack_weights.restype = i32
         L.soniq_quantize_act.argtypes = [P, P, i64, i32, P, P, P]
         L.soniq_quantize_act.restype = i32
+        L.soniq_quantize_act_oneshot.argtypes = [P, P, i64, P, P, P]
+        L.soniq_quantize_act_oneshot.restype = i32
         L.soniq_mp_gemm.argtypes = [P, P, P, i32, i64, P, P, i32, P, i32, P, u32, P]
         L.soniq_mp_gemm.restype = i32
         L.soniq_mp_conv2d.argtypes = [P, P, P, P, i32, P, P, P, i32, P, u32, P]
@@ -177,6 +180,21 @@ def quantize_act(layout: Layout, A: torch.Tensor, scale_mode: str = "tensor",
         Ap = torch.empty((M, layout.row_bytes(False)), dtype=torch.uint8, device=A.device)
     _check(lib().soniq_quantize_act(ctypes.byref(layout.c), _ptr(A), M, mode, _ptr(s_a), _ptr(Ap),
                                     _stream(stream)), "soniq_quantize_act")
+    return Ap, s_a
+
+
+def quantize_act_oneshot(layout: Layout, A: torch.Tensor, s_a: Optional[torch.Tensor] = None,
+                         Ap: Optional[torch.Tensor] = None, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """soniq_quantize_act_oneshot: per-tensor quantize with fixed library scratch
+    (no allocation, no two-pass fallback; oversize inputs raise)."""
+    _need(A, torch.float16, "A")
+    M = A.shape[0]
+    if s_a is None:
+        s_a = torch.empty((2,), dtype=torch.float32, device=A.device)
+    if Ap is None:
+        Ap = torch.empty((M, layout.row_bytes(False)), dtype=torch.uint8, device=A.device)
+    _check(lib().soniq_quantize_act_oneshot(ctypes.byref(layout.c), _ptr(A), M, _ptr(s_a), _ptr(Ap),
+                                            _stream(stream)), "soniq_quantize_act_oneshot")
     return Ap, s_a
 
 
