@@ -32,6 +32,10 @@ import numpy as np  # noqa: E402
 
 METRIC = "mixed-precision GEMM effective TOPS (and GEMV GB/s) and % of roofline on 1 GB300"
 L2_FLUSH_BYTES = 256 << 20       # > 129 MB L2
+# dram__bytes_read.sum + dram__bytes_write.sum of one mp_mma_kernel launch on the
+# default conv workload, from an ncu capture of `python bench.py --case conv_4b8b`
+# (to be reset to None whenever the kernel changes after that capture)
+CONV_TRAFFIC_BYTES = 2990336.0
 
 
 def peaks():
@@ -502,8 +506,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--case", default=None, help="profile one kernel family on one workload")
-    ap.add_argument("--traffic", type=float, default=None,
-                    help="DRAM bytes per conv launch from an ncu capture of the same kernel")
+    ap.add_argument("--traffic", type=float, default=CONV_TRAFFIC_BYTES,
+                    help="DRAM bytes per conv launch from an ncu capture of the current kernel")
     args = ap.parse_args()
     if args.case:
         run_case(args)
