@@ -35,7 +35,7 @@ L2_FLUSH_BYTES = 256 << 20       # > 129 MB L2
 # dram__bytes_read.sum + dram__bytes_write.sum of one mp_mma_kernel launch on the
 # default conv workload, from an ncu capture of `python bench.py --case conv_4b8b`
 # (to be reset to None whenever the kernel changes after that capture)
-CONV_TRAFFIC_BYTES = 2990336.0
+CONV_TRAFFIC_BYTES = None
 
 
 def peaks():

@@ -1109,6 +1109,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
                 if (lane == 0) mbar_arrive(bar(BAR_SLOT_FREE + (i & 1)));
             }
         }
+    }
+
+    // ------------------------------------------------------------- epilogue
+    // Every warp but the MMA warp: warp w reads TMEM lanes 32*(w%4).. (its
+    // quadrant of rows) and columns 32*((w-1)/4) .. +31, so the four warps of
+    // each quadrant (one per role) share the tile's columns.
+    // (With a segmented group the int32 sum is written by the epilogue warps'
+    // drains, so they alone finish the tile, all columns, after their last drain.)
+    const bool shared_epi = p.seg_group < 0;
+    if (warp != WARP_MMA && (shared_epi || warp >= WARP_EPI)) {
+        const int quad = warp & 3;                 // TMEM lanes 32*quad .. +31
+        const int row = quad * 32 + lane;
+        const int cc0 = shared_epi ? 2 * ((warp - 1) >> 2) : 0;   // first 16-column block of this warp
+        const int cc1 = shared_epi ? cc0 + 2 : BN / 16;
+        const uint32_t lane_base = tmem_base + ((uint32_t)(quad * 32) << 16);
+        const int gs = p.seg_group;
+        bool ok = true;
         // warp-uniform outcomes: the TMEM loads below are .sync.aligned
         if (ok) ok = __all_sync(0xffffffffu, wait_bounded(bar(BAR_ACC_FULL), 0, abort_flag, p));
         if (ok) ok = __all_sync(0xffffffffu, wait_bounded(bar(BAR_ROWSUM), 0, abort_flag, p));
@@ -1126,7 +1143,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) mp_mma_kernel(const __grid_con
 #pragma unroll
             for (int g = 0; g < 2; ++g) col[g] = g == gs ? 3 * BN : p.acc_col[g];
 #pragma unroll 1
-            for (int cc = 0; cc < BN / 16; ++cc) {
+            for (int cc = cc0; cc < cc1; ++cc) {
                 int32_t acc[2][16];
                 uint32_t v[2][16];
                 tmem_ld16x2(lane_base + col[0] + cc * 16, lane_base + col[1] + cc * 16, v[0], v[1]);
