@@ -524,33 +524,20 @@ __device__ __forceinline__ void halo_tap(const Params& p, HaloRow& hr, int taps)
 }
 
 // This row's 4 blocks of the next chunk (n words each, block i at w[n*i]),
-// read from the halo; taps outside the image read code 0.
+// read from the halo; taps outside the image read code 0.  The tap
+// bookkeeping for the four blocks runs first, then all loads issue back to
+// back (a tap outside the image loads from the halo base and is zeroed).
 template <int N>
 __device__ __forceinline__ void read_halo(const Params& p, const Group& G, HaloRow& hr, uint32_t* w) {
     const int taps = p.R * p.S;
     const int cpt = G.pa >> 5;
     const bool vec = N % 4 == 0 && ((hr.base + (uint32_t)G.a_off) & 15u) == 0;
+    uint32_t addr[4];
+    bool in[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const uint32_t a = hr.addr + (uint32_t)G.a_off + (uint32_t)(hr.cb * 4 * N);
-        if (hr.in) {
-            if (vec) {
-#pragma unroll
-                for (int j = 0; j < (N & ~3); j += 4) {
-                    const uint4 v = lds128(a + 4 * j);
-                    w[N * i + j] = v.x;
-                    w[N * i + j + 1] = v.y;
-                    w[N * i + j + 2] = v.z;
-                    w[N * i + j + 3] = v.w;
-                }
-            } else {
-#pragma unroll
-                for (int j = 0; j < N; ++j) w[N * i + j] = lds32(a + 4 * j);
-            }
-        } else {
-#pragma unroll
-            for (int j = 0; j < N; ++j) w[N * i + j] = 0u;
-        }
+        in[i] = hr.in;
+        addr[i] = hr.in ? hr.addr + (uint32_t)G.a_off + (uint32_t)(hr.cb * 4 * N) : hr.base;
         if (++hr.cb == cpt) {
             hr.cb = 0;
             ++hr.tap;
@@ -560,6 +547,26 @@ __device__ __forceinline__ void read_halo(const Params& p, const Group& G, HaloR
             }
             halo_tap(p, hr, taps);
         }
+    }
+    if (vec) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < (N & ~3); j += 4) {
+                const uint4 v = lds128(addr[i] + 4 * j);
+                w[N * i + j] = in[i] ? v.x : 0u;
+                w[N * i + j + 1] = in[i] ? v.y : 0u;
+                w[N * i + j + 2] = in[i] ? v.z : 0u;
+                w[N * i + j + 3] = in[i] ? v.w : 0u;
+            }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < N; ++j) {
+                const uint32_t v = lds32(addr[i] + 4 * j);
+                w[N * i + j] = in[i] ? v : 0u;
+            }
     }
 }
 
