@@ -35,7 +35,7 @@ L2_FLUSH_BYTES = 256 << 20       # > 129 MB L2
 # dram__bytes_read.sum + dram__bytes_write.sum of one mp_mma_kernel launch on the
 # default conv workload, from an ncu capture of `python bench.py --case conv_4b8b`
 # (to be reset to None whenever the kernel changes after that capture)
-CONV_TRAFFIC_BYTES = None
+CONV_TRAFFIC_BYTES = 2994176.0
 
 
 def peaks():
@@ -165,16 +165,17 @@ def run_gpu(args):
     side = torch.cuda.Stream()
     side.wait_stream(stream)
     n0 = sq.launch_count()
-    g_quant, g_conv = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    g_step, g_quant, g_conv = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_step, stream=side):
+        step()
+    launches_per_step = sq.launch_count() - n0
     with torch.cuda.graph(g_quant, stream=side):
         sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp)
     with torch.cuda.graph(g_conv, stream=side):
         sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y)
-    launches_per_step = sq.launch_count() - n0
     for _ in range(max(args.warmup, 3)):
         flush.zero_()
-        g_quant.replay()
-        g_conv.replay()
+        g_step.replay()
     torch.cuda.synchronize()
 
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
@@ -187,11 +188,9 @@ def run_gpu(args):
     torch.cuda.synchronize()
     for i in range(args.steps):
         flush.zero_()                       # L2 flushed between timed steps (outside the events)
-        a, b, c = ev[i]
+        a, _, c = ev[i]
         a.record(stream)
-        g_quant.replay()
-        b.record(stream)
-        g_conv.replay()
+        g_step.replay()
         c.record(stream)
     torch.cuda.synchronize()
     launches = launches_per_step * args.steps
@@ -201,9 +200,18 @@ def run_gpu(args):
     if sq.sync_status() != 0:
         raise RuntimeError("device error during the timed steps")
     step_ms = [a.elapsed_time(c) for a, b, c in ev]
-    conv_ms = [b.elapsed_time(c) for a, b, c in ev]
-    quant_ms = [a.elapsed_time(b) for a, b, c in ev]
     total_ms = sum(step_ms)
+    # the two kernels alone, same flush and replay discipline (roofline of the conv)
+    conv_ms, quant_ms = [], []
+    for g, out in ((g_conv, conv_ms), (g_quant, quant_ms)):
+        for i in range(args.steps):
+            flush.zero_()
+            a, _, c = ev[i]
+            a.record(stream)
+            g.replay()
+            c.record(stream)
+        torch.cuda.synchronize()
+        out.extend(a.elapsed_time(c) for a, _, c in ev)
     if world > 1:
         t = torch.tensor([total_ms, sum(conv_ms)], dtype=torch.float64, device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -264,7 +272,7 @@ def run_gpu(args):
            "config": {"workload": spec.name, "M": spec.M, "N": spec.C_out, "K": spec.K,
                       "bits": d["bits"], "count": d["count"], "parallelism": f"replicas{world}",
                       "l2": "flushed between timed steps (256 MB write)",
-                      "launch": "each library call replayed as a CUDA graph (e2e: plain API calls)"},
+                      "launch": "the step (both library calls) replayed as one CUDA graph; e2e: plain API calls"},
            "e2e": {"value": round(e2e_value, 3), "unit": "TOPS",
                    "h2d_bytes_per_step": int(Xh.numel() * 2), "d2h_bytes_per_step": int(Yh.numel() * 2),
                    "ms_per_step": round(e2e_ms, 5)},
