@@ -544,9 +544,15 @@ __global__ void __launch_bounds__(kBulkThreads, 1) gemv_bulk_kernel(const GemvPa
 
         // tasks in piece order; a half-warp waits for a piece's barrier before its first task there
         const int half = threadIdx.x >> 4, nhalf = blockDim.x >> 4, r = threadIdx.x & 15;
+        const int dpiece = nhalf / tpp, dj = nhalf - dpiece * tpp;   // task t -> (piece, j), stepped by nhalf
         int waited = -1;
-        for (int t = half; t < npieces * tpp && ok; t += nhalf) {
-            const int piece = t / tpp, j = t - piece * tpp;
+        int piece = half / tpp, j = half - (half / tpp) * tpp;
+        for (; piece < npieces && ok; piece += dpiece, j += dj) {
+            if (j >= tpp) {
+                j -= tpp;
+                ++piece;
+                if (piece >= npieces) break;
+            }
             if (piece != waited) {
                 ok = gemv_wait(smem_addr(smem + p.bar_off + 8 * piece), (uint32_t)(round & 1), p);
                 waited = piece;
