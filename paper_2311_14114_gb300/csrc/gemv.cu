@@ -5,13 +5,13 @@
 // integer dot products):
 //   * each CTA expands the activation codes (M rows) once into shared memory
 //     as bytes, with their per-group row sums R_g[m];
-//   * weight rows are contiguous in HBM, so a CTA pulls a batch of rows with
-//     bulk TMA copies into one of two shared-memory buffers while its warps
-//     work on the other (the memory system sees a few large requests per
-//     SM, not one small load per lane);
-//   * a warp takes one row at a time; lane l expands the 128-code chunks l,
-//     l+32, ... of each group to bytes, flips the sign bit (j -> j + 2^(n-1),
-//     unsigned) and accumulates dp4a(u, j + 2^(n-1)) in uint32;
+//   * weight rows are contiguous in HBM and arrive by bulk copies (one per
+//     row) into shared memory: gemv_bulk_kernel (M <= 2) requests all of an
+//     SM's rows at once, gemv_kernel (M <= 16) streams batches of 32 rows
+//     through two buffers;
+//   * the sign bit of every weight code is flipped (j -> j + 2^(n-1),
+//     unsigned) and dp4a(u, j + 2^(n-1)) accumulates in uint32, from the
+//     packed slices directly (M <= 2) or from codes expanded to bytes;
 //   * Acc_g = sum - 2^(n-1) * R_g[m], exact; the fp32 epilogue applies the
 //     group scales (decode rules of Sec. 3 steps 2-3).
 #include <cuda_bf16.h>
