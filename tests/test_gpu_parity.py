@@ -267,6 +267,17 @@ def test_gemv_row_scales_pad32(sq):
     check_linear(sq, d, pad=32, act_mode="row", what="gemv row scales")
 
 
+@pytest.mark.parametrize("M", [1, 2])
+@pytest.mark.parametrize("K,N,bits", [
+    (32768, 2000, (6, 8)),   # 24+ KB rows: a CTA's rows run in several rounds through shared memory
+    (4096, 7, (3, 6)),       # fewer rows than one 16-row piece
+    (1000, 2431, (1, 5)),    # ragged pieces and a ragged last CTA, pad 32
+])
+def test_gemv_bulk_rounds_and_ragged_pieces(sq, M, K, N, bits):
+    d = wl.random_linear(700 + M + N, M=M, K=K, N=N, bits_lo=bits[0], bits_hi=bits[1], frac_hi=0.3)
+    check_linear(sq, d, pad=32 if K == 1000 else 128, what=f"gemv M={M} K={K} N={N}")
+
+
 def test_gemv_matches_mma(sq):
     d = wl.random_linear(301, M=16, K=768, N=256, bits_lo=3, bits_hi=6, frac_hi=0.15)
     a = run_linear(sq, d, flags=1)
