@@ -448,6 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvParams p) {
 // are conflict-free and activation reads are broadcasts) as soon as their
 // piece has landed, and adds its partial sums into per-row shared totals.
 constexpr int kBulkThreads = 1024;
+constexpr int kBulkMaxM = 4;
 constexpr int kPieceRows = 16;
 constexpr int kMaxPieces = 8;
 
@@ -611,6 +612,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) gemv_bulk_kernel(const GemvPa
 // the round's weight rows.  Rows per CTA: N over the SMs; rows per round: as
 // many as fit (at most kMaxPieces pieces).
 size_t gemv_bulk_smem(const LayoutGeom& geo, int64_t M, int64_t N, GemvParams* p) {
+    const int64_t mt = M <= 1 ? 1 : (M <= 2 ? 2 : 4);   // per-row totals held per activation row
     int64_t ws = geo.w_row_bytes;
     if ((ws / 16) % 2 == 0) ws += 16;
     p->wstride = (int32_t)ws;
@@ -624,11 +626,11 @@ size_t gemv_bulk_smem(const LayoutGeom& geo, int64_t M, int64_t N, GemvParams* p
     const size_t budget = 200 * 1024;
     int64_t round = rows_cta < kPieceRows * kMaxPieces ? rows_cta : kPieceRows * kMaxPieces;
     const size_t fixed = 128 + (size_t)8 * rows_cta + 16 + 8 * kMaxPieces + 16 + a_bytes + 16 * 2 + 128;
-    while (round > 1 && fixed + (size_t)2 * 2 * round * 4 + (size_t)round * ws > budget) --round;
+    while (round > 1 && fixed + (size_t)2 * mt * round * 4 + (size_t)round * ws > budget) --round;
     p->max_batches = (int32_t)rows_cta;
     p->batch_rows = (int32_t)round;
     p->sum_off = (int32_t)o;
-    o += (size_t)2 * 2 * round * 4;
+    o += (size_t)2 * mt * round * 4;
     o = (o + 15) & ~(size_t)15;
     p->scale_off = (int32_t)o;
     o += (size_t)2 * rows_cta * 4;
@@ -715,7 +717,7 @@ cudaError_t run(const GemvParams& p, size_t smem, cudaStream_t st) {
 bool gemv_supported(const LayoutGeom& geo, int64_t M, int64_t N) {
     GemvParams p;
     if (M < 1 || M > 16 || geo.w_row_bytes % 16 != 0) return false;
-    if (M <= 2) return gemv_bulk_smem(geo, M, N, &p) <= 210 * 1024;
+    if (M <= kBulkMaxM) return gemv_bulk_smem(geo, M, N, &p) <= 210 * 1024;
     return gemv_smem(geo, M, N, &p) <= 220 * 1024;
 }
 
@@ -740,9 +742,11 @@ cudaError_t launch_gemv(const LayoutGeom& geo, const GemvArgs& a, cudaStream_t s
     p.err = device_error_word();
     if (p.err == nullptr) return cudaErrorUnknown;
     p.timeout_ns = 2000000000LL;
-    if (a.M <= 2) {
+    if (a.M <= kBulkMaxM) {
         const size_t smem = gemv_bulk_smem(geo, a.M, a.N, &p);
-        return a.M == 1 ? run_bulk<1>(p, smem, st) : run_bulk<2>(p, smem, st);
+        if (a.M == 1) return run_bulk<1>(p, smem, st);
+        if (a.M == 2) return run_bulk<2>(p, smem, st);
+        return run_bulk<4>(p, smem, st);
     }
     const size_t smem = gemv_smem(geo, a.M, a.N, &p);
     if (a.M <= 4) return run<4>(p, smem, st);
