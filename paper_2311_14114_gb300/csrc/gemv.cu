@@ -5,10 +5,9 @@
 // integer dot products):
 //   * each CTA expands the activation codes (M rows) once into shared memory
 //     as bytes, with their per-group row sums R_g[m];
-//   * weight rows are contiguous in HBM and arrive by bulk copies (one per
-//     row) into shared memory: gemv_bulk_kernel (M <= 2) requests all of an
-//     SM's rows at once, gemv_kernel (M <= 16) streams batches of 32 rows
-//     through two buffers;
+//   * weight rows are contiguous in HBM; each SM takes a contiguous range of
+//     them and requests all of it at once, one bulk copy per row into shared
+//     memory (in rounds if the range does not fit);
 //   * the sign bit of every weight code is flipped (j -> j + 2^(n-1),
 //     unsigned) and dp4a(u, j + 2^(n-1)) accumulates in uint32, from the
 //     packed slices directly (M <= 2) or from codes expanded to bytes;
@@ -36,14 +35,13 @@ struct GemvParams {
     GroupGeom g[2];
     int32_t a_s_off[2];   // byte offset of group g's activation bytes in shared memory
     int32_t a_m_stride[2];// bytes per activation row of group g in shared memory
-    int32_t sum_off;      // per-row integer sums of a batch [batch_rows][2][MT]
-    int32_t scale_off;    // activation scales [16][2], then weight scales [max_batches][32][2]
-    int32_t max_batches;  // batches per CTA at most
-    int32_t bar_off;      // two mbarriers
-    int32_t buf_off;      // two weight buffers of buf_bytes
-    int32_t buf_bytes;
-    int32_t batch_rows;   // weight rows per batch (<= 32: lane = row)
-    int32_t wstride;      // bytes between weight rows in a buffer
+    int32_t sum_off;      // per-row totals of a round [2][MT][round_rows]
+    int32_t scale_off;    // weight scales of a round [round_rows][2]
+    int32_t rows_cta;     // weight rows per CTA (the last CTA may have fewer)
+    int32_t round_rows;   // weight rows per round through shared memory
+    int32_t bar_off;      // one mbarrier per 16-row piece of a round
+    int32_t buf_off;      // the round's weight rows
+    int32_t wstride;      // bytes between weight rows in the buffer
     unsigned* err;        // device error word (a bounded wait ran out)
     long long timeout_ns;
 };
@@ -52,17 +50,9 @@ struct GemvParams {
 // padding per chunk put the chunks of consecutive lanes on different banks.
 constexpr int A_CHUNK = 144;
 
-constexpr int kThreads = 512;
-
 __device__ __forceinline__ uint4 lds128(uint32_t addr) {
     uint4 v;
     asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
-    return v;
-}
-
-__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
-    uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
     return v;
 }
 
@@ -72,23 +62,11 @@ __host__ __device__ constexpr uint32_t top_bit_mask(int w) {
     return w == 8 ? 0x80808080u : w == 4 ? 0x88888888u : w == 2 ? 0xAAAAAAAAu : 0xFFFFFFFFu;
 }
 
-// sum over a block of u * (w-bit slice field), the slice's w words at `sw`:
-// shifting slice word q right by w*k and masking each byte's low w bits gives
-// the fields of codes 4t..4t+3, t = q*(8/w) + k, next to activation word a[t].
-template <int W>
-__device__ __forceinline__ uint32_t slice_dot(const uint32_t* sw, const uint32_t* a, uint32_t acc) {
-    constexpr int PER = 8 / W;
-    constexpr uint32_t MASK = W == 8 ? 0xFFFFFFFFu : W == 4 ? 0x0F0F0F0Fu : W == 2 ? 0x03030303u : 0x01010101u;
-#pragma unroll
-    for (int q = 0; q < W; ++q)
-#pragma unroll
-        for (int k = 0; k < PER; ++k) acc = __dp4a((sw[q] >> (W * k)) & MASK, a[q * PER + k], acc);
-    return acc;
-}
-
-// The same sums without shifting the slice words: field position k of every
-// byte is masked in place, so s[k] collects 2^(W*k) times its products and is
-// shifted down once per chunk (exact: every term carries that factor).
+// Sum over a block of u * (w-bit slice field), the slice's w words at `sw`:
+// field k of every byte of slice word q belongs to codes 4t..4t+3 with
+// t = q*(8/w) + k, next to activation word a[t].  The field is masked in place
+// rather than shifted down, so s[k] collects 2^(w*k) times its products; the
+// caller shifts it down once per chunk (exact: every term carries that factor).
 template <int W>
 __device__ __forceinline__ void slice_dot_masked(const uint32_t* sw, const uint32_t* a, uint32_t (&s)[8 / W]) {
     constexpr int PER = 8 / W;
@@ -197,59 +175,6 @@ __device__ __forceinline__ void gemv_chunk(uint32_t wsrc, uint32_t a_s, int astr
     gemv_chunk_w<NW, MT>(w, a_s, astride, M, acc);
 }
 
-template <int MT>
-__device__ __forceinline__ void gemv_chunk_n(int nw, uint32_t wsrc, uint32_t a_s, int astride, int M,
-                                             uint32_t (&acc)[MT]) {
-    switch (nw) {
-        case 1: gemv_chunk<1, MT>(wsrc, a_s, astride, M, acc); break;
-        case 2: gemv_chunk<2, MT>(wsrc, a_s, astride, M, acc); break;
-        case 3: gemv_chunk<3, MT>(wsrc, a_s, astride, M, acc); break;
-        case 4: gemv_chunk<4, MT>(wsrc, a_s, astride, M, acc); break;
-        case 5: gemv_chunk<5, MT>(wsrc, a_s, astride, M, acc); break;
-        case 6: gemv_chunk<6, MT>(wsrc, a_s, astride, M, acc); break;
-        case 7: gemv_chunk<7, MT>(wsrc, a_s, astride, M, acc); break;
-        default: gemv_chunk<8, MT>(wsrc, a_s, astride, M, acc); break;
-    }
-}
-
-// Blocks kb0 .. kb0 + nb - 1 (nb < 4) of a final partial chunk, block by block.
-template <int NW, int MT>
-__device__ __forceinline__ void gemv_tail(uint32_t wgrp, uint32_t a_s, int astride, int M, int kb0, int nb,
-                                          uint32_t (&acc)[MT]) {
-    const uint32_t flip = sign_flip_mask(NW);
-    for (int kb = kb0; kb < kb0 + nb; ++kb) {
-        uint32_t w[NW], wb[8];
-#pragma unroll
-        for (int i = 0; i < NW; ++i) w[i] = lds32(wgrp + (uint32_t)(kb * 4 * NW + 4 * i));
-        block_to_bytes<NW>(w, wb);
-#pragma unroll
-        for (int m = 0; m < MT; ++m) {
-            if (m < M) {
-                const uint32_t aa = a_s + (uint32_t)(m * astride + (kb >> 2) * A_CHUNK + (kb & 3) * 32);
-                const uint4 x0 = lds128(aa), x1 = lds128(aa + 16);
-                const uint32_t a[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-                for (int t = 0; t < 8; ++t) acc[m] = __dp4a(wb[t] ^ flip, a[t], acc[m]);
-            }
-        }
-    }
-}
-
-template <int MT>
-__device__ __forceinline__ void gemv_tail_n(int nw, uint32_t wgrp, uint32_t a_s, int astride, int M,
-                                            int kb0, int nb, uint32_t (&acc)[MT]) {
-    switch (nw) {
-        case 1: gemv_tail<1, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-        case 2: gemv_tail<2, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-        case 3: gemv_tail<3, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-        case 4: gemv_tail<4, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-        case 5: gemv_tail<5, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-        case 6: gemv_tail<6, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-        case 7: gemv_tail<7, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-        default: gemv_tail<8, MT>(wgrp, a_s, astride, M, kb0, nb, acc); break;
-    }
-}
-
 __device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
 __device__ __forceinline__ bool gemv_wait(uint32_t bar, uint32_t parity, const GemvParams& p) {
@@ -272,172 +197,7 @@ __device__ __forceinline__ bool gemv_wait(uint32_t bar, uint32_t parity, const G
     }
 }
 
-// Rows [n0, n0 + nr) into buffer `buf`, one bulk copy per row (issued by the
-// lanes of warp 0) to rows `wstride` bytes apart; one transaction count on the
-// buffer's barrier, armed by lane 0 before any copy can complete.
-__device__ __forceinline__ void gemv_issue(const GemvParams& p, uint8_t* smem, int buf, int64_t n0, int nr,
-                                           int lane) {
-    const uint32_t bar = smem_addr(smem + p.bar_off + 8 * buf);
-    if (lane == 0) {
-        const uint32_t bytes = (uint32_t)nr * (uint32_t)p.w_row_bytes;
-        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-    }
-    __syncwarp();
-    const uint32_t dst = smem_addr(smem + p.buf_off + buf * p.buf_bytes);
-    for (int r = lane; r < nr; r += 32)
-        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                         dst + (uint32_t)(r * p.wstride)),
-                     "l"(p.Wp + (n0 + r) * p.w_row_bytes), "r"((uint32_t)p.w_row_bytes), "r"(bar)
-                     : "memory");
-}
-
-// A persistent grid, one CTA per SM.  Each CTA expands the activation codes
-// once, then walks batches of `batch_rows` (<= 32) weight rows, double
-// buffered.  In a batch, lane l of every warp owns row l and warp w takes
-// the 128-code chunks w, w + nwarps, ... of the row's two groups (all lanes
-// of a warp work on the same chunk, so activation reads are broadcasts);
-// the per-row sums meet in shared memory.
-template <int MT>
-__global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvParams p) {
-    extern __shared__ __align__(128) uint8_t smem[];
-    int32_t* rowsum = reinterpret_cast<int32_t*>(smem);                       // [2][16]
-    uint32_t* sums = reinterpret_cast<uint32_t*>(smem + p.sum_off);           // [batch_rows][2][MT]
-    float* sa_s = reinterpret_cast<float*>(smem + p.scale_off);               // [16][2] activation scales
-    float* sw_all = sa_s + 32;                                                // [batches of this CTA][64] weight scales
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-    const int nbatch = (p.N + p.batch_rows - 1) / p.batch_rows;
-    const int c0 = (p.g[0].pa + 127) / 128, c1 = (p.g[1].pa + 127) / 128;   // chunks per group (last may be partial)
-
-    if (threadIdx.x < 32) {
-        rowsum[threadIdx.x] = 0;
-        const int m = threadIdx.x >> 1, g = threadIdx.x & 1;
-        if (m < p.M) sa_s[threadIdx.x] = p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g);
-    }
-    for (int i = threadIdx.x; i < p.batch_rows * 2 * MT; i += blockDim.x) sums[i] = 0u;
-    // the weight scales of every batch this CTA will take, read once up front
-    for (int i = threadIdx.x; i < p.max_batches * 64; i += blockDim.x) {
-        const int k = i >> 6, j = i & 63;
-        const int64_t row = ((int64_t)blockIdx.x + (int64_t)k * gridDim.x) * p.batch_rows + (j >> 1);
-        if (j < 2 * p.batch_rows && row < p.N) sw_all[i] = __ldg(p.s_w + row * 2 + (j & 1));
-    }
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < 2; ++i)
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(smem + p.bar_off + 8 * i)) : "memory");
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    __syncthreads();
-    // the first batch streams in while the activations expand
-    if (warp == 0 && (int)blockIdx.x < nbatch) {
-        const int64_t n0 = (int64_t)blockIdx.x * p.batch_rows;
-        gemv_issue(p, smem, 0, n0, (int)(p.N - n0 < p.batch_rows ? p.N - n0 : p.batch_rows), lane);
-    }
-
-    // ---- expand the activation codes of all M rows into shared memory ----
-#pragma unroll
-    for (int g = 0; g < 2; ++g) {
-        const GroupGeom& G = p.g[g];
-        const int nblk = G.pa / 32;
-        uint8_t* a_s = smem + p.a_s_off[g];
-        for (int item = threadIdx.x; item < p.M * nblk; item += blockDim.x) {
-            const int m = item / nblk, kb = item - m * nblk;
-            const uint32_t* src = reinterpret_cast<const uint32_t*>(
-                p.Ap + (int64_t)m * p.a_row_bytes + G.a_off + kb * 4 * G.bits_a);
-            uint32_t w[8], o[8];
-            for (int i = 0; i < G.bits_a; ++i) w[i] = __ldg(src + i);
-            block_to_bytes_n(G.bits_a, w, o);
-            uint32_t s = 0;
-#pragma unroll
-            for (int t = 0; t < 8; ++t) s = __dp4a(o[t], 0x01010101u, s);
-            uint4* d = reinterpret_cast<uint4*>(a_s + m * p.a_m_stride[g] + (kb >> 2) * A_CHUNK + (kb & 3) * 32);
-            d[0] = make_uint4(o[0], o[1], o[2], o[3]);
-            d[1] = make_uint4(o[4], o[5], o[6], o[7]);
-            atomicAdd(&rowsum[g * 16 + m], (int32_t)s);
-        }
-    }
-    __syncthreads();
-
-    bool ok = true;
-    int it = 0;
-    for (int b = blockIdx.x; b < nbatch && ok; b += gridDim.x, ++it) {
-        const int buf = it & 1;
-        const int64_t n0 = (int64_t)b * p.batch_rows;
-        const int nr = (int)(p.N - n0 < p.batch_rows ? p.N - n0 : p.batch_rows);
-        // the other buffer was released by the __syncthreads that ended the previous batch
-        if (warp == 0 && b + (int)gridDim.x < nbatch) {
-            const int64_t n1 = (int64_t)(b + gridDim.x) * p.batch_rows;
-            gemv_issue(p, smem, buf ^ 1, n1, (int)(p.N - n1 < p.batch_rows ? p.N - n1 : p.batch_rows), lane);
-        }
-        ok = gemv_wait(smem_addr(smem + p.bar_off + 8 * buf), (uint32_t)((it >> 1) & 1), p);
-        if (__syncthreads_or(!ok)) break;
-        if (lane < nr) {
-            const uint32_t wrow = smem_addr(smem) + (uint32_t)(p.buf_off + buf * p.buf_bytes + lane * p.wstride);
-            uint32_t acc[2][MT];
-#pragma unroll
-            for (int g = 0; g < 2; ++g)
-#pragma unroll
-                for (int m = 0; m < MT; ++m) acc[g][m] = 0u;
-            for (int c = warp; c < c0 + c1; c += nwarps) {
-                const int g = c >= c0;
-                const GroupGeom& G = p.g[g];
-                const int cc = g ? c - c0 : c;
-                const uint32_t a_s = smem_addr(smem) + (uint32_t)(p.a_s_off[g] + cc * A_CHUNK);
-                const int left = G.pa - cc * 128;   // activation codes from this chunk on
-                if (left >= 128) {
-                    if (g) gemv_chunk_n<MT>(G.bits_w, wrow + G.w_off + cc * 16 * G.bits_w, a_s, p.a_m_stride[1], p.M, acc[1]);
-                    else gemv_chunk_n<MT>(G.bits_w, wrow + G.w_off + cc * 16 * G.bits_w, a_s, p.a_m_stride[0], p.M, acc[0]);
-                } else {
-                    // a final partial chunk: its blocks one by one (beyond pa the weights pair with no code)
-                    const uint32_t a0 = smem_addr(smem) + (uint32_t)p.a_s_off[g];
-                    if (g) gemv_tail_n<MT>(G.bits_w, wrow + G.w_off, a0, p.a_m_stride[1], p.M, cc * 4, left / 32, acc[1]);
-                    else gemv_tail_n<MT>(G.bits_w, wrow + G.w_off, a0, p.a_m_stride[0], p.M, cc * 4, left / 32, acc[0]);
-                }
-            }
-#pragma unroll
-            for (int g = 0; g < 2; ++g)
-#pragma unroll
-                for (int m = 0; m < MT; ++m)
-                    if (m < p.M && acc[g][m] != 0u) atomicAdd(&sums[(lane * 2 + g) * MT + m], acc[g][m]);
-        }
-        __syncthreads();
-        // epilogue: one thread per (row, m)
-        for (int t = threadIdx.x; t < nr * p.M; t += blockDim.x) {
-            const int r = t / p.M, m = t - r * p.M;
-            const int64_t n = n0 + r;
-            float y = 0.0f;
-#pragma unroll
-            for (int g = 0; g < 2; ++g) {
-                const GroupGeom& G = p.g[g];
-                uint32_t* sp = &sums[(r * 2 + g) * MT + m];
-                const uint32_t v = *sp;
-                *sp = 0u;
-                if (G.pa == 0) continue;
-                const int32_t off = 1 << (G.bits_w - 1);
-                const int32_t a = (int32_t)(v - (uint32_t)(off * rowsum[g * 16 + m]));
-                const float inv = 1.0f / ((float)((1 << G.bits_a) - 1) * (float)off);
-                const float sw = sw_all[it * 64 + r * 2 + g] * inv;
-                const float sa = sa_s[m * 2 + g];
-                y = g == 0 ? (sa * sw) * (float)a : fmaf(sa * sw, (float)a, y);
-                if (p.acc_dbg != nullptr) p.acc_dbg[((int64_t)g * p.M + m) * p.N + n] = a;
-            }
-            const int64_t idx = (int64_t)m * p.N + n;
-            if (p.out_bf16) reinterpret_cast<__nv_bfloat16*>(p.Y)[idx] = __float2bfloat16_rn(y);
-            else reinterpret_cast<__half*>(p.Y)[idx] = __float2half_rn(y);
-        }
-        __syncthreads();   // buffer and sums are free for the next batch
-    }
-    // copies still in flight (the abandoned batch and its prefetched successor)
-    // must land before the CTA exits
-    if (threadIdx.x == 0 && !ok) {
-        const int b = (int)blockIdx.x + it * (int)gridDim.x;
-        for (int j = 0; j < 2; ++j) {
-            const int k = it + j;
-            if (b + j * (int)gridDim.x < nbatch)
-                gemv_wait(smem_addr(smem + p.bar_off + 8 * (k & 1)), (uint32_t)((k >> 1) & 1), p);
-        }
-    }
-}
-
-// ---- GEMV for one or two activation rows: the whole share in flight at once --
+// ---- the whole share of the weight rows in flight at once ------------------
 //
 // One CTA per SM takes a contiguous range of weight rows.  At its start warp
 // 0 issues one bulk copy per row into shared memory (rows at an odd multiple
@@ -447,8 +207,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const GemvParams p) {
 // piece: half-warp h takes tasks h, h + 64, ... (lane = row, so weight reads
 // are conflict-free and activation reads are broadcasts) as soon as their
 // piece has landed, and adds its partial sums into per-row shared totals.
-constexpr int kBulkThreads = 1024;
-constexpr int kBulkMaxM = 4;
+constexpr int kBulkMaxM = 16;
+
+// 1024 threads (64 registers each) for up to four activation rows; 512 (128
+// registers) for more, whose per-row sums and expanded blocks need the room.
+template <int MT>
+constexpr int bulk_threads() { return MT <= 4 ? 1024 : 512; }
 constexpr int kPieceRows = 16;
 constexpr int kMaxPieces = 8;
 
@@ -469,13 +233,13 @@ __device__ __forceinline__ void bulk_task(const GemvParams& p, int g, int nw, ui
 }
 
 template <int MT>
-__global__ void __launch_bounds__(kBulkThreads, 1) gemv_bulk_kernel(const GemvParams p) {
+__global__ void __launch_bounds__(bulk_threads<MT>(), 1) gemv_bulk_kernel(const GemvParams p) {
     extern __shared__ __align__(128) uint8_t smem[];
     int32_t* rowsum = reinterpret_cast<int32_t*>(smem);                  // [2][16]
     uint32_t* acc_s = reinterpret_cast<uint32_t*>(smem + p.sum_off);     // [2][MT][round rows]
-    float* sw_s = reinterpret_cast<float*>(smem + p.scale_off);          // [rows of the CTA][2] weight scales
+    float* sw_s = reinterpret_cast<float*>(smem + p.scale_off);          // [round rows][2] weight scales
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int rows_cta = p.max_batches, round_rows = p.batch_rows;
+    const int rows_cta = p.rows_cta, round_rows = p.round_rows;
     const int64_t n_begin = (int64_t)blockIdx.x * rows_cta;
     const int64_t n_end = n_begin + rows_cta < p.N ? n_begin + rows_cta : p.N;
     const int nch0 = p.g[0].pw / 128, nch1 = p.g[1].pw / 128, tpp = nch0 + nch1;   // tasks per piece
@@ -487,7 +251,6 @@ __global__ void __launch_bounds__(kBulkThreads, 1) gemv_bulk_kernel(const GemvPa
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (threadIdx.x < 32) rowsum[threadIdx.x] = 0;
-    for (int i = threadIdx.x; i < 2 * (int)(n_end - n_begin); i += blockDim.x) sw_s[i] = __ldg(p.s_w + n_begin * 2 + i);
     __syncthreads();
 
     bool ok = true;
@@ -514,6 +277,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) gemv_bulk_kernel(const GemvPa
                     : "memory");
         }
         for (int i = threadIdx.x; i < 2 * MT * round_rows; i += blockDim.x) acc_s[i] = 0u;
+        for (int i = threadIdx.x; i < 2 * nr; i += blockDim.x) sw_s[i] = __ldg(p.s_w + n0 * 2 + i);
         if (round == 0) {
             // activation codes as bytes, chunk-padded, zero beyond PA up to the weights' PW
 #pragma unroll
@@ -587,7 +351,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) gemv_bulk_kernel(const GemvPa
                 const int32_t off = 1 << (G.bits_w - 1);
                 const int32_t a = (int32_t)(v - (uint32_t)(off * rowsum[g * 16 + m]));
                 const float inv = 1.0f / ((float)((1 << G.bits_a) - 1) * (float)off);
-                const float sw = sw_s[(n - n_begin) * 2 + g] * inv;
+                const float sw = sw_s[rr * 2 + g] * inv;
                 const float sa = p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g);
                 y = g == 0 ? (sa * sw) * (float)a : fmaf(sa * sw, (float)a, y);
                 if (p.acc_dbg != nullptr) p.acc_dbg[((int64_t)g * p.M + m) * p.N + n] = a;
@@ -612,7 +376,7 @@ __global__ void __launch_bounds__(kBulkThreads, 1) gemv_bulk_kernel(const GemvPa
 // the round's weight rows.  Rows per CTA: N over the SMs; rows per round: as
 // many as fit (at most kMaxPieces pieces).
 size_t gemv_bulk_smem(const LayoutGeom& geo, int64_t M, int64_t N, GemvParams* p) {
-    const int64_t mt = M <= 1 ? 1 : (M <= 2 ? 2 : 4);   // per-row totals held per activation row
+    const int64_t mt = M <= 1 ? 1 : (M <= 2 ? 2 : (M <= 4 ? 4 : (M <= 8 ? 8 : 16)));   // per-row totals per activation row
     int64_t ws = geo.w_row_bytes;
     if ((ws / 16) % 2 == 0) ws += 16;
     p->wstride = (int32_t)ws;
@@ -623,17 +387,20 @@ size_t gemv_bulk_smem(const LayoutGeom& geo, int64_t M, int64_t N, GemvParams* p
     size_t o = 128;
     size_t a_bytes = 0;
     for (int g = 0; g < 2; ++g) a_bytes += (size_t)M * (geo.g[g].pw / 128) * A_CHUNK;
-    const size_t budget = 200 * 1024;
+    const size_t budget = 222 * 1024;
+    // fixed: row sums, barriers, activations, alignment slack; per round row:
+    // its per-row totals, its two weight scales and its weight bytes
+    const size_t fixed = 128 + 8 * kMaxPieces + a_bytes + 4 * 16 + 128;
+    const size_t per_row = (size_t)2 * mt * 4 + 2 * 4 + (size_t)ws;
     int64_t round = rows_cta < kPieceRows * kMaxPieces ? rows_cta : kPieceRows * kMaxPieces;
-    const size_t fixed = 128 + (size_t)8 * rows_cta + 16 + 8 * kMaxPieces + 16 + a_bytes + 16 * 2 + 128;
-    while (round > 1 && fixed + (size_t)2 * mt * round * 4 + (size_t)round * ws > budget) --round;
-    p->max_batches = (int32_t)rows_cta;
-    p->batch_rows = (int32_t)round;
+    while (round > 1 && fixed + (size_t)round * per_row > budget) --round;
+    p->rows_cta = (int32_t)rows_cta;
+    p->round_rows = (int32_t)round;
     p->sum_off = (int32_t)o;
     o += (size_t)2 * mt * round * 4;
     o = (o + 15) & ~(size_t)15;
     p->scale_off = (int32_t)o;
-    o += (size_t)2 * rows_cta * 4;
+    o += (size_t)2 * round * 4;
     o = (o + 15) & ~(size_t)15;
     p->bar_off = (int32_t)o;
     o += 8 * kMaxPieces;
@@ -656,58 +423,8 @@ cudaError_t run_bulk(const GemvParams& p, size_t smem, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     e = prefer_max_shared((const void*)gemv_bulk_kernel<MT>);
     if (e != cudaSuccess) return e;
-    const int64_t grid = (p.N + p.max_batches - 1) / p.max_batches;
-    gemv_bulk_kernel<MT><<<(unsigned)grid, kBulkThreads, smem, st>>>(p);
-    note_launch();
-    return cudaGetLastError();
-}
-
-// Shared memory: row sums, chunk-padded activation bytes of both groups,
-// per-row sums of a batch, two barriers, two weight buffers.
-size_t gemv_smem(const LayoutGeom& geo, int64_t M, int64_t N, GemvParams* p) {
-    size_t o = 128;   // row sums [2][16]
-    for (int g = 0; g < 2; ++g) {
-        const int64_t chunks = (geo.g[g].pa + 127) / 128;
-        p->a_s_off[g] = (int32_t)o;
-        p->a_m_stride[g] = (int32_t)(chunks * A_CHUNK);
-        o += (size_t)M * chunks * A_CHUNK;
-        o = (o + 15) & ~(size_t)15;
-    }
-    // weight rows at an odd number of 16-byte units apart: lanes' 16-byte reads hit distinct banks
-    int64_t ws = geo.w_row_bytes;
-    if ((ws / 16) % 2 == 0) ws += 16;
-    p->wstride = (int32_t)ws;
-    int rows = (int)((60 * 1024) / ws);
-    if (rows > 32) rows = 32;
-    if (rows < 1) rows = 1;
-    p->batch_rows = rows;
-    p->sum_off = (int32_t)o;
-    o += (size_t)rows * 2 * 16 * 4;
-    p->scale_off = (int32_t)o;
-    const int64_t nbatch = (N + rows - 1) / rows;
-    const int64_t grid = nbatch < num_sms() ? nbatch : num_sms();
-    p->max_batches = (int32_t)((nbatch + grid - 1) / grid);
-    o += (32 + (size_t)p->max_batches * 64) * 4;
-    p->bar_off = (int32_t)o;
-    o += 16;
-    o = (o + 127) & ~(size_t)127;
-    p->buf_off = (int32_t)o;
-    p->buf_bytes = (int32_t)((rows * ws + 127) / 128 * 128);
-    return o + 2 * (size_t)p->buf_bytes;
-}
-
-template <int MT>
-cudaError_t run(const GemvParams& p, size_t smem, cudaStream_t st) {
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(gemv_kernel<MT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-    }
-    int grid = (p.N + p.batch_rows - 1) / p.batch_rows;
-    const int cap = num_sms();   // one CTA per SM (double-buffered batches)
-    if (grid > cap) grid = cap;
-    cudaError_t ec = prefer_max_shared((const void*)gemv_kernel<MT>);
-    if (ec != cudaSuccess) return ec;
-    gemv_kernel<MT><<<grid, kThreads, smem, st>>>(p);
+    const int64_t grid = (p.N + p.rows_cta - 1) / p.rows_cta;
+    gemv_bulk_kernel<MT><<<(unsigned)grid, bulk_threads<MT>(), smem, st>>>(p);
     note_launch();
     return cudaGetLastError();
 }
@@ -716,9 +433,8 @@ cudaError_t run(const GemvParams& p, size_t smem, cudaStream_t st) {
 
 bool gemv_supported(const LayoutGeom& geo, int64_t M, int64_t N) {
     GemvParams p;
-    if (M < 1 || M > 16 || geo.w_row_bytes % 16 != 0) return false;
-    if (M <= kBulkMaxM) return gemv_bulk_smem(geo, M, N, &p) <= 210 * 1024;
-    return gemv_smem(geo, M, N, &p) <= 220 * 1024;
+    if (M < 1 || M > kBulkMaxM || N < 1 || geo.w_row_bytes % 16 != 0) return false;
+    return gemv_bulk_smem(geo, M, N, &p) <= 224 * 1024;
 }
 
 cudaError_t launch_gemv(const LayoutGeom& geo, const GemvArgs& a, cudaStream_t st) {
@@ -742,16 +458,12 @@ cudaError_t launch_gemv(const LayoutGeom& geo, const GemvArgs& a, cudaStream_t s
     p.err = device_error_word();
     if (p.err == nullptr) return cudaErrorUnknown;
     p.timeout_ns = 2000000000LL;
-    if (a.M <= kBulkMaxM) {
-        const size_t smem = gemv_bulk_smem(geo, a.M, a.N, &p);
-        if (a.M == 1) return run_bulk<1>(p, smem, st);
-        if (a.M == 2) return run_bulk<2>(p, smem, st);
-        return run_bulk<4>(p, smem, st);
-    }
-    const size_t smem = gemv_smem(geo, a.M, a.N, &p);
-    if (a.M <= 4) return run<4>(p, smem, st);
-    if (a.M <= 8) return run<8>(p, smem, st);
-    return run<16>(p, smem, st);
+    const size_t smem = gemv_bulk_smem(geo, a.M, a.N, &p);
+    if (a.M == 1) return run_bulk<1>(p, smem, st);
+    if (a.M == 2) return run_bulk<2>(p, smem, st);
+    if (a.M <= 4) return run_bulk<4>(p, smem, st);
+    if (a.M <= 8) return run_bulk<8>(p, smem, st);
+    return run_bulk<16>(p, smem, st);
 }
 
 }  // namespace soniq
