@@ -372,6 +372,7 @@ def run_suite(args, sq, wl, pk, flush):
              "pack_weights_us": round(pack_ms * 1e3, 2)}
         if kind == "gemv":
             moved = Wp.numel() + s_w.numel() * 4
+            r["path"] = "CUDA-core GEMV" if spec.M <= 12 else "tensor-core kernel"
             r["gemv_GBps_algorithmic"] = round(wbytes / (gemm_ms * 1e-3) / 1e9, 1)
             r["frac_hbm"] = round(wbytes / (gemm_ms * 1e-3) / 1e9 / pk["hbm"], 4)
             r["weight_bytes_moved"] = int(moved)

@@ -211,9 +211,9 @@ SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, co
  * integer dot products):
  *   Acc_g[m][n] = sum over k in group g of u[m][k] * j[n][k]   (exact int32)
  *   Y[m][n]     = sum_g s_a(m,g) * s_w[n][g] / ((2^na_g - 1) * 2^(nw_g - 1)) * Acc_g[m][n]
- * computed in fp32 and rounded to nearest fp16 (or bf16).  M <= 16 runs a
+ * computed in fp32 and rounded to nearest fp16 (or bf16).  M <= 12 runs a
  * bandwidth-bound CUDA-core GEMV, larger M the tcgen05 tensor-core kernel
- * (flags can force either).
+ * (flags can force either; the GEMV takes M <= 16).
  *
  *   Ap, s_a    from soniq_quantize_act with the same layout (pad_unit 32 or 128);
  *              s_a [2] (PER_TENSOR / CALIBRATED) or [M][2] (PER_ROW).

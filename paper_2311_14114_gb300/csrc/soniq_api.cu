@@ -311,7 +311,9 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     // K <= 65536 keeps |Acc| < 2^31 and the GEMV's unsigned offset sums below 2^32
     const int per_row = scale_mode == SONIQ_SCALE_PER_ROW;
     cudaStream_t s = as_stream(stream);
-    const bool want_gemv = (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= 16 && !(flags & SONIQ_FLAG_FORCE_MMA));
+    // up to 12 rows the CUDA-core GEMV is faster; from 13 the tensor-core kernel (whose time hardly
+    // grows with M below 128) overtakes it (decode N=11008, K=4096: 47.6 vs 41.5 us at M=16)
+    const bool want_gemv = (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= 12 && !(flags & SONIQ_FLAG_FORCE_MMA));
     if (want_gemv && gemv_supported(geo, M, N)) {
         GemvArgs a{Ap, Wp, s_a, s_w, Y, acc_dbg, (int32_t)M, N, per_row, out_dtype == SONIQ_OUT_BF16};
         return cuda_status(launch_gemv(geo, a, s));
