@@ -262,6 +262,14 @@ def test_gemv(sq, M, bits):
     check_linear(sq, d, what=f"gemv M={M}")
 
 
+@pytest.mark.parametrize("M,flags", [(12, 0), (13, 0), (13, 1), (16, 1)])
+def test_gemv_dispatch_threshold_and_forced(sq, M, flags):
+    """Both sides of the GEMV / tensor-core dispatch threshold with default flags,
+    and the GEMV forced above it, against the oracle (bytes, accumulators, fp16)."""
+    d = wl.random_linear(210 + M, M=M, K=1000, N=333, bits_lo=3, bits_hi=6, frac_hi=0.15, n_outliers=2)
+    check_linear(sq, d, flags=flags, what=f"gemv M={M} flags={flags}")
+
+
 def test_gemv_row_scales_pad32(sq):
     d = wl.random_linear(300, M=5, K=700, N=99, bits_lo=2, bits_hi=8, frac_hi=0.2)
     check_linear(sq, d, pad=32, act_mode="row", what="gemv row scales")
@@ -378,6 +386,18 @@ def test_full_mlp_up(sq):
 def test_full_decode(sq, M):
     d = wl.make_linear(wl.DECODE[M])
     check_linear(sq, d, what=wl.DECODE[M].name)
+
+
+SWEEP_POINTS = [(s.bits_lo, s.bits_hi, s.frac_hi) for s in wl.sweep_specs()]
+
+
+@pytest.mark.parametrize("lo,hi,frac", SWEEP_POINTS, ids=lambda v: str(v))
+def test_sweep_every_point_full_k(sq, lo, hi, frac):
+    """Every (low bits, high bits, high fraction) point of the precision sweep at
+    its full K = N = 4096, on 256 activation rows; sampled rows against the oracle."""
+    spec = wl.LinearSpec("sweep", M=8192, K=4096, N=4096, bits_lo=lo, bits_hi=hi, frac_hi=frac)
+    d = wl.make_linear(spec, M=256)
+    check_linear(sq, d, rows=_sample_rows(256, 24, 4), what=f"sweep lo{lo} hi{hi} f{frac}")
 
 
 @pytest.mark.parametrize("lo,hi,frac", [(1, 8, 1.0), (2, 4, 0.1), (3, 6, 0.5), (4, 8, 0.25)])
