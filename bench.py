@@ -1,22 +1,29 @@
 #!/usr/bin/env python3
 """Benchmark of SONIQ's inference hot path on GB300.
 
-Default workload: the ResNet-18-shaped 3x3 convolution (batch 64, 14x14x256 ->
-256, 70% of input channels at 4 bits and 30% at 8 bits) run as implicit GEMM.
-One step = one pass of the per-inference path over the batch:
-    soniq_quantize_act (max-abs scale + quantize + pack the NHWC input)
-    soniq_mp_conv2d    (tcgen05 implicit GEMM + fused scale epilogue)
-Weights are packed once before timing (offline, Sec. 3: the layout is fixed
-after training).  The metric is effective TOPS = 2 * M * N * K / step time
-with the logical (unpadded) K = 9 * 256.
+Headline workload: the precision-sweep GEMM M=8192, K=N=4096 at the point
+4-bit low / 8-bit high / 25 % high channels (1024 of 4096 channels at 8 bits),
+activations fp16 ~N(0,1), weights ~N(0, 0.02).  One step = one pass of the
+per-inference path over the batch:
+    soniq_quantize_act (per-tensor max-abs scale + quantize + pack, Sec. 3 steps 1-2)
+    soniq_mp_gemm      (exact integer products per precision group + scale epilogue)
+Weights are packed once before timing (offline: the layout is fixed after
+training).  The metric is effective TOPS = 2 * M * N * K / step time with the
+logical (unpadded) K.
 
---suite adds the other workload families (linear, MLP up-projection, decode
-GEMV, precision sweep) as a per-kernel table under "suite".
---impl reference times the CPU oracle on bounded samples of the same workload.
+The default run also prints a "suite" with every other workload family: the
+small linear layer, the ResNet-18 conv (4/8 and 1/4 bits), the MLP
+up-projection, the decode GEMV (M = 1, 4, 16; GB/s of packed weights), the
+per-tensor quantize (GB/s) and all 60 points of the precision sweep, each as
+TOPS or GB/s and as a fraction of its roofline.
+
+--impl reference times the CPU oracle on the same workload (bounded samples,
+extrapolated to a full step as stated in its line).
 """
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
 import statistics
@@ -32,10 +39,11 @@ import numpy as np  # noqa: E402
 
 METRIC = "mixed-precision GEMM effective TOPS (and GEMV GB/s) and % of roofline on 1 GB300"
 L2_FLUSH_BYTES = 256 << 20       # > 129 MB L2
-# dram__bytes_read.sum + dram__bytes_write.sum of one mp_mma_kernel launch on the
-# default conv workload, from an ncu capture of `python bench.py --case conv_4b8b`
-# (to be reset to None whenever the kernel changes after that capture)
-CONV_TRAFFIC_BYTES = 2994176.0
+KERNEL_SOURCES = ("paper_2311_14114_gb300/csrc/mma_gemm.cu",)
+# dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant
+# kernel on the headline workload, from one ncu capture, keyed by the sha256 of
+# the kernel sources it was captured with: a different source reports null.
+TRAFFIC = {"sha256": None, "bytes": None, "capture": None}
 
 
 def peaks():
@@ -46,6 +54,19 @@ def peaks():
         return dict(hbm=float(d["hbm_gbs"]), bf16=float(d["bf16_tflops"]),
                     bf16_sus=float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), src="measured")
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+def kernel_sha():
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def headline_spec():
+    from paper_2311_14114_gb300 import workloads as wl
+    return wl.SWEEP_HEADLINE
 
 
 # --------------------------------------------------------------------------
@@ -105,19 +126,68 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------------------
-# the GPU arm
+# rooflines
 # --------------------------------------------------------------------------
 
-def conv_ops(spec, count):
-    """Logical integer ops per group: 2 * M * C_out * (R*S*count_g)."""
-    return [2 * spec.M * spec.C_out * spec.R * spec.S * c for c in count]
+def group_kinds(bits_a, bits_w):
+    """Tensor pipe of each group: 0 = E4M3 (codes <= 4 bits on both sides), 1 = fp16."""
+    return [0 if (a <= 4 and w <= 4) else 1 for a, w in zip(bits_a, bits_w)]
 
 
 def mixed_peak(ops, kinds, pk):
-    """Tensor peak for a step that runs ops[g] on the pipe of kinds[g]
-    (0: E4M3 at 2x the bf16 rate, 1: fp16 at the bf16 rate)."""
-    t = sum(o / (pk["bf16"] * (2.0 if k == 0 else 1.0)) for o, k in zip(ops, kinds))
+    """Tensor peak for work that runs ops[g] on the pipe of kinds[g] (E4M3 at
+    2x the measured bf16 rate, the nominal fp8:bf16 ratio; fp16 at the bf16
+    rate), time-weighted over the groups."""
+    t = sum(o / (pk["bf16"] * (2.0 if k == 0 else 1.0)) for o, k in zip(ops, kinds) if o > 0)
     return sum(ops) / t if t > 0 else pk["bf16"]
+
+
+def linear_ops(M, N, count):
+    return [2 * M * N * c for c in count]
+
+
+def quant_bytes(M, K, count, bits):
+    """Algorithmic bytes of an activation quantize: fp16 read + packed codes written."""
+    return M * K * 2 + M * sum(c * b for c, b in zip(count, bits)) / 8
+
+
+# --------------------------------------------------------------------------
+# the GPU arm
+# --------------------------------------------------------------------------
+
+def _graph(fn, stream):
+    import torch
+    side = torch.cuda.Stream()
+    side.wait_stream(stream)
+    with torch.cuda.stream(side):
+        fn()                                # scratch buffers of this stream exist before capture
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        fn()
+    return g
+
+
+def _time_graph(g, steps, flush, stream, warm=3):
+    """Per-replay device times (ms) of a captured graph; L2 flushed before each
+    replay, outside the events."""
+    import torch
+    for _ in range(warm):
+        flush.zero_()
+        g.replay()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for i in range(steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        g.replay()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    return [a.elapsed_time(b) for a, b in ev]
+
+
+def _time_fn(fn, steps, flush, stream):
+    """Median device time (ms) of a library call replayed as a CUDA graph."""
+    return statistics.median(_time_graph(_graph(fn, stream), steps, flush, stream))
 
 
 def run_gpu(args):
@@ -135,22 +205,26 @@ def run_gpu(args):
         dist.init_process_group("nccl")
     pk = peaks()
 
-    spec = wl.CONV_RESNET
-    d = wl.make_conv(spec)
-    lay = sq.Layout(d["perm"], d["count"], d["bits"], pad_unit=32)
+    spec = headline_spec()
+    d = wl.make_linear(spec)
+    lay = sq.Layout(d["perm"], d["count"], d["bits"])
     stream = torch.cuda.current_stream()
-    X = torch.from_numpy(d["X"]).cuda().reshape(-1, spec.C)
+    A = torch.from_numpy(d["A"]).cuda()
     Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
-    cd = sq.conv_desc(spec.batch, spec.H, spec.W, spec.C_out, spec.R, spec.S, spec.stride, spec.pad)
-    P, Q = sq.conv_out_hw(cd)
-    Xp = torch.empty((spec.batch * spec.H * spec.W, lay.row_bytes()), dtype=torch.uint8, device="cuda")
+    Ap = torch.empty((spec.M, lay.row_bytes()), dtype=torch.uint8, device="cuda")
     s_a = torch.empty(2, dtype=torch.float32, device="cuda")
-    Y = torch.empty((spec.batch, P, Q, spec.C_out), dtype=torch.float16, device="cuda")
+    Y = torch.empty((spec.M, spec.N), dtype=torch.float16, device="cuda")
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
 
+    def quant():
+        sq.quantize_act(lay, A, "tensor", s_a=s_a, Ap=Ap)
+
+    def gemm():
+        sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y)
+
     def step():
-        sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp)
-        sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y)
+        quant()
+        gemm()
 
     for _ in range(max(args.warmup, 3)):
         flush.zero_()
@@ -159,65 +233,35 @@ def run_gpu(args):
     if sq.sync_status() != 0:
         raise RuntimeError("device error during warm-up")
 
-    # The device-timed steps replay CUDA graphs of the two library calls (as a
-    # serving loop would), so host-side call overhead does not sit between the
+    # The device-timed steps replay a CUDA graph of the two library calls (as a
+    # serving loop would), so host call overhead does not sit between the
     # events; the end-to-end number below goes through the plain API calls.
-    side = torch.cuda.Stream()
-    side.wait_stream(stream)
     n0 = sq.launch_count()
-    g_step, g_quant, g_conv = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_step, stream=side):
-        step()
-    launches_per_step = sq.launch_count() - n0
-    with torch.cuda.graph(g_quant, stream=side):
-        sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp)
-    with torch.cuda.graph(g_conv, stream=side):
-        sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y)
-    for _ in range(max(args.warmup, 3)):
-        flush.zero_()
-        g_step.replay()
-    torch.cuda.synchronize()
+    g_step = _graph(step, stream)
+    launches_per_step = (sq.launch_count() - n0) // 2     # the call before capture and the captured one
+    g_quant, g_gemm = _graph(quant, stream), _graph(gemm, stream)
 
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    for i in range(args.steps):
-        flush.zero_()                       # L2 flushed between timed steps (outside the events)
-        a, _, c = ev[i]
-        a.record(stream)
-        g_step.replay()
-        c.record(stream)
-    torch.cuda.synchronize()
-    launches = launches_per_step * args.steps
+    step_ms = _time_graph(g_step, args.steps, flush, stream, warm=max(args.warmup, 3))
     if world > 1:
         dist.barrier()
     clk = clocks.stop()
     if sq.sync_status() != 0:
         raise RuntimeError("device error during the timed steps")
-    step_ms = [a.elapsed_time(c) for a, b, c in ev]
+    launches = launches_per_step * args.steps
+    # the two kernels alone, same flush and replay discipline
+    gemm_ms = _time_graph(g_gemm, args.steps, flush, stream)
+    quant_ms = _time_graph(g_quant, args.steps, flush, stream)
     total_ms = sum(step_ms)
-    # the two kernels alone, same flush and replay discipline (roofline of the conv)
-    conv_ms, quant_ms = [], []
-    for g, out in ((g_conv, conv_ms), (g_quant, quant_ms)):
-        for i in range(args.steps):
-            flush.zero_()
-            a, _, c = ev[i]
-            a.record(stream)
-            g.replay()
-            c.record(stream)
-        torch.cuda.synchronize()
-        out.extend(a.elapsed_time(c) for a, _, c in ev)
     if world > 1:
-        t = torch.tensor([total_ms, sum(conv_ms)], dtype=torch.float64, device="cuda")
+        t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, conv_total = float(t[0]), float(t[1])
-    else:
-        conv_total = sum(conv_ms)
+        total_ms = float(t[0])
     ms_per_step = total_ms / args.steps
     ops = spec.ops
     value = world * ops / (ms_per_step * 1e-3) / 1e12
@@ -228,10 +272,10 @@ def run_gpu(args):
     # neighbouring steps overlap this step's kernels: uploads, kernels and
     # downloads run on three streams with two sets of buffers.
     NB = 2
-    Xh = [torch.from_numpy(d["X"]).reshape(-1, spec.C).pin_memory() for _ in range(NB)]
-    Yh = [torch.empty((spec.batch, P, Q, spec.C_out), dtype=torch.float16).pin_memory() for _ in range(NB)]
-    Xd = [torch.empty_like(X) for _ in range(NB)]
-    Xpd = [torch.empty_like(Xp) for _ in range(NB)]
+    Ah = [torch.from_numpy(d["A"]).pin_memory() for _ in range(NB)]
+    Yh = [torch.empty((spec.M, spec.N), dtype=torch.float16).pin_memory() for _ in range(NB)]
+    Ad = [torch.empty_like(A) for _ in range(NB)]
+    Apd = [torch.empty_like(Ap) for _ in range(NB)]
     sad = [torch.empty_like(s_a) for _ in range(NB)]
     Yd = [torch.empty_like(Y) for _ in range(NB)]
     s_up, s_cmp, s_down = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
@@ -246,15 +290,15 @@ def run_gpu(args):
         k = i % NB
         with torch.cuda.stream(s_up):
             if used[k]:
-                s_up.wait_event(cmp_done[k])          # the kernels of step i - NB have read Xd[k]
-            Xd[k].copy_(Xh[k], non_blocking=True)
+                s_up.wait_event(cmp_done[k])          # the kernels of step i - NB have read Ad[k]
+            Ad[k].copy_(Ah[k], non_blocking=True)
             up_done[k].record(s_up)
         with torch.cuda.stream(s_cmp):
             s_cmp.wait_event(up_done[k])
             if used[k]:
                 s_cmp.wait_event(down_done[k])        # Yd[k] of step i - NB has been read back
-            sq.quantize_act(lay, Xd[k], "tensor", s_a=sad[k], Ap=Xpd[k], stream=s_cmp)
-            sq.mp_conv2d(lay, cd, Xpd[k], sad[k], Wp, s_w, Y=Yd[k], stream=s_cmp)
+            sq.quantize_act(lay, Ad[k], "tensor", s_a=sad[k], Ap=Apd[k], stream=s_cmp)
+            sq.mp_gemm(lay, Apd[k], sad[k], Wp, s_w, Y=Yd[k], stream=s_cmp)
             cmp_done[k].record(s_cmp)
         with torch.cuda.stream(s_down):
             s_down.wait_event(cmp_done[k])
@@ -280,132 +324,129 @@ def run_gpu(args):
         e2e_ms = float(t[0])
     e2e_value = world * ops / (e2e_ms * 1e-3) / 1e12
 
-    # ---- roofline of the dominant kernel (the implicit-GEMM conv) ----
-    conv_avg_ms = conv_total / args.steps
-    achieved = ops / (conv_avg_ms * 1e-3) / 1e12
-    kinds = [0 if b <= 4 else 1 for b in d["bits"]]
-    peak = mixed_peak(conv_ops(spec, d["count"]), kinds, pk)
-    roofline = {"kernel": "mp_mma_kernel (implicit-GEMM conv)", "bound": "tensor",
+    # ---- roofline of the dominant kernel (the tensor-core GEMM) ----
+    gemm_avg = statistics.mean(gemm_ms)
+    achieved = ops / (gemm_avg * 1e-3) / 1e12
+    kinds = group_kinds(d["bits"], d["bits"])
+    peak = mixed_peak(linear_ops(spec.M, spec.N, d["count"]), kinds, pk)
+    sha = kernel_sha()
+    traffic = TRAFFIC["bytes"] if TRAFFIC["sha256"] == sha else None
+    roofline = {"kernel": "soniq_mp_gemm tensor-core path", "bound": "tensor",
                 "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
-                "frac": round(achieved / peak, 4), "traffic": args.traffic,
+                "frac": round(achieved / peak, 4), "traffic": traffic,
                 "peak_source": f"{pk['src']}: bf16 {pk['bf16']} TFLOP/s burst; E4M3 = 2x bf16 "
                                f"(nominal ratio), fp16 = bf16 rate; time-weighted over the groups",
+                "gemm_us": round(gemm_avg * 1e3, 2),
                 "quantize_us": round(statistics.mean(quant_ms) * 1e3, 2),
-                "conv_us": round(conv_avg_ms * 1e3, 2)}
+                "quantize_GBps": round(quant_bytes(spec.M, spec.K, d["count"], d["bits"])
+                                       / (statistics.mean(quant_ms) * 1e-3) / 1e9, 1)}
 
     out = {"metric": METRIC, "value": round(value, 3), "unit": "TOPS", "n_gpus": world,
            "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": round(ms_per_step, 5),
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "u8xs8->i32 (E4M3/fp16 tensor pipes, exact)", "data": "synthetic",
-           "config": {"workload": spec.name, "M": spec.M, "N": spec.C_out, "K": spec.K,
-                      "bits": d["bits"], "count": d["count"], "parallelism": f"replicas{world}",
-                      "l2": "flushed between timed steps (256 MB write)",
-                      "launch": "the step (both library calls) replayed as one CUDA graph; e2e: plain API calls"},
+           "config": headline_config(spec, d, world),
            "e2e": {"value": round(e2e_value, 3), "unit": "TOPS",
-                   "h2d_bytes_per_step": int(Xh[0].numel() * 2), "d2h_bytes_per_step": int(Yh[0].numel() * 2),
+                   "h2d_bytes_per_step": int(Ah[0].numel() * 2), "d2h_bytes_per_step": int(Yh[0].numel() * 2),
                    "ms_per_step": round(e2e_ms, 5),
                    "pipelining": "upload, kernels and download of neighbouring steps overlap (3 streams, 2 buffer sets)"},
            "gpu_launches": int(launches),
            "roofline": roofline,
            "clocks": clk}
-    if args.suite:
-        out["suite"] = run_suite(args, sq, wl, pk, flush)
+    if not args.no_suite:
+        out["suite"] = run_suite(args, sq, wl, pk, flush, d)
     if rank == 0 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(spec, d, budget_s=args.cpu_seconds)
+        out["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
     if rank == 0:
         print(json.dumps(out), flush=True)
     if world > 1:
         dist.destroy_process_group()
 
 
-def _time_events(fn, steps, flush, stream):
-    """Median device time of fn (a library call), replayed as a CUDA graph so
-    that host call overhead is not timed; L2 flushed before every replay."""
-    import torch
-    for _ in range(2):
-        fn()
-    torch.cuda.synchronize()
-    side = torch.cuda.Stream()
-    side.wait_stream(stream)
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=side):
-        fn()
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
-    for _ in range(3):
-        flush.zero_()
-        g.replay()
-    for i in range(steps):
-        flush.zero_()
-        ev[i][0].record(stream)
-        g.replay()
-        ev[i][1].record(stream)
-    torch.cuda.synchronize()
-    return statistics.median(a.elapsed_time(b) for a, b in ev)
+def headline_config(spec, d, world):
+    """The `config` of both arms' lines (identical)."""
+    return {"workload": spec.name, "M": spec.M, "N": spec.N, "K": spec.K, "bits": d["bits"],
+            "count": d["count"], "parallelism": f"replicas{world}",
+            "l2": "flushed between timed steps (256 MB write)",
+            "launch": "the step (both library calls) replayed as one CUDA graph; e2e: plain API calls"}
 
 
-def run_suite(args, sq, wl, pk, flush):
-    """Per-kernel measurements for the other workload families."""
+def run_suite(args, sq, wl, pk, flush, head):
+    """Every workload family, each library call replayed as a CUDA graph after
+    an L2 flush (median of the replays)."""
     import torch
     stream = torch.cuda.current_stream()
+    steps = max(5, args.suite_steps)
     rows = []
 
-    def linear_case(spec, kind):
-        d = wl.make_linear(spec)
+    def linear_case(spec, d=None, gemv=False):
+        d = wl.make_linear(spec) if d is None else d
         lay = sq.Layout(d["perm"], d["count"], d["bits"])
         A = torch.from_numpy(d["A"]).cuda()
         W = torch.from_numpy(d["W"]).cuda()
         Wp, s_w = sq.pack_weights(lay, W)
         Ap, s_a = sq.quantize_act(lay, A)
         Y = torch.empty((spec.M, spec.N), dtype=torch.float16, device="cuda")
-        gemm_ms = _time_events(lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y), args.steps, flush, stream)
-        quant_ms = _time_events(lambda: sq.quantize_act(lay, A, "tensor", s_a=s_a, Ap=Ap), args.steps, flush, stream)
-        pack_ms = _time_events(lambda: sq.pack_weights(lay, W, Wp=Wp, s_w=s_w), max(3, args.steps // 4), flush, stream)
+        gemm_ms = _time_fn(lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y), steps, flush, stream)
+        quant_ms = _time_fn(lambda: sq.quantize_act(lay, A, "tensor", s_a=s_a, Ap=Ap), steps, flush, stream)
         ops = spec.ops
-        kinds = [0 if b <= 4 else 1 for b in d["bits"]]
-        peak = mixed_peak([2 * spec.M * spec.N * c for c in d["count"]], kinds, pk)
-        wbytes = sum(c * b for c, b in zip(d["count"], d["bits"])) / 8 * spec.N
-        abytes = spec.M * spec.K * 2 + spec.M * sum(c * b for c, b in zip(d["count"], d["bits"])) / 8
         r = {"workload": spec.name, "M": spec.M, "N": spec.N, "K": spec.K, "bits": d["bits"],
-             "gemm_us": round(gemm_ms * 1e3, 2), "TOPS": round(ops / (gemm_ms * 1e-3) / 1e12, 2),
-             "quantize_us": round(quant_ms * 1e3, 2),
-             "quantize_GBps": round(abytes / (quant_ms * 1e-3) / 1e9, 1),
-             "pack_weights_us": round(pack_ms * 1e3, 2)}
-        if kind == "gemv":
-            moved = Wp.numel() + s_w.numel() * 4
-            r["path"] = "CUDA-core GEMV" if spec.M <= 12 else "tensor-core kernel"
-            r["gemv_GBps_algorithmic"] = round(wbytes / (gemm_ms * 1e-3) / 1e9, 1)
-            r["frac_hbm"] = round(wbytes / (gemm_ms * 1e-3) / 1e9 / pk["hbm"], 4)
-            r["weight_bytes_moved"] = int(moved)
+             "count": d["count"], "gemm_us": round(gemm_ms * 1e3, 2),
+             "TOPS": round(ops / (gemm_ms * 1e-3) / 1e12, 2), "quantize_us": round(quant_ms * 1e3, 2),
+             "quantize_GBps": round(quant_bytes(spec.M, spec.K, d["count"], d["bits"]) / (quant_ms * 1e-3) / 1e9, 1)}
+        if gemv:
+            wbytes = sum(c * b for c, b in zip(d["count"], d["bits"])) / 8 * spec.N
+            gbs = wbytes / (gemm_ms * 1e-3) / 1e9
+            r["path"] = sq.gemm_path(lay, spec.M, spec.N)
+            r["GBps_packed_weights"] = round(gbs, 1)
+            r["frac_hbm_measured"] = round(gbs / pk["hbm"], 4)
+            r["frac_hbm_8TBps"] = round(gbs / 8000.0, 4)
+            r["weight_bytes_algorithmic"] = int(wbytes)
+            r["weight_bytes_moved"] = int(Wp.numel() + s_w.numel() * 4)
         else:
+            peak = mixed_peak(linear_ops(spec.M, spec.N, d["count"]), group_kinds(d["bits"], d["bits"]), pk)
             r["frac_tensor_peak"] = round(ops / (gemm_ms * 1e-3) / 1e12 / peak, 4)
             r["peak_TFLOPs"] = round(peak, 1)
         rows.append(r)
+        del A, W, Wp, Ap, Y
 
-    linear_case(wl.LINEAR_SMALL, "gemm")
-    linear_case(wl.MLP_UP, "gemm")
+    def conv_case(spec):
+        d = wl.make_conv(spec)
+        lay = sq.Layout(d["perm"], d["count"], d["bits"], pad_unit=32)
+        X = torch.from_numpy(d["X"]).cuda().reshape(-1, spec.C)
+        Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
+        Xp, s_a = sq.quantize_act(lay, X)
+        cd = sq.conv_desc(spec.batch, spec.H, spec.W, spec.C_out, spec.R, spec.S, spec.stride, spec.pad)
+        P, Q = sq.conv_out_hw(cd)
+        Y = torch.empty((spec.batch, P, Q, spec.C_out), dtype=torch.float16, device="cuda")
+        ms = _time_fn(lambda: sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y), steps, flush, stream)
+        qms = _time_fn(lambda: sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp), steps, flush, stream)
+        ops = [2 * spec.M * spec.C_out * spec.R * spec.S * c for c in d["count"]]
+        peak = mixed_peak(ops, group_kinds(d["bits"], d["bits"]), pk)
+        qb = quant_bytes(spec.batch * spec.H * spec.W, spec.C, d["count"], d["bits"])
+        rows.append({"workload": spec.name, "M": spec.M, "N": spec.C_out, "K": spec.K, "bits": d["bits"],
+                     "count": d["count"], "conv_us": round(ms * 1e3, 2),
+                     "TOPS": round(spec.ops / (ms * 1e-3) / 1e12, 2),
+                     "frac_tensor_peak": round(spec.ops / (ms * 1e-3) / 1e12 / peak, 4),
+                     "peak_TFLOPs": round(peak, 1), "quantize_us": round(qms * 1e3, 2),
+                     "quantize_GBps": round(qb / (qms * 1e-3) / 1e9, 1),
+                     "quantize_frac_hbm": round(qb / (qms * 1e-3) / 1e9 / pk["hbm"], 4)})
+
+    linear_case(wl.LINEAR_SMALL)
+    conv_case(wl.CONV_RESNET)
+    conv_case(wl.CONV_RESNET_1B4B)
+    linear_case(wl.MLP_UP)
     for m in (1, 4, 16):
-        linear_case(wl.DECODE[m], "gemv")
-    pts = wl.sweep_specs() if args.full_sweep else [
-        s for s in wl.sweep_specs() if (s.bits_lo, s.bits_hi) in ((2, 8), (4, 8), (1, 4), (3, 6))]
-    for s in pts:
+        linear_case(wl.DECODE[m], gemv=True)
+    # the 60 sweep points share the headline point's seeded A and W draws; each
+    # point has its own seeded precision assignment (same as its own workload's)
+    for s in wl.sweep_specs():
+        perm, count, _ = wl.assignment(np.random.default_rng(s.seed), s.K, s.frac_hi, s.n_outliers)
+        d = dict(A=head["A"], W=head["W"], perm=perm, count=count, bits=[s.bits_lo, s.bits_hi])
         try:
-            linear_case(s, "gemm")
+            linear_case(s, d)
         except Exception as e:  # report, do not hide
             rows.append({"workload": s.name, "error": str(e)})
-    conv_b = wl.CONV_RESNET_1B4B
-    d = wl.make_conv(conv_b)
-    lay = sq.Layout(d["perm"], d["count"], d["bits"], pad_unit=32)
-    X = torch.from_numpy(d["X"]).cuda().reshape(-1, conv_b.C)
-    Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
-    Xp, s_a = sq.quantize_act(lay, X)
-    cd = sq.conv_desc(conv_b.batch, conv_b.H, conv_b.W, conv_b.C_out)
-    Y = torch.empty((conv_b.batch, 14, 14, conv_b.C_out), dtype=torch.float16, device="cuda")
-    ms = _time_events(lambda: sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y), args.steps, flush, stream)
-    kinds = [0 if b <= 4 else 1 for b in d["bits"]]
-    peak = mixed_peak(conv_ops(conv_b, d["count"]), kinds, pk)
-    rows.append({"workload": conv_b.name, "conv_us": round(ms * 1e3, 2),
-                 "TOPS": round(conv_b.ops / (ms * 1e-3) / 1e12, 2),
-                 "frac_tensor_peak": round(conv_b.ops / (ms * 1e-3) / 1e12 / peak, 4)})
     return rows
 
 
@@ -420,32 +461,74 @@ def _threads():
         return os.cpu_count() or 1
 
 
-def oracle_conv_sample(spec, d, n_pix):
-    """The oracle pipeline for the conv step on n_pix output pixels: scales,
-    codes and packing of the whole input, weights once, accumulators and
-    epilogue for the sampled pixels."""
+def oracle_step_parts(d, rows, s_w=None, J=None):
+    """The oracle's pipeline for one headline step, in two timed parts:
+    per-tensor scales, codes and packing of the whole input (t_q), and exact
+    accumulators plus the fp64 epilogue for the output rows `rows` (t_acc).
+    Weight codes are made once, outside the timing (offline in both arms)."""
     import oracle
-    rng = np.random.default_rng(0)
-    pix = np.sort(rng.choice(spec.M, size=min(n_pix, spec.M), replace=False))
-    return oracle.conv2d(d["X"], d["W"], d["perm"], d["count"], d["bits"], d["bits"], spec.R, spec.S,
-                         stride=spec.stride, pad=spec.pad, pix=pix), len(pix)
+    if J is None:
+        s_w = oracle.weight_scales(d["W"], d["perm"], d["count"])
+        J = oracle.weight_codes(d["W"], d["perm"], d["count"], d["bits"], s_w)
+    t0 = time.perf_counter()
+    A32 = d["A"].astype(np.float32)
+    s_a = oracle.act_scales(A32, d["perm"], d["count"])
+    U = oracle.act_codes(A32, d["perm"], d["count"], d["bits"], s_a)
+    oracle.pack_act_rows(U, d["count"], d["bits"], 128)
+    t1 = time.perf_counter()
+    acc = oracle.gemm_acc(U, J, d["count"], rows=rows)
+    oracle.epilogue(acc, s_a, s_w, d["bits"], d["bits"], rows=rows)
+    t2 = time.perf_counter()
+    return t1 - t0, t2 - t1, s_w, J
 
 
-def cpu_baseline(spec, d, budget_s=12.0):
+def oracle_worker(args):
+    """Runs in a child process (OMP_NUM_THREADS set by the parent): times the
+    oracle on the headline workload and prints one JSON line."""
+    from paper_2311_14114_gb300 import workloads as wl
     import oracle
     oracle.build()
-    t0 = time.perf_counter()
-    oracle_conv_sample(spec, d, 256)
-    t1 = time.perf_counter() - t0
-    n_pix = int(min(spec.M, max(256, 256 * budget_s / max(t1, 1e-3))))
-    t0 = time.perf_counter()
-    _, n = oracle_conv_sample(spec, d, n_pix)
-    dt = time.perf_counter() - t0
-    ops = 2 * n * spec.C_out * spec.K
-    return {"value": round(ops / dt / 1e12, 6), "unit": "TOPS", "cores": _threads(), "kind": "oracle",
-            "sample": f"{n} of {spec.M} output pixels (full-input scales/codes/packing, sampled "
-                      f"accumulators + epilogue), {dt:.1f} s",
-            "seconds": round(dt, 2)}
+    spec = headline_spec()
+    d = wl.make_linear(spec)
+    rng = np.random.default_rng(0)
+    probe = np.sort(rng.choice(spec.M, size=8, replace=False))
+    tq, ta, s_w, J = oracle_step_parts(d, probe)
+    per_row = ta / len(probe)
+    n = int(min(spec.M, max(8, (args.cpu_seconds - tq) / max(per_row, 1e-6))))
+    rows = np.sort(rng.choice(spec.M, size=n, replace=False))
+    tq, ta, _, _ = oracle_step_parts(d, rows, s_w, J)
+    print(json.dumps({"t_q": tq, "t_acc": ta, "rows": n, "M": spec.M}), flush=True)
+
+
+def _oracle_child(threads, seconds):
+    env = dict(os.environ, OMP_NUM_THREADS=str(threads))
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-worker",
+                        "--cpu-seconds", str(seconds)], capture_output=True, text=True, env=env, timeout=900)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle worker failed: {r.stderr[-2000:]}")
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def _extrapolated(res, ops_full):
+    """Full-step oracle time: the whole-input quantize plus the sampled
+    accumulator time scaled to all M rows; returns (TOPS, step seconds)."""
+    t_step = res["t_q"] + res["t_acc"] * res["M"] / res["rows"]
+    return ops_full / t_step / 1e12, t_step
+
+
+def cpu_baseline(budget_s=12.0):
+    spec = headline_spec()
+    cores = _threads()
+    one = _oracle_child(1, budget_s)
+    allc = _oracle_child(cores, budget_s)
+    v1, t1 = _extrapolated(one, spec.ops)
+    va, ta = _extrapolated(allc, spec.ops)
+    return {"value": round(va, 6), "unit": "TOPS", "cores": cores, "kind": "oracle",
+            "sample": (f"headline workload; per-tensor scales, codes and packing of all {spec.M} rows "
+                       f"({allc['t_q']:.2f} s), exact accumulators + fp64 epilogue for {allc['rows']} sampled "
+                       f"output rows ({allc['t_acc']:.2f} s), scaled to a full step of {ta:.1f} s"),
+            "single_thread": {"value": round(v1, 6), "unit": "TOPS", "cores": 1,
+                              "sample": f"{one['rows']} sampled rows, full step {t1:.1f} s"}}
 
 
 def run_reference(args):
@@ -456,27 +539,28 @@ def run_reference(args):
     from paper_2311_14114_gb300 import workloads as wl
     import oracle
     oracle.build()
-    spec = wl.CONV_RESNET
-    d = wl.make_conv(spec)
-    per_step_pix = 192
+    spec = headline_spec()
+    d = wl.make_linear(spec)
+    rng = np.random.default_rng(1)
+    rows_per_step = 16
+    s_w = J = None
     for _ in range(args.warmup):
-        oracle_conv_sample(spec, d, 32)
-    times = []
+        _, _, s_w, J = oracle_step_parts(d, np.arange(2), s_w, J)
+    t_steps = []
     for _ in range(args.steps):
-        t0 = time.perf_counter()
-        _, n = oracle_conv_sample(spec, d, per_step_pix)
-        times.append(time.perf_counter() - t0)
-    dt = sum(times)
-    ops = 2 * per_step_pix * spec.C_out * spec.K * args.steps
-    value = ops / dt / 1e12
-    sample = (f"each step: {per_step_pix} of {spec.M} output pixels (full-input scales/codes/"
-              f"packing, sampled accumulators + epilogue)")
+        rows = np.sort(rng.choice(spec.M, size=rows_per_step, replace=False))
+        tq, ta, s_w, J = oracle_step_parts(d, rows, s_w, J)
+        t_steps.append(tq + ta * spec.M / rows_per_step)
+    t_step = sum(t_steps) / len(t_steps)
+    value = spec.ops / t_step / 1e12
+    sample = (f"each step: per-tensor scales, codes and packing of all {spec.M} rows, exact accumulators + "
+              f"fp64 epilogue for {rows_per_step} sampled output rows, scaled to all rows")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt / args.steps * 1e3, 3),
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t_step * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64 (CPU oracle)",
         "data": "synthetic",
-        "config": {"workload": spec.name, "M": spec.M, "N": spec.C_out, "K": spec.K, "bits": d["bits"]},
+        "config": headline_config(spec, d, world),
         "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": _threads(), "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -485,7 +569,7 @@ def run_reference(args):
 
 def run_case(args):
     """One kernel family on one workload, for profiling (ncu) and tuning:
-    conv_4b8b | conv_1b4b | quant_conv | gemm:MxNxK:lo:hi:frac | gemv:M."""
+    headline | quant_headline | conv_4b8b | conv_1b4b | quant_conv | gemm:MxNxK:lo:hi:frac | gemv:M."""
     import torch
     from paper_2311_14114_gb300 import soniq as sq
     from paper_2311_14114_gb300 import workloads as wl
@@ -506,16 +590,23 @@ def run_case(args):
             fn, ops = (lambda: sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp)), 0
         else:
             fn, ops = (lambda: sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y)), spec.ops
-    elif name.startswith("gemm:"):
-        _, shape, lo, hi, frac = name.split(":")
-        M, N, K = (int(x) for x in shape.split("x"))
-        spec = wl.LinearSpec(name, M=M, K=K, N=N, bits_lo=int(lo), bits_hi=int(hi), frac_hi=float(frac))
+    elif name.startswith("gemm:") or name in ("headline", "quant_headline"):
+        if name.startswith("gemm:"):
+            _, shape, lo, hi, frac = name.split(":")
+            M, N, K = (int(x) for x in shape.split("x"))
+            spec = wl.LinearSpec(name, M=M, K=K, N=N, bits_lo=int(lo), bits_hi=int(hi), frac_hi=float(frac))
+        else:
+            spec = headline_spec()
         d = wl.make_linear(spec)
         lay = sq.Layout(d["perm"], d["count"], d["bits"])
         Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
-        Ap, s_a = sq.quantize_act(lay, torch.from_numpy(d["A"]).cuda())
-        Y = torch.empty((M, N), dtype=torch.float16, device="cuda")
-        fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y, flags=sq.FLAG_FORCE_MMA)), spec.ops
+        A = torch.from_numpy(d["A"]).cuda()
+        Ap, s_a = sq.quantize_act(lay, A)
+        Y = torch.empty((spec.M, spec.N), dtype=torch.float16, device="cuda")
+        if name == "quant_headline":
+            fn, ops = (lambda: sq.quantize_act(lay, A, "tensor", s_a=s_a, Ap=Ap)), 0
+        else:
+            fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y, flags=args.flags)), spec.ops
     elif name.startswith("gemv:"):
         spec = wl.DECODE[int(name.split(":")[1])]
         d = wl.make_linear(spec)
@@ -523,10 +614,10 @@ def run_case(args):
         Wp, s_w = sq.pack_weights(lay, torch.from_numpy(d["W"]).cuda())
         Ap, s_a = sq.quantize_act(lay, torch.from_numpy(d["A"]).cuda())
         Y = torch.empty((spec.M, spec.N), dtype=torch.float16, device="cuda")
-        fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y)), spec.ops
+        fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y, flags=args.flags)), spec.ops
     else:
         raise SystemExit(f"unknown case {name}")
-    ms = _time_events(fn, args.steps, flush, stream)
+    ms = _time_fn(fn, args.steps, flush, stream)
     if sq.sync_status() != 0:
         raise RuntimeError("device error")
     print(json.dumps({"case": name, "us": round(ms * 1e3, 2),
@@ -539,15 +630,17 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="soniq", choices=["soniq", "reference"])
-    ap.add_argument("--suite", action="store_true")
-    ap.add_argument("--full-sweep", action="store_true")
+    ap.add_argument("--no-suite", action="store_true", help="skip the per-workload suite")
+    ap.add_argument("--suite-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0)
-    ap.add_argument("--case", default=None, help="profile one kernel family on one workload")
-    ap.add_argument("--traffic", type=float, default=CONV_TRAFFIC_BYTES,
-                    help="DRAM bytes per conv launch from an ncu capture of the current kernel")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--case", default=None, help="time one kernel family on one workload")
+    ap.add_argument("--flags", type=int, default=0, help="soniq_mp_gemm flags for --case")
+    ap.add_argument("--oracle-worker", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
-    if args.case:
+    if args.oracle_worker:
+        oracle_worker(args)
+    elif args.case:
         run_case(args)
     elif args.impl == "reference":
         run_reference(args)

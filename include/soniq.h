@@ -13,7 +13,9 @@
  *
  * Conventions for every call:
  *   * Device pointers are CUDA global-memory addresses owned by the caller;
- *     the library never allocates, frees or retains them.
+ *     the library never allocates, frees or retains them.  Calls that need
+ *     working memory take it from the caller as a `scratch` pointer and its
+ *     size in bytes; a *_scratch_bytes() query (host only) says how much.
  *   * Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
  *     default stream).  Argument errors are detected on the host before any
  *     CUDA call and returned synchronously.  Launch failures return
@@ -34,7 +36,7 @@
 extern "C" {
 #endif
 
-#define SONIQ_ABI_VERSION 1
+#define SONIQ_ABI_VERSION 2
 
 /* Exported symbols (the library is built with hidden default visibility). */
 #if defined(__GNUC__)
@@ -111,6 +113,14 @@ enum {
                                             wait runs out and the call reports SONIQ_ERR_TIMEOUT */
 };
 
+/* Kernels behind soniq_mp_gemm (see soniq_mp_gemm_path). */
+enum {
+    SONIQ_PATH_GEMV = 0,    /* CUDA-core GEMV streaming the packed weights (small M) */
+    SONIQ_PATH_TENSOR = 1   /* tcgen05 tensor-core kernel expanding packed tiles on chip */
+};
+/* Without flags, soniq_mp_gemm runs the GEMV for M <= SONIQ_GEMV_MAX_M. */
+#define SONIQ_GEMV_MAX_M 12
+
 /* Convolution geometry.  Input NHWC [batch][H][W][C_in], output NHWC
  * [batch][P][Q][C_out], P = (H + 2*pad_h - R)/stride_h + 1, Q likewise. */
 typedef struct soniq_conv_desc {
@@ -169,37 +179,70 @@ SONIQ_API soniq_status soniq_pack_weights(const soniq_layout *layout, const floa
  * (2^n - 1)), 0, 2^n - 1); s = 0 gives u = 0.  Channels are gathered through
  * layout->perm and each group is zero-padded to PA_g codes.
  *
- *   A          device fp16 [M][K] (IEEE binary16 bits), 2-byte aligned.
+ *   A          device fp16 [M][K] (IEEE binary16 bits), 2-byte aligned; K <= 32768.
  *   M          rows (tokens, or pixels of an NHWC image); 0 is a no-op.
  *   scale_mode SONIQ_SCALE_PER_TENSOR: s_a is an output [2];
  *              SONIQ_SCALE_PER_ROW:    s_a is an output [M][2];
  *              SONIQ_SCALE_CALIBRATED: s_a is an input [2].
  *   s_a        device fp32, see scale_mode.
  *   Ap         device out [M][soniq_packed_row_bytes(layout, 0, 1)], 4-byte aligned.
+ *   scratch, scratch_bytes
+ *              optional caller-owned device memory, 16-byte aligned.  With
+ *              SONIQ_SCALE_PER_TENSOR and scratch_bytes >=
+ *              soniq_quantize_act_scratch_bytes(), inputs whose rows fit on
+ *              chip (about M * K <= 15 * 2^20) are quantized in one pass over
+ *              A by a cooperative kernel whose grid barrier and per-CTA maxima
+ *              live in the scratch; otherwise (or with scratch = NULL) the
+ *              scale is found by a separate max-abs pass first.  Other modes
+ *              ignore the scratch.
+ *              Contract: the scratch must be zero-filled before its first use
+ *              (cudaMemsetAsync once after allocating it); every completed
+ *              call leaves it zero-filled again.  After soniq_sync_status
+ *              reports SONIQ_ERR_TIMEOUT, zero it again before reuse.  Calls
+ *              that may overlap on the GPU (different streams) must use
+ *              different scratch buffers.
  */
 SONIQ_API soniq_status soniq_quantize_act(const soniq_layout *layout, const void *A, int64_t M,
-                                int32_t scale_mode, float *s_a, uint8_t *Ap,
-                                soniq_stream_t stream);
+                                int32_t scale_mode, float *s_a, uint8_t *Ap, void *scratch,
+                                size_t scratch_bytes, soniq_stream_t stream);
+
+/* Scratch bytes that soniq_quantize_act can use for these arguments (0 when
+ * the call needs none).  Host only; -1 on a bad argument. */
+SONIQ_API int64_t soniq_quantize_act_scratch_bytes(const soniq_layout *layout, int64_t M,
+                                                   int32_t scale_mode);
 
 /*
- * Per-tensor activation quantize-and-pack that allocates nothing and never
- * takes a second pass.  The paper has no counterpart: this is an engineering
- * variant of soniq_quantize_act with scale_mode SONIQ_SCALE_PER_TENSOR, for
- * callers that must not let the library reach any memory other than the
- * arguments and a fixed scratch (for instance inside CUDA graph capture).
+ * Per-tensor activation quantize-and-pack that allocates nothing and takes no
+ * scratch argument.  The paper has no counterpart; this is an engineering
+ * variant of soniq_quantize_act (SONIQ_SCALE_PER_TENSOR, one pass) for
+ * callers that cannot call cudaMalloc or hand the library device memory of
+ * their own: for instance a host that only gives the library the tensors of
+ * the layer (an inference runtime whose allocator is not reachable from the
+ * code that calls this library, or a real-time loop in which allocating, and
+ * the device synchronization that cudaMalloc/cudaFree may cause, is not
+ * allowed).
  *
  * It computes exactly what soniq_quantize_act computes in per-tensor mode
- * (same s_a and packed bytes), in one cooperative kernel whose grid barrier
- * and per-CTA maxima live in a file-scope static device array of the library
- * (8 KB per device, resolved once per device with cudaGetSymbolAddress).
- *   Limits: one CTA per SM, at most 1024 CTAs; each CTA's M / (number of SMs)
- *   rows, padded, must fit in 200 KB of shared memory (2 * K bytes per row plus
- *   the permutation), i.e. M * K up to about 15 * 2^20 on a 152-SM GB300.
- *   Larger inputs return SONIQ_ERR_UNSUPPORTED before any launch.
- *   Concurrency: calls share that scratch, so two calls that overlap in time
- *   (on different streams of one device) race; serialize them.
- *   A barrier wait that runs out (2 s) is reported by soniq_sync_status, which
- *   also clears the barrier.
+ * (same s_a and packed bytes).  Its working memory is a file-scope static
+ * device array of the library (8 KB on every device that loads the library,
+ * held until the process exits): a grid barrier (arrival count, generation)
+ * and the per-CTA maxima of at most 1024 CTAs.
+ *   Set-up: the first call on each device, with that device current, looks up
+ *   the array's device address (cudaGetSymbolAddress) and sets the kernel's
+ *   shared-memory attributes; make that first call before any stream capture.
+ *   Limits: one CTA of 1024 threads per SM, each holding its M / (number of
+ *   SMs) rows in at most 200 KB of shared memory (2 * K bytes per row plus the
+ *   permutation): M * K up to about 15 * 2^20 on a 152-SM GB300.  Larger
+ *   inputs return SONIQ_ERR_UNSUPPORTED before anything is launched; there is
+ *   no two-pass fallback.
+ *   Sharing: every call uses the same array.  The barrier count must start at
+ *   zero: it is zero when the library loads and every completed call leaves it
+ *   at zero; the per-CTA maxima are written before they are read.  Two calls
+ *   that overlap on the GPU (different streams) race on the array and give
+ *   wrong results; serialize them.
+ *   Timeouts: a barrier wait that runs out (2 s) makes soniq_sync_status
+ *   return SONIQ_ERR_TIMEOUT; that call then waits for the whole device and
+ *   resets the barrier, so the next call starts clean.
  * Arguments as for soniq_quantize_act; s_a is an output [2].
  */
 SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, const void *A, int64_t M,
@@ -211,9 +254,10 @@ SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, co
  * integer dot products):
  *   Acc_g[m][n] = sum over k in group g of u[m][k] * j[n][k]   (exact int32)
  *   Y[m][n]     = sum_g s_a(m,g) * s_w[n][g] / ((2^na_g - 1) * 2^(nw_g - 1)) * Acc_g[m][n]
- * computed in fp32 and rounded to nearest fp16 (or bf16).  M <= 12 runs a
- * bandwidth-bound CUDA-core GEMV, larger M the tcgen05 tensor-core kernel
- * (flags can force either; the GEMV takes M <= 16).
+ * computed in fp32 and rounded to nearest fp16 (or bf16).  M <= SONIQ_GEMV_MAX_M
+ * runs a bandwidth-bound CUDA-core GEMV, larger M the tcgen05 tensor-core
+ * kernel (flags can force either; the GEMV takes M <= 16); soniq_mp_gemm_path
+ * tells which.
  *
  *   Ap, s_a    from soniq_quantize_act with the same layout (pad_unit 32 or 128);
  *              s_a [2] (PER_TENSOR / CALIBRATED) or [M][2] (PER_ROW).
@@ -229,7 +273,18 @@ SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, co
 SONIQ_API soniq_status soniq_mp_gemm(const soniq_layout *layout, const uint8_t *Ap, const float *s_a,
                            int32_t scale_mode, int64_t M, const uint8_t *Wp, const float *s_w,
                            int32_t N, void *Y, int32_t out_dtype, int32_t *acc_dbg,
-                           uint32_t flags, soniq_stream_t stream);
+                           uint32_t flags, void *scratch, size_t scratch_bytes,
+                           soniq_stream_t stream);
+
+/* The kernel soniq_mp_gemm runs for these arguments (SONIQ_PATH_*), or -1
+ * if it would return an error.  Host only (reads the device's SM count). */
+SONIQ_API int32_t soniq_mp_gemm_path(const soniq_layout *layout, int64_t M, int32_t N, uint32_t flags,
+                                     size_t scratch_bytes);
+
+/* Scratch bytes soniq_mp_gemm can use for these arguments (0: none).  Host
+ * only; -1 on a bad argument. */
+SONIQ_API int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout *layout, int64_t M, int32_t N,
+                                              uint32_t flags);
 
 /*
  * Mixed-precision quantized convolution as implicit GEMM (Sec. 4.1: the CPU
@@ -248,13 +303,29 @@ SONIQ_API soniq_status soniq_mp_gemm(const soniq_layout *layout, const uint8_t *
 SONIQ_API soniq_status soniq_mp_conv2d(const soniq_layout *layout, const soniq_conv_desc *cd,
                              const uint8_t *Xp, const float *s_a, int32_t scale_mode,
                              const uint8_t *Wp, const float *s_w, void *Y, int32_t out_dtype,
-                             int32_t *acc_dbg, uint32_t flags, soniq_stream_t stream);
+                             int32_t *acc_dbg, uint32_t flags, void *scratch, size_t scratch_bytes,
+                             soniq_stream_t stream);
+
+/* Scratch bytes soniq_mp_conv2d can use for these arguments (0: none).  Host
+ * only; -1 on a bad argument. */
+SONIQ_API int64_t soniq_mp_conv2d_scratch_bytes(const soniq_layout *layout, const soniq_conv_desc *cd,
+                                                uint32_t flags);
 
 /* Waits for `stream`, then returns SONIQ_ERR_TIMEOUT if any kernel of this
  * library on the current device recorded a timed-out wait since the last
  * call (and clears that record), SONIQ_ERR_CUDA on a CUDA error, else
- * SONIQ_OK. */
+ * SONIQ_OK.  When the timed-out wait was the grid barrier of
+ * soniq_quantize_act_oneshot, it also waits for the whole device and then
+ * resets that barrier. */
 SONIQ_API soniq_status soniq_sync_status(soniq_stream_t stream);
+
+/* Test hook, not for production use.  When armed (armed != 0), the next
+ * launch of the one-pass per-tensor quantize kernel, from soniq_quantize_act
+ * or soniq_quantize_act_oneshot, has its first CTA skip its grid-barrier
+ * arrival: the other CTAs' bounded waits run out after 2 s, the outputs are
+ * not written, and soniq_sync_status reports SONIQ_ERR_TIMEOUT.  The hook
+ * disarms itself at that launch.  No fault, trap or hang is involved. */
+SONIQ_API void soniq_test_drop_barrier_arrival(int32_t armed);
 
 #ifdef __cplusplus
 }

@@ -352,8 +352,10 @@ struct FusedParams {
     uint8_t* Ap;
     float* s_a;              // [2] out
     unsigned* bar;           // grid barrier: [0] arrivals (0 between launches), [1] generation
-    float* part;             // [gridDim][2] per-CTA maxima (library scratch)
+    float* part;             // [gridDim][2] per-CTA maxima
     unsigned* err;           // device error word
+    unsigned err_bit;        // bit ORed into it when the barrier wait runs out
+    int32_t drop_arrival;    // test hook: CTA 0 does not arrive at the barrier
     const int32_t* perm;
     int64_t M;
     int32_t K;
@@ -549,7 +551,7 @@ __global__ void __launch_bounds__(1024) quantize_fused_kernel(const FusedParams 
         p.part[2 * blockIdx.x + 1] = f1;
         const unsigned gen = *reinterpret_cast<volatile unsigned*>(p.bar + 1);
         __threadfence();
-        if (atomicAdd(p.bar, 1u) == gridDim.x - 1) {
+        if (!(p.drop_arrival && blockIdx.x == 0) && atomicAdd(p.bar, 1u) == gridDim.x - 1) {
             *reinterpret_cast<volatile unsigned*>(p.bar) = 0u;
             __threadfence();
             atomicAdd(p.bar + 1, 1u);
@@ -562,7 +564,7 @@ __global__ void __launch_bounds__(1024) quantize_fused_kernel(const FusedParams 
                 asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
                 if (t0 == 0) t0 = t;
                 else if (t - t0 > p.timeout_ns) {
-                    atomicOr(p.err, 1u);
+                    atomicOr(p.err, p.err_bit);
                     abort_s = 1;
                     break;
                 }
@@ -763,7 +765,7 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
 // next to a co-resident grid; returns cudaErrorNotSupported otherwise.
 cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
                                   float* s_a, uint8_t* Ap, cudaStream_t st, unsigned* bar, float* part,
-                                  int max_ctas) {
+                                  int max_ctas, unsigned err_bit) {
     static __thread int attr_dev = -1;
     FusedParams p;
     p.A = A;
@@ -772,6 +774,8 @@ cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, co
     p.err = device_error_word();
     p.bar = bar;
     p.part = part;
+    p.err_bit = err_bit;
+    p.drop_arrival = 0;
     if (p.err == nullptr || p.bar == nullptr || p.part == nullptr) return cudaErrorNotSupported;
     p.perm = perm;
     p.M = M;
@@ -815,6 +819,7 @@ cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, co
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    p.drop_arrival = take_drop_arrival() ? 1 : 0;
     e = cudaLaunchKernelEx(&cfg, quantize_fused_kernel, p);
     if (e == cudaSuccess) note_launch();
     return e;

@@ -16,17 +16,22 @@ namespace soniq {
 namespace {
 
 // One word per device: kernels atomically OR error bits into it when a
-// bounded wait runs out; soniq_sync_status reads and clears it.
+// bounded wait runs out (kErrWait, kErrQuantBarrier, kErrOneshotBarrier);
+// soniq_sync_status reads and clears it.
 __device__ unsigned g_error_word;
-__device__ unsigned g_grid_barrier[2];                     // per-tensor quantize: arrivals, generation
-__device__ float g_grid_partials[2 * kMaxGridPartials];    // per-tensor quantize: per-CTA maxima
 
-// Scratch of soniq_quantize_act_oneshot: its own grid barrier (arrival count,
-// generation; zero at module load and left at zero by every completed call)
-// and per-CTA maxima for at most kOneShotMaxCtas CTAs (8 KB).
+// Working memory of soniq_quantize_act_oneshot, the entry point that takes no
+// scratch from its caller: a grid barrier (arrival count, generation; zero
+// when the module loads and left at zero by every completed call) and the
+// per-CTA maxima of at most kOneShotMaxCtas CTAs (8 KB in all).  Host code
+// reaches it only through the address cudaGetSymbolAddress returns.
 constexpr int kOneShotMaxCtas = 1024;
 static __device__ __align__(256) unsigned g_oneshot_barrier[2];
 static __device__ __align__(256) float g_oneshot_partials[2 * kOneShotMaxCtas];
+
+// Test hook (soniq_test_drop_barrier_arrival): the next one-pass quantize
+// launch drops one grid-barrier arrival.
+std::atomic<int> g_drop_arrival{0};
 
 std::atomic<int64_t> g_launches{0};
 
@@ -63,18 +68,6 @@ unsigned* device_error_word() {
     return g_err_addr[dev];
 }
 
-unsigned* grid_barrier_word() {
-    static unsigned* addr[64] = {};
-    const int dev = current_device();
-    if (dev < 0 || dev >= 64) return nullptr;
-    if (addr[dev] == nullptr) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_grid_barrier) != cudaSuccess) return nullptr;
-        addr[dev] = static_cast<unsigned*>(p);
-    }
-    return addr[dev];
-}
-
 // Device addresses of the one-shot scratch, resolved once per device at first
 // use; false if the runtime cannot resolve them.
 bool oneshot_scratch(unsigned** bar, float** part) {
@@ -97,17 +90,7 @@ bool oneshot_scratch(unsigned** bar, float** part) {
     return true;
 }
 
-float* grid_partials() {
-    static float* addr[64] = {};
-    const int dev = current_device();
-    if (dev < 0 || dev >= 64) return nullptr;
-    if (addr[dev] == nullptr) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_grid_partials) != cudaSuccess) return nullptr;
-        addr[dev] = static_cast<float*>(p);
-    }
-    return addr[dev];
-}
+bool take_drop_arrival() { return g_drop_arrival.exchange(0) != 0; }
 
 void note_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
@@ -176,6 +159,22 @@ using namespace soniq;
 namespace {
 
 cudaStream_t as_stream(soniq_stream_t s) { return reinterpret_cast<cudaStream_t>(s); }
+
+// The kernel soniq_mp_gemm runs: a SONIQ_PATH_* value, -1 when the
+// tensor-core kernel would be chosen but cannot take the layout (mma_check
+// says why), -2 when the GEMV was forced but cannot take the shape.
+int gemm_path(const LayoutGeom& geo, int64_t M, int32_t N, uint32_t flags, size_t scratch_bytes) {
+    (void)scratch_bytes;
+    // up to SONIQ_GEMV_MAX_M rows the CUDA-core GEMV is faster; above, the tensor-core
+    // kernel (whose time hardly grows with M below 128) overtakes it (decode N=11008,
+    // K=4096: 47.6 vs 41.5 us at M=16)
+    const bool want_gemv =
+        (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= SONIQ_GEMV_MAX_M && !(flags & SONIQ_FLAG_FORCE_MMA));
+    if (want_gemv && gemv_supported(geo, M, N)) return SONIQ_PATH_GEMV;
+    if (flags & SONIQ_FLAG_FORCE_GEMV) return -2;
+    if (mma_check(geo) != SONIQ_OK) return -1;
+    return SONIQ_PATH_TENSOR;
+}
 
 soniq_status check_scale_mode_act(int32_t mode) {
     return (mode == SONIQ_SCALE_PER_TENSOR || mode == SONIQ_SCALE_PER_ROW || mode == SONIQ_SCALE_CALIBRATED)
@@ -249,8 +248,15 @@ soniq_status soniq_pack_weights(const soniq_layout* L, const float* W, int32_t N
     return cuda_status(launch_pack_weights(geo, L->perm, W, N, scale_mode == SONIQ_SCALE_PER_ROW, Wp, s_w, s));
 }
 
+int64_t soniq_quantize_act_scratch_bytes(const soniq_layout* L, int64_t M, int32_t scale_mode) {
+    LayoutGeom geo;
+    if (make_geom(L, 1, &geo) != SONIQ_OK || M < 0 || check_scale_mode_act(scale_mode) != SONIQ_OK) return -1;
+    return scale_mode == SONIQ_SCALE_PER_TENSOR && M > 0 ? kQuantScratchBytes : 0;
+}
+
 soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M, int32_t scale_mode,
-                                float* s_a, uint8_t* Ap, soniq_stream_t stream) {
+                                float* s_a, uint8_t* Ap, void* scratch, size_t scratch_bytes,
+                                soniq_stream_t stream) {
     LayoutGeom geo;
     soniq_status st = make_geom(L, 1, &geo);
     if (st != SONIQ_OK) return st;
@@ -259,15 +265,21 @@ soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M,
     if ((st = check_scale_mode_act(scale_mode)) != SONIQ_OK) return st;
     if (M == 0) return SONIQ_OK;
     if (A == nullptr || s_a == nullptr || Ap == nullptr || L->perm == nullptr) return SONIQ_ERR_INVALID_ARG;
-    if (!aligned(A, 2) || !aligned(Ap, 4) || !aligned(s_a, 4)) return SONIQ_ERR_ALIGNMENT;
+    if (!aligned(A, 2) || !aligned(Ap, 4) || !aligned(s_a, 4) || (scratch != nullptr && !aligned(scratch, 16)))
+        return SONIQ_ERR_ALIGNMENT;
     cudaStream_t s = as_stream(stream);
     const uint16_t* A16 = static_cast<const uint16_t*>(A);
     if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
-        cudaError_t e = launch_quantize_fused(geo, L->perm, A16, M, s_a, Ap, s, grid_barrier_word(), grid_partials(),
-                                              kMaxGridPartials);
-        if (e == cudaSuccess) return SONIQ_OK;
-        if (e != cudaErrorNotSupported) return cuda_status(e);
-        e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);   // two passes: rows do not fit on chip
+        if (scratch != nullptr && scratch_bytes >= (size_t)kQuantScratchBytes) {
+            // one pass: barrier words at the start of the scratch, per-CTA maxima after 256 bytes
+            unsigned* bar = static_cast<unsigned*>(scratch);
+            float* part = reinterpret_cast<float*>(static_cast<uint8_t*>(scratch) + 256);
+            cudaError_t e = launch_quantize_fused(geo, L->perm, A16, M, s_a, Ap, s, bar, part, kMaxGridPartials,
+                                                  kErrQuantBarrier);
+            if (e == cudaSuccess) return SONIQ_OK;
+            if (e != cudaErrorNotSupported) return cuda_status(e);
+        }
+        cudaError_t e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);   // two passes
         if (e != cudaSuccess) return cuda_status(e);
     }
     return cuda_status(launch_quantize_act(geo, L->perm, A16, M, scale_mode, s_a, Ap, s));
@@ -287,14 +299,16 @@ soniq_status soniq_quantize_act_oneshot(const soniq_layout* L, const void* A, in
     float* part = nullptr;
     if (!oneshot_scratch(&bar, &part)) return SONIQ_ERR_CUDA;
     const cudaError_t e = launch_quantize_fused(geo, L->perm, static_cast<const uint16_t*>(A), M, s_a, Ap,
-                                                as_stream(stream), bar, part, kOneShotMaxCtas);
+                                                as_stream(stream), bar, part, kOneShotMaxCtas, kErrOneshotBarrier);
     if (e == cudaErrorNotSupported) return SONIQ_ERR_UNSUPPORTED;   // rows do not fit on chip: no fallback
     return cuda_status(e);
 }
 
 soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float* s_a, int32_t scale_mode,
                            int64_t M, const uint8_t* Wp, const float* s_w, int32_t N, void* Y,
-                           int32_t out_dtype, int32_t* acc_dbg, uint32_t flags, soniq_stream_t stream) {
+                           int32_t out_dtype, int32_t* acc_dbg, uint32_t flags, void* scratch,
+                           size_t scratch_bytes, soniq_stream_t stream) {
+    (void)scratch;
     LayoutGeom geo;
     soniq_status st = make_geom(L, 1, &geo);
     if (st != SONIQ_OK) return st;
@@ -311,15 +325,12 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     // K <= 65536 keeps |Acc| < 2^31 and the GEMV's unsigned offset sums below 2^32
     const int per_row = scale_mode == SONIQ_SCALE_PER_ROW;
     cudaStream_t s = as_stream(stream);
-    // up to 12 rows the CUDA-core GEMV is faster; from 13 the tensor-core kernel (whose time hardly
-    // grows with M below 128) overtakes it (decode N=11008, K=4096: 47.6 vs 41.5 us at M=16)
-    const bool want_gemv = (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= 12 && !(flags & SONIQ_FLAG_FORCE_MMA));
-    if (want_gemv && gemv_supported(geo, M, N)) {
+    const int path = gemm_path(geo, M, N, flags, scratch_bytes);
+    if (path < 0) return path == -2 ? SONIQ_ERR_UNSUPPORTED : mma_check(geo);
+    if (path == SONIQ_PATH_GEMV) {
         GemvArgs a{Ap, Wp, s_a, s_w, Y, acc_dbg, (int32_t)M, N, per_row, out_dtype == SONIQ_OUT_BF16};
         return cuda_status(launch_gemv(geo, a, s));
     }
-    if (flags & SONIQ_FLAG_FORCE_GEMV) return SONIQ_ERR_UNSUPPORTED;
-    if ((st = mma_check(geo)) != SONIQ_OK) return st;
     MmaArgs a{};
     a.Ap = Ap;
     a.Wp = Wp;
@@ -339,7 +350,9 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
 soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, const uint8_t* Xp,
                              const float* s_a, int32_t scale_mode, const uint8_t* Wp, const float* s_w,
                              void* Y, int32_t out_dtype, int32_t* acc_dbg, uint32_t flags,
-                             soniq_stream_t stream) {
+                             void* scratch, size_t scratch_bytes, soniq_stream_t stream) {
+    (void)scratch;
+    (void)scratch_bytes;
     if (cd == nullptr) return SONIQ_ERR_INVALID_ARG;
     if (cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->pad_h < 0 || cd->pad_w < 0 ||
         cd->batch < 0 || cd->H < 1 || cd->W < 1 || cd->C_out < 0)
@@ -387,6 +400,28 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
     return cuda_status(launch_mma(geo, a, as_stream(stream)));
 }
 
+int32_t soniq_mp_gemm_path(const soniq_layout* L, int64_t M, int32_t N, uint32_t flags, size_t scratch_bytes) {
+    LayoutGeom geo;
+    if (make_geom(L, 1, &geo) != SONIQ_OK || M < 1 || N < 1) return -1;
+    if ((flags & SONIQ_FLAG_FORCE_GEMV) && (flags & SONIQ_FLAG_FORCE_MMA)) return -1;
+    const int p = gemm_path(geo, M, N, flags, scratch_bytes);
+    return p < 0 ? -1 : p;
+}
+
+int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout* L, int64_t M, int32_t N, uint32_t flags) {
+    LayoutGeom geo;
+    if (make_geom(L, 1, &geo) != SONIQ_OK || M < 0 || N < 0) return -1;
+    (void)flags;
+    return 0;
+}
+
+int64_t soniq_mp_conv2d_scratch_bytes(const soniq_layout* L, const soniq_conv_desc* cd, uint32_t flags) {
+    LayoutGeom geo;
+    if (cd == nullptr || cd->R < 1 || cd->S < 1 || make_geom(L, cd->R * cd->S, &geo) != SONIQ_OK) return -1;
+    (void)flags;
+    return 0;
+}
+
 soniq_status soniq_sync_status(soniq_stream_t stream) {
     cudaError_t e = cudaStreamSynchronize(as_stream(stream));
     if (e != cudaSuccess) return SONIQ_ERR_CUDA;
@@ -394,15 +429,21 @@ soniq_status soniq_sync_status(soniq_stream_t stream) {
     if (addr == nullptr) return SONIQ_ERR_CUDA;
     unsigned v = 0;
     if (cudaMemcpy(&v, addr, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return SONIQ_ERR_CUDA;
-    if (v != 0) {
-        const unsigned zero = 0;
-        if (cudaMemcpy(addr, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return SONIQ_ERR_CUDA;
-        // an abandoned grid barrier may have left arrivals behind: start it afresh
-        unsigned* bar = grid_barrier_word();
-        if (bar != nullptr && cudaMemset(bar, 0, 2 * sizeof(unsigned)) != cudaSuccess) return SONIQ_ERR_CUDA;
-        return SONIQ_ERR_TIMEOUT;
+    if (v == 0) return SONIQ_OK;
+    if (v & kErrOneshotBarrier) {
+        // The abandoned one-shot barrier kept the arrivals of the CTAs that got
+        // there.  Once no kernel of any stream can still be using it, start it afresh.
+        unsigned* bar = nullptr;
+        float* part = nullptr;
+        if (cudaDeviceSynchronize() != cudaSuccess || !oneshot_scratch(&bar, &part) ||
+            cudaMemset(bar, 0, 2 * sizeof(unsigned)) != cudaSuccess)
+            return SONIQ_ERR_CUDA;
     }
-    return SONIQ_OK;
+    const unsigned zero = 0;
+    if (cudaMemcpy(addr, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return SONIQ_ERR_CUDA;
+    return SONIQ_ERR_TIMEOUT;
 }
+
+void soniq_test_drop_barrier_arrival(int32_t armed) { g_drop_arrival.store(armed != 0 ? 1 : 0); }
 
 }  // extern "C"

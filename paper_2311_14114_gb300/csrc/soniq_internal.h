@@ -36,13 +36,16 @@ soniq_status make_geom(const soniq_layout* L, int32_t taps, LayoutGeom* geo);
 
 // Device address of the library's error word on the current device (0 on failure).
 unsigned* device_error_word();
-// Library scratch on the current device for the one-pass per-tensor quantize
-// (0 on failure): a grid barrier (arrival count, generation) and per-CTA maxima
-// [kMaxGridPartials][2].  One set per device: per-tensor activation quantize
-// calls must not run concurrently on different streams of the same device.
+// Bits of the device error word, by the kind of wait that ran out.
+constexpr unsigned kErrWait = 1u;             // a bounded mbarrier wait (tensor-core kernel, GEMV)
+constexpr unsigned kErrQuantBarrier = 2u;     // grid barrier of the one-pass quantize, caller scratch
+constexpr unsigned kErrOneshotBarrier = 4u;   // grid barrier of soniq_quantize_act_oneshot
+// Caller scratch of the one-pass per-tensor quantize: the barrier words in the
+// first 256 bytes, then the per-CTA maxima [kMaxGridPartials][2].
 constexpr int kMaxGridPartials = 1024;
-unsigned* grid_barrier_word();
-float* grid_partials();
+constexpr int64_t kQuantScratchBytes = 256 + 8 * kMaxGridPartials;
+// True once for the launch that the test hook soniq_test_drop_barrier_arrival armed.
+bool take_drop_arrival();
 void note_launch(int n = 1);
 int num_sms();
 // Asks for the largest shared-memory carve-out for `func` (once per device):
@@ -59,10 +62,11 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
                                 cudaStream_t st);
 // One-pass per-tensor quantize (cooperative launch); its grid barrier (two
 // words, zero between launches) and per-CTA maxima [max_ctas][2] are `bar` and
-// `part`.  cudaErrorNotSupported when the rows do not fit on chip.
+// `part`; a barrier wait that runs out ORs `err_bit` into the error word.
+// cudaErrorNotSupported when the rows do not fit on chip.
 cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
                                   float* s_a, uint8_t* Ap, cudaStream_t st, unsigned* bar, float* part,
-                                  int max_ctas);
+                                  int max_ctas, unsigned err_bit);
 cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, const float* W,
                                  int32_t N, float* s_out, cudaStream_t st);
 cudaError_t launch_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W,

@@ -23,11 +23,14 @@ STATUS_NAMES = {0: "SONIQ_OK", 1: "SONIQ_ERR_INVALID_ARG", 2: "SONIQ_ERR_UNSUPPO
 SCALE_PER_TENSOR, SCALE_PER_ROW, SCALE_CALIBRATED = 0, 1, 2
 OUT_F16, OUT_BF16 = 0, 1
 FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_TEST_DROP_ARRIVE = 1, 2, 0x100
+PATH_NAMES = {0: "CUDA-core GEMV", 1: "tensor-core kernel"}
 
 EXPORTED = ["soniq_abi_version", "soniq_status_string", "soniq_group_codes",
             "soniq_packed_row_bytes", "soniq_validate_layout", "soniq_launch_count",
-            "soniq_pack_weights", "soniq_quantize_act", "soniq_quantize_act_oneshot", "soniq_mp_gemm",
-            "soniq_mp_conv2d", "soniq_sync_status"]
+            "soniq_pack_weights", "soniq_quantize_act", "soniq_quantize_act_scratch_bytes",
+            "soniq_quantize_act_oneshot", "soniq_mp_gemm", "soniq_mp_gemm_path", "soniq_mp_gemm_scratch_bytes",
+            "soniq_mp_conv2d", "soniq_mp_conv2d_scratch_bytes", "soniq_sync_status",
+            "soniq_test_drop_barrier_arrival"]
 
 _SCALE = {"tensor": SCALE_PER_TENSOR, "row": SCALE_PER_ROW, "calibrated": SCALE_CALIBRATED}
 
@@ -75,16 +78,26 @@ def lib() -> ctypes.CDLL:
         L.soniq_launch_count.restype = i64
         L.soniq_pack_weights.argtypes = [P, P, i32, i32, i32, P, P, P]
         L.soniq_pack_weights.restype = i32
-        L.soniq_quantize_act.argtypes = [P, P, i64, i32, P, P, P]
+        L.soniq_quantize_act.argtypes = [P, P, i64, i32, P, P, P, ctypes.c_size_t, P]
         L.soniq_quantize_act.restype = i32
+        L.soniq_quantize_act_scratch_bytes.argtypes = [P, i64, i32]
+        L.soniq_quantize_act_scratch_bytes.restype = i64
         L.soniq_quantize_act_oneshot.argtypes = [P, P, i64, P, P, P]
         L.soniq_quantize_act_oneshot.restype = i32
-        L.soniq_mp_gemm.argtypes = [P, P, P, i32, i64, P, P, i32, P, i32, P, u32, P]
+        L.soniq_mp_gemm.argtypes = [P, P, P, i32, i64, P, P, i32, P, i32, P, u32, P, ctypes.c_size_t, P]
         L.soniq_mp_gemm.restype = i32
-        L.soniq_mp_conv2d.argtypes = [P, P, P, P, i32, P, P, P, i32, P, u32, P]
+        L.soniq_mp_gemm_path.argtypes = [P, i64, i32, u32, ctypes.c_size_t]
+        L.soniq_mp_gemm_path.restype = i32
+        L.soniq_mp_gemm_scratch_bytes.argtypes = [P, i64, i32, u32]
+        L.soniq_mp_gemm_scratch_bytes.restype = i64
+        L.soniq_mp_conv2d.argtypes = [P, P, P, P, i32, P, P, P, i32, P, u32, P, ctypes.c_size_t, P]
         L.soniq_mp_conv2d.restype = i32
+        L.soniq_mp_conv2d_scratch_bytes.argtypes = [P, P, u32]
+        L.soniq_mp_conv2d_scratch_bytes.restype = i64
         L.soniq_sync_status.argtypes = [P]
         L.soniq_sync_status.restype = i32
+        L.soniq_test_drop_barrier_arrival.argtypes = [i32]
+        L.soniq_test_drop_barrier_arrival.restype = None
         _lib = L
     return _lib
 
@@ -106,6 +119,33 @@ def _stream(stream=None):
 def _need(t: torch.Tensor, dtype, name: str):
     if not t.is_cuda or t.dtype != dtype or not t.is_contiguous():
         raise ValueError(f"{name} must be a contiguous CUDA {dtype} tensor")
+
+
+# Scratch buffers the binding hands to the library, one per (device, stream):
+# calls on one stream run in order, so they may share it; calls on different
+# streams get different buffers.  Each is zero-filled when created (the
+# quantize barrier must start at zero) and grows by reallocation when a call
+# needs more.
+_scratch = {}
+
+
+def _get_scratch(nbytes: int, device, stream) -> Optional[torch.Tensor]:
+    if nbytes <= 0:
+        return None
+    s = torch.cuda.current_stream(device) if stream is None else stream
+    key = (torch.device(device).index, s.cuda_stream)
+    buf = _scratch.get(key)
+    if buf is None or buf.numel() < nbytes:
+        with torch.cuda.stream(s):
+            buf = torch.zeros(((nbytes + 255) // 256) * 256, dtype=torch.uint8, device=device)
+        _scratch[key] = buf
+    return buf
+
+
+def reset_scratch():
+    """Zero every cached scratch buffer (needed after a SONIQ_ERR_TIMEOUT)."""
+    for buf in _scratch.values():
+        buf.zero_()
 
 
 class Layout:
@@ -165,9 +205,11 @@ def pack_weights(layout: Layout, W: torch.Tensor, scale_mode: str = "row",
 
 def quantize_act(layout: Layout, A: torch.Tensor, scale_mode: str = "tensor",
                  s_a: Optional[torch.Tensor] = None, Ap: Optional[torch.Tensor] = None,
-                 stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+                 stream=None, scratch: Optional[torch.Tensor] = False) -> Tuple[torch.Tensor, torch.Tensor]:
     """soniq_quantize_act.  A: fp16 [M][K] on the GPU.  For scale_mode
-    'calibrated', s_a ([2] fp32) is an input."""
+    'calibrated', s_a ([2] fp32) is an input.  scratch: a zero-filled uint8
+    CUDA tensor, None for no scratch (two-pass per-tensor path), or left out
+    for the binding's per-stream buffer."""
     _need(A, torch.float16, "A")
     M = A.shape[0]
     mode = _SCALE[scale_mode]
@@ -178,8 +220,12 @@ def quantize_act(layout: Layout, A: torch.Tensor, scale_mode: str = "tensor",
                           device=A.device)
     if Ap is None:
         Ap = torch.empty((M, layout.row_bytes(False)), dtype=torch.uint8, device=A.device)
+    if scratch is False:
+        need = int(lib().soniq_quantize_act_scratch_bytes(ctypes.byref(layout.c), M, mode))
+        scratch = _get_scratch(need, A.device, stream)
+    nbytes = 0 if scratch is None else scratch.numel() * scratch.element_size()
     _check(lib().soniq_quantize_act(ctypes.byref(layout.c), _ptr(A), M, mode, _ptr(s_a), _ptr(Ap),
-                                    _stream(stream)), "soniq_quantize_act")
+                                    _ptr(scratch), nbytes, _stream(stream)), "soniq_quantize_act")
     return Ap, s_a
 
 
@@ -207,10 +253,21 @@ def mp_gemm(layout: Layout, Ap: torch.Tensor, s_a: torch.Tensor, Wp: torch.Tenso
     if Y is None:
         Y = torch.empty((M, N), dtype=out_dtype, device=Ap.device)
     od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
+    need = int(lib().soniq_mp_gemm_scratch_bytes(ctypes.byref(layout.c), M, N, int(flags)))
+    scratch = _get_scratch(need, Ap.device, stream)
     _check(lib().soniq_mp_gemm(ctypes.byref(layout.c), _ptr(Ap), _ptr(s_a), _SCALE[scale_mode], M,
                                _ptr(Wp), _ptr(s_w), N, _ptr(Y), od, _ptr(acc_dbg), int(flags),
-                               _stream(stream)), "soniq_mp_gemm")
+                               _ptr(scratch), max(need, 0), _stream(stream)), "soniq_mp_gemm")
     return Y
+
+
+def gemm_path(layout: Layout, M: int, N: int, flags: int = 0) -> str:
+    """soniq_mp_gemm_path: the kernel soniq_mp_gemm runs for these arguments."""
+    need = max(int(lib().soniq_mp_gemm_scratch_bytes(ctypes.byref(layout.c), M, N, int(flags))), 0)
+    p = int(lib().soniq_mp_gemm_path(ctypes.byref(layout.c), M, N, int(flags), need))
+    if p < 0:
+        raise SoniqError(SONIQ_ERR_INVALID_ARG, "soniq_mp_gemm_path")
+    return PATH_NAMES.get(p, str(p))
 
 
 def conv_desc(batch, H, W, C_out, R=3, S=3, stride=(1, 1), pad=(1, 1)) -> CConvDesc:
@@ -232,15 +289,30 @@ def mp_conv2d(layout: Layout, cd: CConvDesc, Xp: torch.Tensor, s_a: torch.Tensor
     if Y is None:
         Y = torch.empty((cd.batch, P, Q, cd.C_out), dtype=out_dtype, device=Xp.device)
     od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
+    need = int(lib().soniq_mp_conv2d_scratch_bytes(ctypes.byref(layout.c), ctypes.byref(cd), int(flags)))
+    scratch = _get_scratch(need, Xp.device, stream)
     _check(lib().soniq_mp_conv2d(ctypes.byref(layout.c), ctypes.byref(cd), _ptr(Xp), _ptr(s_a),
                                  _SCALE[scale_mode], _ptr(Wp), _ptr(s_w), _ptr(Y), od,
-                                 _ptr(acc_dbg), int(flags), _stream(stream)), "soniq_mp_conv2d")
+                                 _ptr(acc_dbg), int(flags), _ptr(scratch), max(need, 0),
+                                 _stream(stream)), "soniq_mp_conv2d")
     return Y
 
 
 def sync_status(stream=None) -> int:
-    """soniq_sync_status: waits for the stream, returns the status code."""
-    return int(lib().soniq_sync_status(_stream(stream)))
+    """soniq_sync_status: waits for the stream, returns the status code.  After
+    a timeout the binding's scratch buffers are zeroed again (the contract of
+    the scratch-taking calls)."""
+    st = int(lib().soniq_sync_status(_stream(stream)))
+    if st == SONIQ_ERR_TIMEOUT:
+        torch.cuda.synchronize()
+        reset_scratch()
+        torch.cuda.synchronize()
+    return st
+
+
+def test_drop_barrier_arrival(armed: bool = True):
+    """soniq_test_drop_barrier_arrival (test hook)."""
+    lib().soniq_test_drop_barrier_arrival(1 if armed else 0)
 
 
 def launch_count() -> int:

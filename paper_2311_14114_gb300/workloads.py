@@ -167,6 +167,12 @@ def sweep_specs() -> List[LinearSpec]:
     return out
 
 
+# The precision-sweep point the benchmark headline is quoted on: 4-bit low,
+# 8-bit high, 25 % of the 4096 channels (1024) at 8 bits.
+SWEEP_HEADLINE = LinearSpec("sweep_8192x4096x4096_lo4_hi8_f25", M=8192, K=4096, N=4096, bits_lo=4,
+                            bits_hi=8, frac_hi=0.25)
+
+
 def random_linear(seed: int, M: int, K: int, N: int, bits_lo: int, bits_hi: int,
                   frac_hi: float, n_outliers: int = 0, outlier_scale: float = 8.0):
     """Small seeded case for parity sweeps."""

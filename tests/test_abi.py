@@ -39,7 +39,7 @@ def test_library_exports_every_declared_symbol(L):
     for name in names:
         assert hasattr(L, name), name
     assert sorted(soniq.EXPORTED) == names
-    assert L.soniq_abi_version() == 1
+    assert L.soniq_abi_version() == 2
 
 
 def _layout(soniq, K=300, count=(200, 100), bits=(3, 8), pad=128, perm=None):
@@ -92,25 +92,43 @@ def test_host_side_argument_errors_need_no_gpu(L):
     # misaligned packed weights
     assert L.soniq_pack_weights(ctypes.byref(lay), fake, 10, 1, 1, ctypes.c_void_p(4097 + 3), fake, None) == 3
     # bad scale mode
-    assert L.soniq_quantize_act(ctypes.byref(lay), fake, 10, 7, fake, fake, None) == 1
+    assert L.soniq_quantize_act(ctypes.byref(lay), fake, 10, 7, fake, fake, None, 0, None) == 1
     # empty input is a no-op that touches nothing
-    assert L.soniq_quantize_act(ctypes.byref(lay), None, 0, 0, None, None, None) == 0
-    assert L.soniq_mp_gemm(ctypes.byref(lay), None, None, 0, 0, None, None, 5, None, 0, None, 0, None) == 0
+    assert L.soniq_quantize_act(ctypes.byref(lay), None, 0, 0, None, None, None, 0, None) == 0
+    # misaligned scratch
+    assert L.soniq_quantize_act(ctypes.byref(lay), fake, 10, 0, fake, fake, ctypes.c_void_p(4100), 9000,
+                                None) == 3
+    assert L.soniq_mp_gemm(ctypes.byref(lay), None, None, 0, 0, None, None, 5, None, 0, None, 0, None, 0, None) == 0
     # both dispatch overrides at once
-    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 3, None) == 1
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 3, None, 0, None) == 1
     # bad output dtype
-    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 9, None, 0, None) == 1
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 9, None, 0, None, 0, None) == 1
     # conv: per-row activation scales are rejected (a dot product spans pixels)
     cd = soniq.conv_desc(1, 8, 8, 16)
     assert L.soniq_mp_conv2d(ctypes.byref(lay), ctypes.byref(cd), fake, fake, 1, fake, fake, fake, 0,
-                             None, 0, None) == 1
+                             None, 0, None, 0, None) == 1
     # conv: filter larger than the padded image
     cd = soniq.conv_desc(1, 2, 2, 16, R=5, S=5, pad=(0, 0))
     assert L.soniq_mp_conv2d(ctypes.byref(lay), ctypes.byref(cd), fake, fake, 0, fake, fake, fake, 0,
-                             None, 0, None) == 1
+                             None, 0, None, 0, None) == 1
     # K beyond the supported range
     big = _layout(soniq, K=70000, count=(70000, 0), bits=(2, 2), perm=ctypes.c_void_p(16))
-    assert L.soniq_mp_gemm(ctypes.byref(big), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 0, None) == 2
+    assert L.soniq_mp_gemm(ctypes.byref(big), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 0, None, 0, None) == 2
+
+
+def test_scratch_size_queries(L):
+    """The per-tensor quantize asks for a barrier and per-CTA maxima; the other
+    activation modes ask for nothing; bad layouts give -1 (host only)."""
+    from paper_2311_14114_gb300 import soniq
+    lay = _layout(soniq, perm=ctypes.c_void_p(16))
+    L.soniq_quantize_act_scratch_bytes.restype = ctypes.c_int64
+    L.soniq_quantize_act_scratch_bytes.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32]
+    assert L.soniq_quantize_act_scratch_bytes(ctypes.byref(lay), 1000, 0) == 256 + 8 * 1024
+    assert L.soniq_quantize_act_scratch_bytes(ctypes.byref(lay), 1000, 1) == 0
+    assert L.soniq_quantize_act_scratch_bytes(ctypes.byref(lay), 1000, 2) == 0
+    assert L.soniq_quantize_act_scratch_bytes(ctypes.byref(lay), 1000, 9) == -1
+    bad = _layout(soniq, count=(200, 99))
+    assert L.soniq_quantize_act_scratch_bytes(ctypes.byref(bad), 1000, 0) == -1
 
 
 def test_status_strings(L):

@@ -21,8 +21,20 @@ def test_reference_arm_prints_one_contract_line():
     assert line["impl"] == "reference"
     assert line["steps"] == 2 and line["warmup"] == 1 and line["n_gpus"] == 1
     assert line["value"] > 0 and line["unit"] == "TOPS" and line["higher_is_better"] is True
-    assert line["config"]["workload"].startswith("conv_resnet18")
+    from paper_2311_14114_gb300 import workloads as wl
+    assert line["config"]["workload"] == wl.SWEEP_HEADLINE.name
+    for key in ("M", "N", "K", "bits", "count", "parallelism", "l2", "launch"):
+        assert key in line["config"], key
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["cpu_baseline"]["value"] == line["value"]
     assert line["e2e"]["value"] == line["value"] and line["e2e"]["unit"] == line["unit"]
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
+
+
+def test_cpu_baseline_worker_reports_a_sampled_step():
+    env = dict(os.environ, OMP_NUM_THREADS="2")
+    r = subprocess.run([sys.executable, "bench.py", "--oracle-worker", "--cpu-seconds", "1"],
+                       cwd=ROOT, capture_output=True, text=True, timeout=600, env=env)
+    assert r.returncode == 0, r.stderr[-2000:]
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    assert res["t_q"] > 0 and res["t_acc"] > 0 and 8 <= res["rows"] <= res["M"] == 8192

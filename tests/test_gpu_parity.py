@@ -421,3 +421,42 @@ def test_timeout_is_reported_and_context_survives(sq):
     assert sq.sync_status() == 5            # SONIQ_ERR_TIMEOUT, then cleared
     assert sq.sync_status() == 0
     check_linear(sq, d, flags=2, what="after timeout")
+
+
+def test_quantize_barrier_timeout_is_reported_and_scratch_recovers(sq):
+    """The one-pass per-tensor quantize with caller scratch: a dropped barrier
+    arrival (host-armed test hook) runs the other CTAs' bounded waits out; the
+    call reports SONIQ_ERR_TIMEOUT, the binding zeroes its scratch as the
+    contract asks, and the next calls are exact."""
+    d = wl.random_linear(401, M=2000, K=640, N=8, bits_lo=3, bits_hi=8, frac_hi=0.3, n_outliers=2)
+    lay = sq.Layout(d["perm"], d["count"], d["bits"])
+    A = _dev(d["A"])
+    assert sq.sync_status() == 0
+    sq.test_drop_barrier_arrival(True)
+    sq.quantize_act(lay, A, "tensor")
+    assert sq.sync_status() == sq.SONIQ_ERR_TIMEOUT
+    assert sq.sync_status() == 0
+    A32 = d["A"].astype(np.float32)
+    s_ref = oracle.act_scales(A32, d["perm"], d["count"])
+    Ap_ref = oracle.pack_act_rows(oracle.act_codes(A32, d["perm"], d["count"], d["bits"], s_ref),
+                                  d["count"], d["bits"], 128)
+    for _ in range(2):
+        Ap, s_a = sq.quantize_act(lay, A, "tensor")
+        assert sq.sync_status() == 0
+        assert np.array_equal(s_a.cpu().numpy(), s_ref)
+        assert np.array_equal(Ap.cpu().numpy(), Ap_ref)
+
+
+@pytest.mark.parametrize("K", [512, 3000])
+def test_quantize_per_tensor_without_scratch_two_pass(sq, K):
+    """scratch = NULL takes the two-pass per-tensor path (max-abs pass, then quantize)."""
+    d = wl.random_linear(402, M=500, K=K, N=8, bits_lo=2, bits_hi=8, frac_hi=0.3, n_outliers=2)
+    lay = sq.Layout(d["perm"], d["count"], d["bits"], pad_unit=32)
+    Ap, s_a = sq.quantize_act(lay, _dev(d["A"]), "tensor", scratch=None)
+    assert sq.sync_status() == 0
+    A32 = d["A"].astype(np.float32)
+    s_ref = oracle.act_scales(A32, d["perm"], d["count"])
+    Ap_ref = oracle.pack_act_rows(oracle.act_codes(A32, d["perm"], d["count"], d["bits"], s_ref),
+                                  d["count"], d["bits"], 32)
+    assert np.array_equal(s_a.cpu().numpy(), s_ref)
+    assert np.array_equal(Ap.cpu().numpy(), Ap_ref)
