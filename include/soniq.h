@@ -107,16 +107,20 @@ enum { SONIQ_OUT_F16 = 0, SONIQ_OUT_BF16 = 1 };
 
 enum {
     SONIQ_FLAG_FORCE_GEMV = 1u,          /* soniq_mp_gemm: use the CUDA-core GEMV for any M <= 16 */
-    SONIQ_FLAG_FORCE_MMA = 2u,           /* soniq_mp_gemm: use the tensor-core kernel for any M */
-    SONIQ_FLAG_TEST_DROP_ARRIVE = 0x100u /* test hook: the tensor-core kernel's operand producer
-                                            skips its first arrival, so the consumer's bounded
-                                            wait runs out and the call reports SONIQ_ERR_TIMEOUT */
+    SONIQ_FLAG_FORCE_MMA = 2u,           /* soniq_mp_gemm: use a tensor-core kernel for any M */
+    SONIQ_FLAG_FORCE_FUSED = 4u,         /* tensor-core work takes the fused kernel even when
+                                            scratch for the staged path is given */
+    SONIQ_FLAG_TEST_DROP_ARRIVE = 0x100u /* test hook: the tensor-core kernels' operand producer
+                                            skips its first arrival (fused) or its first K-stage
+                                            (staged), so the consumer's bounded wait runs out and
+                                            the call reports SONIQ_ERR_TIMEOUT */
 };
 
 /* Kernels behind soniq_mp_gemm (see soniq_mp_gemm_path). */
 enum {
-    SONIQ_PATH_GEMV = 0,    /* CUDA-core GEMV streaming the packed weights (small M) */
-    SONIQ_PATH_TENSOR = 1   /* tcgen05 tensor-core kernel expanding packed tiles on chip */
+    SONIQ_PATH_GEMV = 0,           /* CUDA-core GEMV streaming the packed weights (small M) */
+    SONIQ_PATH_TENSOR = 1,         /* tcgen05 kernel expanding packed tiles on chip (no scratch) */
+    SONIQ_PATH_TENSOR_STAGED = 2   /* codes expanded once into scratch, then a tcgen05 GEMM */
 };
 /* Without flags, soniq_mp_gemm runs the GEMV for M <= SONIQ_GEMV_MAX_M. */
 #define SONIQ_GEMV_MAX_M 12
@@ -275,6 +279,16 @@ SONIQ_API soniq_status soniq_mp_gemm(const soniq_layout *layout, const uint8_t *
                            int32_t N, void *Y, int32_t out_dtype, int32_t *acc_dbg,
                            uint32_t flags, void *scratch, size_t scratch_bytes,
                            soniq_stream_t stream);
+
+/* Scratch of soniq_mp_gemm and soniq_mp_conv2d.  With scratch (256-byte
+ * aligned) of at least the *_scratch_bytes() size, the tensor-core work takes
+ * the staged path: every packed code is expanded once into tensor-pipe
+ * operands in the scratch (E4M3 bytes for groups of <= 4-bit codes, fp16 for
+ * wider ones; a convolution's activations as implicit-GEMM rows), and a
+ * persistent tcgen05 GEMM reads them.  Without it (scratch = NULL or too
+ * small) the fused kernel expands packed tiles on chip.  Both give the same
+ * bits.  The scratch needs no initialization; calls that may overlap on the
+ * GPU must use different scratch buffers. */
 
 /* The kernel soniq_mp_gemm runs for these arguments (SONIQ_PATH_*), or -1
  * if it would return an error.  Host only (reads the device's SM count). */

@@ -164,16 +164,24 @@ cudaStream_t as_stream(soniq_stream_t s) { return reinterpret_cast<cudaStream_t>
 // tensor-core kernel would be chosen but cannot take the layout (mma_check
 // says why), -2 when the GEMV was forced but cannot take the shape.
 int gemm_path(const LayoutGeom& geo, int64_t M, int32_t N, uint32_t flags, size_t scratch_bytes) {
-    (void)scratch_bytes;
     // up to SONIQ_GEMV_MAX_M rows the CUDA-core GEMV is faster; above, the tensor-core
-    // kernel (whose time hardly grows with M below 128) overtakes it (decode N=11008,
-    // K=4096: 47.6 vs 41.5 us at M=16)
+    // kernels (whose time hardly grows with M below 128) overtake it
     const bool want_gemv =
         (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= SONIQ_GEMV_MAX_M && !(flags & SONIQ_FLAG_FORCE_MMA));
     if (want_gemv && gemv_supported(geo, M, N)) return SONIQ_PATH_GEMV;
     if (flags & SONIQ_FLAG_FORCE_GEMV) return -2;
+    if (!(flags & SONIQ_FLAG_FORCE_FUSED)) {
+        const int64_t need = staged_scratch_bytes(geo, M, N);
+        if (need > 0 && (int64_t)scratch_bytes >= need) return SONIQ_PATH_TENSOR_STAGED;
+    }
     if (mma_check(geo) != SONIQ_OK) return -1;
     return SONIQ_PATH_TENSOR;
+}
+
+int64_t conv_rows(const soniq_conv_desc* cd) {
+    const int64_t P = (cd->H + 2 * cd->pad_h - cd->R) / cd->stride_h + 1;
+    const int64_t Q = (cd->W + 2 * cd->pad_w - cd->S) / cd->stride_w + 1;
+    return (int64_t)cd->batch * P * Q;
 }
 
 soniq_status check_scale_mode_act(int32_t mode) {
@@ -308,7 +316,6 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
                            int64_t M, const uint8_t* Wp, const float* s_w, int32_t N, void* Y,
                            int32_t out_dtype, int32_t* acc_dbg, uint32_t flags, void* scratch,
                            size_t scratch_bytes, soniq_stream_t stream) {
-    (void)scratch;
     LayoutGeom geo;
     soniq_status st = make_geom(L, 1, &geo);
     if (st != SONIQ_OK) return st;
@@ -325,12 +332,13 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     // K <= 65536 keeps |Acc| < 2^31 and the GEMV's unsigned offset sums below 2^32
     const int per_row = scale_mode == SONIQ_SCALE_PER_ROW;
     cudaStream_t s = as_stream(stream);
-    const int path = gemm_path(geo, M, N, flags, scratch_bytes);
+    const int path = gemm_path(geo, M, N, flags, scratch != nullptr ? scratch_bytes : 0);
     if (path < 0) return path == -2 ? SONIQ_ERR_UNSUPPORTED : mma_check(geo);
     if (path == SONIQ_PATH_GEMV) {
         GemvArgs a{Ap, Wp, s_a, s_w, Y, acc_dbg, (int32_t)M, N, per_row, out_dtype == SONIQ_OUT_BF16};
         return cuda_status(launch_gemv(geo, a, s));
     }
+    if (path == SONIQ_PATH_TENSOR_STAGED && !aligned(scratch, 256)) return SONIQ_ERR_ALIGNMENT;
     MmaArgs a{};
     a.Ap = Ap;
     a.Wp = Wp;
@@ -344,6 +352,7 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     a.out_bf16 = out_dtype == SONIQ_OUT_BF16;
     a.flags = flags;
     a.conv = 0;
+    if (path == SONIQ_PATH_TENSOR_STAGED) return cuda_status(launch_staged(geo, a, scratch, scratch_bytes, s));
     return cuda_status(launch_mma(geo, a, s));
 }
 
@@ -351,8 +360,6 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
                              const float* s_a, int32_t scale_mode, const uint8_t* Wp, const float* s_w,
                              void* Y, int32_t out_dtype, int32_t* acc_dbg, uint32_t flags,
                              void* scratch, size_t scratch_bytes, soniq_stream_t stream) {
-    (void)scratch;
-    (void)scratch_bytes;
     if (cd == nullptr) return SONIQ_ERR_INVALID_ARG;
     if (cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->pad_h < 0 || cd->pad_w < 0 ||
         cd->batch < 0 || cd->H < 1 || cd->W < 1 || cd->C_out < 0)
@@ -373,7 +380,11 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
     if (!aligned(Xp, 4) || !aligned(Wp, 16) || !aligned(Y, 16) || !aligned(s_a, 4) || !aligned(s_w, 4) ||
         (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
         return SONIQ_ERR_ALIGNMENT;
-    if ((st = mma_check(geo)) != SONIQ_OK) return st;
+    const bool staged = !(flags & SONIQ_FLAG_FORCE_FUSED) && scratch != nullptr &&
+                        staged_scratch_bytes(geo, M, cd->C_out) > 0 &&
+                        (int64_t)scratch_bytes >= staged_scratch_bytes(geo, M, cd->C_out);
+    if (staged && !aligned(scratch, 256)) return SONIQ_ERR_ALIGNMENT;
+    if (!staged && (st = mma_check(geo)) != SONIQ_OK) return st;
     MmaArgs a{};
     a.Ap = Xp;
     a.Wp = Wp;
@@ -397,6 +408,7 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
     a.sw = cd->stride_w;
     a.ph = cd->pad_h;
     a.pw = cd->pad_w;
+    if (staged) return cuda_status(launch_staged(geo, a, scratch, scratch_bytes, as_stream(stream)));
     return cuda_status(launch_mma(geo, a, as_stream(stream)));
 }
 
@@ -411,15 +423,22 @@ int32_t soniq_mp_gemm_path(const soniq_layout* L, int64_t M, int32_t N, uint32_t
 int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout* L, int64_t M, int32_t N, uint32_t flags) {
     LayoutGeom geo;
     if (make_geom(L, 1, &geo) != SONIQ_OK || M < 0 || N < 0) return -1;
-    (void)flags;
-    return 0;
+    if (M == 0 || N == 0 || (flags & SONIQ_FLAG_FORCE_FUSED)) return 0;
+    // the GEMV needs none
+    const bool want_gemv =
+        (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= SONIQ_GEMV_MAX_M && !(flags & SONIQ_FLAG_FORCE_MMA));
+    if (want_gemv) return 0;
+    return staged_scratch_bytes(geo, M, N);
 }
 
 int64_t soniq_mp_conv2d_scratch_bytes(const soniq_layout* L, const soniq_conv_desc* cd, uint32_t flags) {
     LayoutGeom geo;
-    if (cd == nullptr || cd->R < 1 || cd->S < 1 || make_geom(L, cd->R * cd->S, &geo) != SONIQ_OK) return -1;
-    (void)flags;
-    return 0;
+    if (cd == nullptr || cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->batch < 0 ||
+        cd->C_out < 0 || make_geom(L, cd->R * cd->S, &geo) != SONIQ_OK)
+        return -1;
+    if (cd->H + 2 * cd->pad_h < cd->R || cd->W + 2 * cd->pad_w < cd->S) return -1;
+    if (flags & SONIQ_FLAG_FORCE_FUSED) return 0;
+    return staged_scratch_bytes(geo, conv_rows(cd), cd->C_out);
 }
 
 soniq_status soniq_sync_status(soniq_stream_t stream) {

@@ -109,4 +109,31 @@ struct MmaArgs {
 soniq_status mma_check(const LayoutGeom& geo);
 cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st);
 
+// ---- the staged tensor-core path (staged_gemm.cu) ---------------------------
+// Packed codes are expanded once into tensor-pipe operands in caller scratch
+// (E4M3 bytes for groups with <= 4-bit codes on both sides, fp16 otherwise),
+// then a persistent tcgen05 GEMM runs over them.
+struct StagedGroup {
+    int32_t kind;          // 0: E4M3, 1: fp16
+    int32_t stages;        // 128-byte K-stages
+    int32_t x0;            // byte offset of the group in an expanded row
+    int32_t seg_stages;    // K-stages per exact fp32 segment
+    int32_t n_seg;         // segments (> 1: drained to int32)
+    int32_t center;        // fp16 activations are stored as u - center
+};
+struct StagedPlan {
+    StagedGroup g[2];
+    int64_t eb;            // bytes of an expanded row (both groups)
+    int32_t seg_group;     // the group that needs segments, or -1
+};
+// False when the layout cannot take the staged path (two segmented groups).
+bool staged_plan(const LayoutGeom& geo, StagedPlan* sp);
+// Scratch bytes of the staged path for rows_a activation rows (conv: output
+// pixels) and N weight rows; 0 if the layout cannot take it.
+int64_t staged_scratch_bytes(const LayoutGeom& geo, int64_t rows_a, int64_t N);
+// Expansion kernels and the GEMM on `st`; cudaErrorNotSupported if the
+// scratch is too small.
+cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch, size_t scratch_bytes,
+                          cudaStream_t st);
+
 }  // namespace soniq

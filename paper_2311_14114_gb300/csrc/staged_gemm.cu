@@ -1,0 +1,715 @@
+// Staged mixed-precision GEMM / implicit-GEMM convolution on the sm_103a
+// tensor cores: expand the packed codes once into tensor-pipe operands in
+// caller scratch, then run a persistent tcgen05 GEMM over them.
+//
+// What it computes (Sec. 3 "Enabling Low-Cost Fixed-Point Operations";
+// Sec. 4.2): for each precision group g the exact integer dot products
+//   Acc_g[m][n] = sum over k in group g of u[m][k] * j[n][k]
+// and Y = sum_g s_a * s_w * Acc_g / ((2^na - 1) * 2^(nw - 1)) in fp32.
+//
+// Why staged.  Expanding packed codes inside the GEMM tiles (the fused
+// kernel of mma_gemm.cu) repeats the expansion of every activation row once
+// per column tile and of every weight row once per row tile, and that work,
+// not the tensor pipe, sets its speed.  Here each code is expanded exactly
+// once, by a streaming kernel, into a byte layout the MMA reads directly;
+// the expanded operands (e.g. 63 MB for an 8192 x 4096 x 4096 layer) stay
+// in the 129 MB L2 while the GEMM reads them.
+//
+// Operand encodings (all exact; one group at a time along K):
+//   * groups with <= 4-bit codes on both sides: E4M3 bytes.  An activation
+//     code u < 16 as a raw byte is the E4M3 value u * 2^-9; a weight code j in
+//     [-8, 7] is stored sign-magnitude, the E4M3 value j * 2^-9.  The fp32
+//     accumulator holds sum u*j * 2^-18 exactly (|sum| <= 65536 * 15 * 8 <
+//     2^24), so the epilogue scales by 2^18.
+//   * wider groups: fp16.  Activations are centred, u - 2^(na-1) (padding and
+//     taps outside the image count as u = 0), weights are j; every product
+//     and partial sum is an integer.  The epilogue adds back
+//     2^(na-1) * C[n] with C[n] the weight row's code sum (from the expander).
+//     A partial sum stays exact while |sum| <= 2^24; a group whose worst case
+//     over its K range could exceed that is accumulated in segments that the
+//     epilogue warps drain into int32 registers.
+//
+// The GEMM kernel: persistent CTAs (one per SM) walk 128 x 128 output tiles.
+//   warp 0     TMA producer: per 128-byte K-stage, one A and one B box (16 KB
+//              each, 128-byte swizzle) into a 6-stage ring
+//   warp 1     TMEM owner and MMA issuer (one thread): 4 MMAs per K-stage into
+//              the tile's accumulators; two accumulator sets (2 x 2 groups x
+//              128 columns = all 512 TMEM columns), so one tile's epilogue
+//              overlaps the next tile's mainloop
+//   warps 2-9  epilogue: two warps per TMEM lane quadrant, 64 columns each
+// Every wait is bounded (2 s); a wait that runs out records an error bit,
+// raises a CTA abort flag and the CTA winds down (copies and MMAs in flight
+// are waited for, TMEM is freed).
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <cstring>
+
+#include "soniq_device.cuh"
+#include "soniq_internal.h"
+#include "tc_ptx.cuh"
+
+namespace soniq {
+namespace staged {
+
+using namespace tc;
+
+constexpr int BM = 128;
+constexpr int BN = 128;
+constexpr int STAGES = 6;
+constexpr int A_BYTES = BM * 128;
+constexpr int B_BYTES = BN * 128;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int WARP_TMA = 0, WARP_MMA = 1, WARP_EPI = 2;
+constexpr int NUM_THREADS = (2 + NUM_EPI_WARPS) * 32;
+constexpr int BAR_FULL = 0, BAR_EMPTY = STAGES, BAR_ACC_FULL = 2 * STAGES, BAR_ACC_EMPTY = 2 * STAGES + 2,
+              BAR_SEG_FULL = 2 * STAGES + 4, BAR_SEG_FREE = 2 * STAGES + 6, BAR_TEARDOWN = 2 * STAGES + 8,
+              NUM_BARS = 2 * STAGES + 9;
+constexpr int SMEM_BAR = STAGES * STAGE_BYTES;
+constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;   // tmem base, abort flag, a zero word
+constexpr int SMEM_TOTAL = SMEM_MISC + 16;
+constexpr int SMEM_ALLOC = SMEM_TOTAL + 1024;        // slack for 1024-byte alignment
+constexpr uint32_t IDESC = idesc(BM, BN);
+constexpr long long kTimeoutNs = 2000000000LL;
+
+struct SGroup {
+    int32_t kind;          // 0: E4M3 bytes, 1: fp16
+    int32_t stages;        // 128-byte K-stages of the group
+    int32_t x0;            // byte offset of the group in an expanded row
+    int32_t seg_stages;    // K-stages per exact segment (segmented group only)
+    int32_t n_seg;         // segments (1: accumulated in one piece)
+    int32_t center;        // fp16 activations carry -center; the epilogue adds center * C[n]
+    float acc_scale;       // 2^18 (E4M3) or 1 (fp16)
+    float inv_levels;      // 1 / ((2^na - 1) * 2^(nw - 1))
+};
+
+struct SParams {
+    CUtensorMap tma_a;     // expanded activations [rows][eb]
+    CUtensorMap tma_b;     // expanded weights [N][eb]
+    const float* s_a;
+    const float* s_w;
+    const int32_t* colsum; // [N][2] weight code sums
+    void* Y;
+    int32_t* acc_dbg;
+    unsigned* err;
+    int64_t M;
+    int32_t N;
+    int32_t m_tiles, n_tiles, total_tiles;
+    int32_t s_a_per_row;
+    int32_t out_bf16;
+    int32_t seg_group;     // group accumulated in drained segments, or -1
+    int32_t drop_first;    // test hook: the producer never issues the first K-stage
+    SGroup g[2];
+};
+
+// ---------------------------------------------------------------------------
+// Expansion of packed rows into tensor-pipe operands
+// ---------------------------------------------------------------------------
+
+struct ExpandParams {
+    const uint8_t* src;        // packed rows
+    int64_t src_row_bytes;
+    uint8_t* dst;              // expanded rows
+    int64_t dst_row_bytes;
+    int32_t* colsum;           // weights: [rows][2] code sums of fp16 groups (else unused)
+    int64_t rows;              // output rows (conv activations: output pixels)
+    int32_t is_weight;
+    int32_t bits[2], kind[2], src_off[2], dst_off[2], blk_src[2], blk_dst[2], center[2];
+    // implicit-GEMM convolution (activations): block kb of group g is tap kb / cpt[g],
+    // channel block kb % cpt[g] of the input pixel that tap reads
+    int32_t conv, H, W, P, Q, R, S, sh, sw, ph, pw;
+    int32_t cpt[2];
+};
+
+// n-bit two's-complement patterns in the bytes of x -> E4M3 sign-magnitude bytes.
+template <int N>
+__device__ __forceinline__ uint32_t twos_to_e4m3(uint32_t x) {
+    const uint32_t neg = ((x >> (N - 1)) & 0x01010101u) * 0xFFu;   // 0xFF in negative bytes
+    const uint32_t mag = ((1u << N) * 0x01010101u) - x;           // 2^N - x per byte, no borrow (x < 2^N)
+    return (x & ~neg) | ((mag | 0x80808080u) & neg);
+}
+
+template <int N>
+__device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int g, int lane) {
+    const int kind = p.kind[g];
+    uint8_t* drow = p.dst + r * p.dst_row_bytes + p.dst_off[g];
+    int64_t img = 0;
+    int hp = 0, wq = 0;
+    if (p.conv) {
+        const int64_t pq = (int64_t)p.P * p.Q;
+        img = r / pq;
+        const int rem = (int)(r - img * pq);
+        const int pp = rem / p.Q, qq = rem - pp * p.Q;
+        hp = pp * p.sh - p.ph;
+        wq = qq * p.sw - p.pw;
+    }
+    const uint32_t flip = 0x01010101u << (N - 1);
+    const __half2 bias = __half2half2(__ushort_as_half(
+        (unsigned short)(0x6400u + (p.is_weight ? (1u << (N - 1)) : (uint32_t)p.center[g]))));
+    int32_t csum = 0;
+    for (int kb = lane; kb < p.blk_dst[g]; kb += 32) {
+        const uint8_t* src = nullptr;
+        if (!p.conv) {
+            if (kb < p.blk_src[g]) src = p.src + r * p.src_row_bytes + p.src_off[g] + kb * 4 * N;
+        } else {
+            const int tap = kb / p.cpt[g];
+            const int cb = kb - tap * p.cpt[g];
+            if (tap < p.R * p.S) {
+                const int rr = tap / p.S, ss = tap - rr * p.S;
+                const int h = hp + rr, w = wq + ss;
+                if (h >= 0 && h < p.H && w >= 0 && w < p.W)
+                    src = p.src + ((img * p.H + h) * p.W + w) * p.src_row_bytes + p.src_off[g] + cb * 4 * N;
+            }
+        }
+        uint32_t words[N];
+#pragma unroll
+        for (int i = 0; i < N; ++i) words[i] = src ? __ldg(reinterpret_cast<const uint32_t*>(src) + i) : 0u;
+        uint32_t o[8];
+        block_to_bytes<N>(words, o);
+        if (kind == 0) {
+            if (p.is_weight) {
+#pragma unroll
+                for (int t = 0; t < 8; ++t) o[t] = twos_to_e4m3<N>(o[t]);
+            }
+            uint4* d = reinterpret_cast<uint4*>(drow + kb * 32);
+            d[0] = make_uint4(o[0], o[1], o[2], o[3]);
+            d[1] = make_uint4(o[4], o[5], o[6], o[7]);
+        } else {
+            uint32_t h[16];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                // weights: offset binary j + 2^(n-1); activations: the code u
+                const uint32_t x = p.is_weight ? (o[t] ^ flip) : o[t];
+                if (p.is_weight) csum += (int32_t)__dp4a(x, 0x01010101u, 0u);
+                uint32_t lo, hi;
+                bytes_to_magic_half2(x, lo, hi);
+                h[2 * t] = half2_sub(lo, bias);
+                h[2 * t + 1] = half2_sub(hi, bias);
+            }
+            uint4* d = reinterpret_cast<uint4*>(drow + kb * 64);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) d[q] = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+        }
+    }
+    if (p.is_weight && kind == 1) {
+        // sum of j over the row's group: the offset-binary sum minus 2^(n-1) per code
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) csum += __shfl_xor_sync(0xffffffffu, csum, o);
+        if (lane == 0) p.colsum[r * 2 + g] = csum - (1 << (N - 1)) * 32 * p.blk_dst[g];
+    }
+}
+
+__global__ void __launch_bounds__(256) expand_kernel(const ExpandParams p) {
+    const int lane = threadIdx.x & 31;
+    const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    for (int64_t item = warp_id; item < p.rows * 2; item += nwarps) {
+        const int64_t r = item >> 1;
+        const int g = (int)(item & 1);
+        if (p.blk_dst[g] == 0) continue;
+        switch (p.bits[g]) {
+            case 1: expand_row<1>(p, r, g, lane); break;
+            case 2: expand_row<2>(p, r, g, lane); break;
+            case 3: expand_row<3>(p, r, g, lane); break;
+            case 4: expand_row<4>(p, r, g, lane); break;
+            case 5: expand_row<5>(p, r, g, lane); break;
+            case 6: expand_row<6>(p, r, g, lane); break;
+            case 7: expand_row<7>(p, r, g, lane); break;
+            default: expand_row<8>(p, r, g, lane); break;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// The persistent GEMM over expanded operands
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void store_out16(const SParams& p, int64_t m, int nb, const float (&y)[16]) {
+    const bool vec = nb + 16 <= p.N && (p.N & 7) == 0;
+    if (p.out_bf16) {
+        __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.Y) + m * p.N;
+        if (vec) {
+#pragma unroll
+            for (int v8 = 0; v8 < 2; ++v8) {
+                uint32_t wv[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    __nv_bfloat162 h2 = __floats2bfloat162_rn(y[v8 * 8 + 2 * e], y[v8 * 8 + 2 * e + 1]);
+                    wv[e] = *reinterpret_cast<uint32_t*>(&h2);
+                }
+                *reinterpret_cast<uint4*>(dst + nb + v8 * 8) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+            }
+        } else {
+            for (int j = 0; j < 16; ++j)
+                if (nb + j < p.N) dst[nb + j] = __float2bfloat16_rn(y[j]);
+        }
+    } else {
+        __half* dst = reinterpret_cast<__half*>(p.Y) + m * p.N;
+        if (vec) {
+#pragma unroll
+            for (int v8 = 0; v8 < 2; ++v8) {
+                uint32_t wv[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    __half2 h2 = __floats2half2_rn(y[v8 * 8 + 2 * e], y[v8 * 8 + 2 * e + 1]);
+                    wv[e] = *reinterpret_cast<uint32_t*>(&h2);
+                }
+                *reinterpret_cast<uint4*>(dst + nb + v8 * 8) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+            }
+        } else {
+            for (int j = 0; j < 16; ++j)
+                if (nb + j < p.N) dst[nb + j] = __float2half_rn(y[j]);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid_constant__ SParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t sbase = smem_u32(smem);
+    const uint32_t bar0 = smem_u32(smem + SMEM_BAR);
+    auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + SMEM_MISC);
+    const uint32_t abort_flag = smem_u32(smem + SMEM_MISC + 4);
+    const uint32_t no_abort = smem_u32(smem + SMEM_MISC + 8);   // stays 0: waits that must run to completion
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < STAGES; ++i) {
+            mbar_init(bar(BAR_FULL + i), 1);
+            mbar_init(bar(BAR_EMPTY + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(BAR_ACC_FULL + i), 1);
+            mbar_init(bar(BAR_ACC_EMPTY + i), NUM_EPI_WARPS);
+            mbar_init(bar(BAR_SEG_FULL + i), 1);
+            mbar_init(bar(BAR_SEG_FREE + i), NUM_EPI_WARPS);
+        }
+        mbar_init(bar(BAR_TEARDOWN), 1);
+        set_flag(abort_flag, 0);
+        set_flag(no_abort, 0);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == WARP_MMA) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                     "r"(512)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == WARP_TMA) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            uint32_t s = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
+                const int m0 = (t % p.m_tiles) * BM, n0 = (t / p.m_tiles) * BN;
+#pragma unroll 1
+                for (int g = 0; g < 2 && ok; ++g) {
+                    const int ns = p.g[g].stages, x0 = p.g[g].x0;
+#pragma unroll 1
+                    for (int i = 0; i < ns; ++i, ++s) {
+                        const uint32_t slot = s % STAGES, ph = (s / STAGES) & 1u;
+                        if (!wait_bounded(bar(BAR_EMPTY + slot), ph ^ 1u, abort_flag, kTimeoutNs, p.err, kErrWait)) {
+                            ok = false;
+                            break;
+                        }
+                        if (p.drop_first && s == 0) continue;   // the MMA's wait for it runs out
+                        const uint32_t dst = sbase + slot * STAGE_BYTES;
+                        mbar_arrive_expect_tx(bar(BAR_FULL + slot), STAGE_BYTES);
+                        tma_load_2d(dst, &p.tma_a, x0 + i * 128, m0, bar(BAR_FULL + slot));
+                        tma_load_2d(dst + A_BYTES, &p.tma_b, x0 + i * 128, n0, bar(BAR_FULL + slot));
+                    }
+                }
+            }
+            // loads still in flight must land before the CTA's shared memory is released
+            for (uint32_t q = s > (uint32_t)STAGES ? s - STAGES : 0u; q < s; ++q)
+                if (!(p.drop_first && q == 0))
+                    wait_bounded(bar(BAR_FULL + q % STAGES), (q / STAGES) & 1u, no_abort, kTimeoutNs, p.err, kErrWait);
+        }
+    } else if (warp == WARP_MMA) {
+        // ------------------------------------------------------------------ MMA
+        if (lane == 0) {
+            uint32_t s = 0, segq[2] = {0u, 0u};
+            bool ok = true;
+            int tcount = 0;
+            for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x, ++tcount) {
+                const int b = tcount & 1;
+                const uint32_t use = (uint32_t)(tcount >> 1);
+                if (!wait_bounded(bar(BAR_ACC_EMPTY + b), (use & 1u) ^ 1u, abort_flag, kTimeoutNs, p.err, kErrWait))
+                    break;
+                tc_fence_after();
+#pragma unroll 1
+                for (int g = 0; g < 2 && ok; ++g) {
+                    const int ns = p.g[g].stages;
+                    if (ns == 0) continue;
+                    const bool f8 = p.g[g].kind == 0;
+                    const bool segd = g == p.seg_group;
+                    const int seg_st = p.g[g].seg_stages;
+                    const uint32_t d = tmem_base + (uint32_t)((b * 2 + g) * BN);
+                    int in_seg = 0;
+#pragma unroll 1
+                    for (int i = 0; i < ns; ++i, ++s) {
+                        const bool first = segd ? in_seg == 0 : i == 0;
+                        if (segd && first && i > 0) {
+                            // the previous segment of this group must be drained before it is overwritten
+                            if (!wait_bounded(bar(BAR_SEG_FREE + b), segq[b] & 1u, abort_flag, kTimeoutNs, p.err,
+                                              kErrWait)) {
+                                ok = false;
+                                break;
+                            }
+                            ++segq[b];
+                            tc_fence_after();
+                        }
+                        const uint32_t slot = s % STAGES, ph = (s / STAGES) & 1u;
+                        if (!wait_bounded(bar(BAR_FULL + slot), ph, abort_flag, kTimeoutNs, p.err, kErrWait)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a_addr = sbase + slot * STAGE_BYTES, b_addr = a_addr + A_BYTES;
+                        if (f8) {
+#pragma unroll
+                            for (int k = 0; k < 4; ++k)
+                                mma_f8<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
+                                              (first && k == 0) ? 0u : 1u);
+                        } else {
+#pragma unroll
+                            for (int k = 0; k < 4; ++k)
+                                mma_f16<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
+                                               (first && k == 0) ? 0u : 1u);
+                        }
+                        mma_commit(bar(BAR_EMPTY + slot));
+                        if (segd) {
+                            if (++in_seg == seg_st || i == ns - 1) {
+                                mma_commit(bar(BAR_SEG_FULL + b));
+                                in_seg = 0;
+                            }
+                        }
+                    }
+                    // the drain of this tile's last segment completes a phase nobody here waits for
+                    if (segd) ++segq[b];
+                }
+                if (ok) mma_commit(bar(BAR_ACC_FULL + b));
+            }
+            // every issued MMA completes before TMEM and shared memory are released
+            mma_commit(bar(BAR_TEARDOWN));
+            wait_bounded(bar(BAR_TEARDOWN), 0u, no_abort, kTimeoutNs, p.err, kErrWait);
+        }
+    } else {
+        // ------------------------------------------------------------- epilogue
+        const int ew = warp - WARP_EPI;
+        const int quad = warp & 3;              // TMEM lane quadrant this warp may read
+        const int half = ew >> 2;               // columns [64 * half, 64 * half + 64) of the tile
+        const int row = quad * 32 + lane;
+        const uint32_t lane_base = tmem_base + ((uint32_t)(quad * 32) << 16);
+        const int gs = p.seg_group;
+        uint32_t segf[2] = {0u, 0u};
+        int tcount = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x, ++tcount) {
+            const int b = tcount & 1;
+            const uint32_t use = (uint32_t)(tcount >> 1);
+            const int64_t m0 = (int64_t)(t % p.m_tiles) * BM;
+            const int n0 = (t / p.m_tiles) * BN;
+            int32_t sacc[64];
+#pragma unroll
+            for (int j = 0; j < 64; ++j) sacc[j] = 0;
+            if (gs >= 0) {
+                const int nseg = gs == 0 ? p.g[0].n_seg : p.g[1].n_seg;
+                const uint32_t col = (uint32_t)((b * 2 + gs) * BN + half * 64);
+                for (int j = 0; j < nseg; ++j) {
+                    if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_SEG_FULL + b), segf[b] & 1u, abort_flag,
+                                                              kTimeoutNs, p.err, kErrWait))) {
+                        ok = false;
+                        break;
+                    }
+                    ++segf[b];
+                    tc_fence_after();
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc) {
+                        uint32_t v[16];
+                        tmem_ld16(lane_base + col + cc * 16, v);
+#pragma unroll
+                        for (int q = 0; q < 16; ++q) sacc[cc * 16 + q] += __float2int_rn(__uint_as_float(v[q]));
+                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar(BAR_SEG_FREE + b));
+                }
+                if (!ok) break;
+            }
+            if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_ACC_FULL + b), use & 1u, abort_flag, kTimeoutNs, p.err,
+                                                      kErrWait)))
+                break;
+            tc_fence_after();
+            const int64_t m = m0 + row;
+            float sa[2];
+#pragma unroll
+            for (int g = 0; g < 2; ++g)
+                sa[g] = m < p.M ? (p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g)) : 0.0f;
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc) {
+                const int nb = n0 + half * 64 + cc * 16;
+                uint32_t v[2][16];
+                tmem_ld16x2(lane_base + (uint32_t)((b * 2 + 0) * BN + half * 64 + cc * 16),
+                            lane_base + (uint32_t)((b * 2 + 1) * BN + half * 64 + cc * 16), v[0], v[1]);
+                int32_t acc[2][16];
+#pragma unroll
+                for (int g = 0; g < 2; ++g) {
+                    const SGroup& G = p.g[g];
+                    if (G.stages == 0) {
+#pragma unroll
+                        for (int q = 0; q < 16; ++q) acc[g][q] = 0;
+                        continue;
+                    }
+                    if (g == gs) {
+#pragma unroll
+                        for (int q = 0; q < 16; ++q) acc[g][q] = sacc[cc * 16 + q];
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 16; ++q)
+                            acc[g][q] = __float2int_rn(__uint_as_float(v[g][q]) * G.acc_scale);
+                    }
+                    if (G.center) {
+#pragma unroll
+                        for (int q = 0; q < 16; ++q) {
+                            const int n = nb + q;
+                            acc[g][q] += n < p.N ? G.center * __ldg(p.colsum + (int64_t)n * 2 + g) : 0;
+                        }
+                    }
+                }
+                if (m < p.M) {
+                    if (p.acc_dbg != nullptr) {
+#pragma unroll
+                        for (int g = 0; g < 2; ++g) {
+                            int32_t* dst = p.acc_dbg + ((int64_t)g * p.M + m) * p.N;
+#pragma unroll
+                            for (int q = 0; q < 16; ++q)
+                                if (nb + q < p.N) dst[nb + q] = acc[g][q];
+                        }
+                    }
+                    float y[16];
+#pragma unroll
+                    for (int q = 0; q < 16; ++q) {
+                        const int n = nb + q < p.N ? nb + q : p.N - 1;
+                        const float sw0 = __ldg(p.s_w + (int64_t)n * 2) * p.g[0].inv_levels;
+                        const float sw1 = __ldg(p.s_w + (int64_t)n * 2 + 1) * p.g[1].inv_levels;
+                        y[q] = fmaf(sa[1] * sw1, (float)acc[1][q], sa[0] * sw0 * (float)acc[0][q]);
+                    }
+                    store_out16(p, m, nb, y);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(BAR_ACC_EMPTY + b));
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == WARP_MMA) {
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+// 2-D map over expanded rows [rows][row_bytes] with a box of one 128-byte
+// K-stage by 128 rows, 128-byte swizzle (the layout the MMA descriptors read).
+bool encode_rows(EncodeTiledFn enc, CUtensorMap* map, const uint8_t* base, int64_t row_bytes, int64_t rows) {
+    cuuint64_t dims[2] = {(cuuint64_t)row_bytes, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
+    cuuint32_t box[2] = {128u, 128u};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int64_t align1k(int64_t x) { return (x + 1023) / 1024 * 1024; }
+
+}  // namespace staged
+
+bool staged_plan(const LayoutGeom& geo, StagedPlan* sp) {
+    int nseg_groups = 0;
+    int64_t x0 = 0;
+    sp->seg_group = -1;
+    for (int g = 0; g < 2; ++g) {
+        const GroupGeom& G = geo.g[g];
+        StagedGroup& S = sp->g[g];
+        S.kind = (G.bits_a <= 4 && G.bits_w <= 4) ? 0 : 1;
+        const int64_t bytes = (int64_t)G.pw * (S.kind == 0 ? 1 : 2);
+        S.stages = (int32_t)(bytes / 128);
+        S.x0 = (int32_t)x0;
+        x0 += bytes;
+        const int64_t maxprod = S.kind == 0 ? (int64_t)((1 << G.bits_a) - 1) * (1 << (G.bits_w - 1))
+                                            : (int64_t)(1 << (G.bits_a - 1)) * (1 << (G.bits_w - 1));
+        const int64_t codes_per_stage = S.kind == 0 ? 128 : 64;
+        const int64_t seg_stages = ((int64_t)1 << 24) / maxprod / codes_per_stage;
+        if (seg_stages < 1) return false;
+        S.seg_stages = (int32_t)(seg_stages < S.stages ? seg_stages : (S.stages > 0 ? S.stages : 1));
+        S.n_seg = S.stages > 0 ? (S.stages + S.seg_stages - 1) / S.seg_stages : 0;
+        S.center = S.kind == 1 ? (1 << (G.bits_a - 1)) : 0;
+        if (S.n_seg > 1) {
+            ++nseg_groups;
+            sp->seg_group = g;
+        }
+    }
+    if (nseg_groups > 1) return false;
+    sp->eb = x0;
+    return x0 > 0 && x0 % 128 == 0;
+}
+
+int64_t staged_scratch_bytes(const LayoutGeom& geo, int64_t rows_a, int64_t N) {
+    StagedPlan sp;
+    if (!staged_plan(geo, &sp)) return 0;
+    return staged::align1k(rows_a * sp.eb) + staged::align1k(N * sp.eb) + staged::align1k(N * 8);
+}
+
+cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch, size_t scratch_bytes,
+                          cudaStream_t st) {
+    using namespace staged;
+    StagedPlan sp;
+    if (!staged_plan(geo, &sp)) return cudaErrorNotSupported;
+    const int64_t rows_a = a.M;
+    if ((int64_t)scratch_bytes < staged_scratch_bytes(geo, rows_a, a.N) || scratch == nullptr ||
+        (uintptr_t)scratch % 256 != 0)
+        return cudaErrorNotSupported;
+    uint8_t* xa = static_cast<uint8_t*>(scratch);
+    uint8_t* xw = xa + align1k(rows_a * sp.eb);
+    int32_t* colsum = reinterpret_cast<int32_t*>(xw + align1k((int64_t)a.N * sp.eb));
+    const int taps = a.conv ? a.R * a.S : 1;
+
+    // ---- expand activations (im2col for a convolution) and weights ----
+    ExpandParams e;
+    memset(&e, 0, sizeof(e));
+    for (int g = 0; g < 2; ++g) {
+        const GroupGeom& G = geo.g[g];
+        e.bits[g] = G.bits_a;
+        e.kind[g] = sp.g[g].kind;
+        e.src_off[g] = G.a_off;
+        e.dst_off[g] = sp.g[g].x0;
+        e.blk_src[g] = G.pa / 32;
+        e.blk_dst[g] = G.pw / 32;
+        e.center[g] = sp.g[g].center;
+        e.cpt[g] = G.pa / 32 > 0 ? G.pa / 32 : 1;
+    }
+    e.src = a.Ap;
+    e.src_row_bytes = geo.a_row_bytes;
+    e.dst = xa;
+    e.dst_row_bytes = sp.eb;
+    e.rows = rows_a;
+    e.is_weight = 0;
+    e.conv = a.conv;
+    e.H = a.H; e.W = a.W; e.P = a.P; e.Q = a.Q; e.R = a.R; e.S = a.S;
+    e.sh = a.sh; e.sw = a.sw; e.ph = a.ph; e.pw = a.pw;
+    (void)taps;
+    auto grid_for = [](int64_t items) {
+        int64_t ctas = (items + 7) / 8;                        // 8 warps per CTA, one (row, group) per warp
+        const int64_t cap = (int64_t)num_sms() * 16;
+        return (int)(ctas < 1 ? 1 : (ctas > cap ? cap : ctas));
+    };
+    expand_kernel<<<grid_for(rows_a * 2), 256, 0, st>>>(e);
+    note_launch();
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+
+    ExpandParams w = e;
+    for (int g = 0; g < 2; ++g) {
+        const GroupGeom& G = geo.g[g];
+        w.bits[g] = G.bits_w;
+        w.src_off[g] = G.w_off;
+        w.blk_src[g] = G.pw / 32;
+        w.center[g] = 0;
+    }
+    w.src = a.Wp;
+    w.src_row_bytes = geo.w_row_bytes;
+    w.dst = xw;
+    w.rows = a.N;
+    w.is_weight = 1;
+    w.colsum = colsum;
+    w.conv = 0;
+    expand_kernel<<<grid_for((int64_t)a.N * 2), 256, 0, st>>>(w);
+    note_launch();
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+
+    // ---- the GEMM ----
+    SParams p;
+    memset(&p, 0, sizeof(p));
+    EncodeTiledFn enc = encode_fn();
+    if (enc == nullptr) return cudaErrorNotSupported;
+    if (!encode_rows(enc, &p.tma_a, xa, sp.eb, rows_a) || !encode_rows(enc, &p.tma_b, xw, sp.eb, a.N))
+        return cudaErrorInvalidValue;
+    p.s_a = a.s_a;
+    p.s_w = a.s_w;
+    p.colsum = colsum;
+    p.Y = a.Y;
+    p.acc_dbg = a.acc_dbg;
+    p.err = device_error_word();
+    if (p.err == nullptr) return cudaErrorUnknown;
+    p.M = a.M;
+    p.N = a.N;
+    p.m_tiles = (int32_t)((a.M + BM - 1) / BM);
+    p.n_tiles = (a.N + BN - 1) / BN;
+    p.total_tiles = p.m_tiles * p.n_tiles;
+    p.s_a_per_row = a.s_a_per_row;
+    p.out_bf16 = a.out_bf16;
+    p.seg_group = sp.seg_group;
+    p.drop_first = (a.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) != 0 ? 1 : 0;
+    for (int g = 0; g < 2; ++g) {
+        const GroupGeom& G = geo.g[g];
+        SGroup& S = p.g[g];
+        S.kind = sp.g[g].kind;
+        S.stages = sp.g[g].stages;
+        S.x0 = sp.g[g].x0;
+        S.seg_stages = sp.g[g].seg_stages;
+        S.n_seg = sp.g[g].n_seg;
+        S.center = sp.g[g].center;
+        S.acc_scale = S.kind == 0 ? 262144.0f : 1.0f;   // 2^18
+        S.inv_levels = (float)(1.0 / ((double)((1 << G.bits_a) - 1) * (double)(1 << (G.bits_w - 1))));
+    }
+    static bool attr_done[64] = {};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        if ((err = cudaFuncSetAttribute(staged_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
+            cudaSuccess)
+            return err;
+        attr_done[dev] = true;
+    }
+    if ((err = prefer_max_shared((const void*)staged_mma_kernel)) != cudaSuccess) return err;
+    const int grid = p.total_tiles < num_sms() ? p.total_tiles : num_sms();
+    staged_mma_kernel<<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
+    note_launch();
+    return cudaGetLastError();
+}
+
+}  // namespace soniq

@@ -22,8 +22,8 @@ STATUS_NAMES = {0: "SONIQ_OK", 1: "SONIQ_ERR_INVALID_ARG", 2: "SONIQ_ERR_UNSUPPO
                 3: "SONIQ_ERR_ALIGNMENT", 4: "SONIQ_ERR_CUDA", 5: "SONIQ_ERR_TIMEOUT"}
 SCALE_PER_TENSOR, SCALE_PER_ROW, SCALE_CALIBRATED = 0, 1, 2
 OUT_F16, OUT_BF16 = 0, 1
-FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_TEST_DROP_ARRIVE = 1, 2, 0x100
-PATH_NAMES = {0: "CUDA-core GEMV", 1: "tensor-core kernel"}
+FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_FORCE_FUSED, FLAG_TEST_DROP_ARRIVE = 1, 2, 4, 0x100
+PATH_NAMES = {0: "CUDA-core GEMV", 1: "tensor-core fused kernel", 2: "tensor-core staged (expand + GEMM)"}
 
 EXPORTED = ["soniq_abi_version", "soniq_status_string", "soniq_group_codes",
             "soniq_packed_row_bytes", "soniq_validate_layout", "soniq_launch_count",
@@ -121,19 +121,21 @@ def _need(t: torch.Tensor, dtype, name: str):
         raise ValueError(f"{name} must be a contiguous CUDA {dtype} tensor")
 
 
-# Scratch buffers the binding hands to the library, one per (device, stream):
-# calls on one stream run in order, so they may share it; calls on different
-# streams get different buffers.  Each is zero-filled when created (the
-# quantize barrier must start at zero) and grows by reallocation when a call
+# Scratch buffers the binding hands to the library, one per (use, device,
+# stream): calls on one stream run in order, so they may share it; calls on
+# different streams get different buffers.  The quantize scratch (whose
+# barrier must start at zero and which every completed call leaves zeroed) is
+# never shared with the GEMM scratch (which the staged path overwrites).
+# Each is zero-filled when created and grows by reallocation when a call
 # needs more.
 _scratch = {}
 
 
-def _get_scratch(nbytes: int, device, stream) -> Optional[torch.Tensor]:
+def _get_scratch(nbytes: int, device, stream, use: str) -> Optional[torch.Tensor]:
     if nbytes <= 0:
         return None
     s = torch.cuda.current_stream(device) if stream is None else stream
-    key = (torch.device(device).index, s.cuda_stream)
+    key = (use, torch.device(device).index, s.cuda_stream)
     buf = _scratch.get(key)
     if buf is None or buf.numel() < nbytes:
         with torch.cuda.stream(s):
@@ -143,9 +145,10 @@ def _get_scratch(nbytes: int, device, stream) -> Optional[torch.Tensor]:
 
 
 def reset_scratch():
-    """Zero every cached scratch buffer (needed after a SONIQ_ERR_TIMEOUT)."""
-    for buf in _scratch.values():
-        buf.zero_()
+    """Zero every cached quantize scratch buffer (needed after a SONIQ_ERR_TIMEOUT)."""
+    for key, buf in _scratch.items():
+        if key[0] == "quantize":
+            buf.zero_()
 
 
 class Layout:
@@ -222,7 +225,7 @@ def quantize_act(layout: Layout, A: torch.Tensor, scale_mode: str = "tensor",
         Ap = torch.empty((M, layout.row_bytes(False)), dtype=torch.uint8, device=A.device)
     if scratch is False:
         need = int(lib().soniq_quantize_act_scratch_bytes(ctypes.byref(layout.c), M, mode))
-        scratch = _get_scratch(need, A.device, stream)
+        scratch = _get_scratch(need, A.device, stream, "quantize")
     nbytes = 0 if scratch is None else scratch.numel() * scratch.element_size()
     _check(lib().soniq_quantize_act(ctypes.byref(layout.c), _ptr(A), M, mode, _ptr(s_a), _ptr(Ap),
                                     _ptr(scratch), nbytes, _stream(stream)), "soniq_quantize_act")
@@ -254,7 +257,7 @@ def mp_gemm(layout: Layout, Ap: torch.Tensor, s_a: torch.Tensor, Wp: torch.Tenso
         Y = torch.empty((M, N), dtype=out_dtype, device=Ap.device)
     od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
     need = int(lib().soniq_mp_gemm_scratch_bytes(ctypes.byref(layout.c), M, N, int(flags)))
-    scratch = _get_scratch(need, Ap.device, stream)
+    scratch = _get_scratch(need, Ap.device, stream, "gemm")
     _check(lib().soniq_mp_gemm(ctypes.byref(layout.c), _ptr(Ap), _ptr(s_a), _SCALE[scale_mode], M,
                                _ptr(Wp), _ptr(s_w), N, _ptr(Y), od, _ptr(acc_dbg), int(flags),
                                _ptr(scratch), max(need, 0), _stream(stream)), "soniq_mp_gemm")
@@ -290,7 +293,7 @@ def mp_conv2d(layout: Layout, cd: CConvDesc, Xp: torch.Tensor, s_a: torch.Tensor
         Y = torch.empty((cd.batch, P, Q, cd.C_out), dtype=out_dtype, device=Xp.device)
     od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
     need = int(lib().soniq_mp_conv2d_scratch_bytes(ctypes.byref(layout.c), ctypes.byref(cd), int(flags)))
-    scratch = _get_scratch(need, Xp.device, stream)
+    scratch = _get_scratch(need, Xp.device, stream, "gemm")
     _check(lib().soniq_mp_conv2d(ctypes.byref(layout.c), ctypes.byref(cd), _ptr(Xp), _ptr(s_a),
                                  _SCALE[scale_mode], _ptr(Wp), _ptr(s_w), _ptr(Y), od,
                                  _ptr(acc_dbg), int(flags), _ptr(scratch), max(need, 0),

@@ -67,20 +67,25 @@ def _max_codes(M, N, K, na, nw):
     return U, J
 
 
+PATHS = pytest.mark.parametrize("flags", [2, 2 | 4], ids=["staged", "fused"])
+
+
+@PATHS
 @pytest.mark.parametrize("na,nw", [(4, 4), (3, 4), (4, 3), (2, 4)])
 @pytest.mark.parametrize("K", [65536, 65536 - 128 + 37])
-def test_e4m3_group_all_extreme_products(sq, na, nw, K):
+def test_e4m3_group_all_extreme_products(sq, na, nw, K, flags):
     M, N = 130, 136                        # two row tiles and two column tiles, both ragged
     U, J = _max_codes(M, N, K, na, nw)
     U[5, : K // 3] = 0                     # a row whose sum stops growing early
-    g_acc, g_y, r_acc, y16, terms = _run_codes(sq, U, J, [K, 0], [na, 1], [nw, 1], flags=2)
+    g_acc, g_y, r_acc, y16, terms = _run_codes(sq, U, J, [K, 0], [na, 1], [nw, 1], flags=flags)
     assert np.abs(r_acc).max() == K * ((1 << na) - 1) * (1 << (nw - 1))
     assert np.array_equal(g_acc, r_acc)
     assert_y_close(g_y, y16, terms, f"extreme E4M3 na={na} nw={nw} K={K}")
 
 
+@PATHS
 @pytest.mark.parametrize("K", [65536, 40000])
-def test_e4m3_partial_sums_cross_2_20_to_2_24_mid_chunk(sq, K):
+def test_e4m3_partial_sums_cross_2_20_to_2_24_mid_chunk(sq, K, flags):
     """Random codes from the top of the range: partial sums grow by about 100
     per code and carry random low bits, crossing 2^20, 2^21, ..., 2^24 at
     arbitrary points inside 128-code chunks."""
@@ -90,7 +95,7 @@ def test_e4m3_partial_sums_cross_2_20_to_2_24_mid_chunk(sq, K):
     J = np.empty((N, K), np.int8)
     J[: N // 2] = rng.integers(4, 8, size=(N // 2, K), dtype=np.int8)      # positive sums
     J[N // 2:] = rng.integers(-8, -5, size=(N - N // 2, K), dtype=np.int8)  # negative sums
-    g_acc, g_y, r_acc, y16, terms = _run_codes(sq, U, J, [K, 0], [4, 1], [4, 1], flags=2)
+    g_acc, g_y, r_acc, y16, terms = _run_codes(sq, U, J, [K, 0], [4, 1], [4, 1], flags=flags)
     big = np.abs(r_acc[0])
     if K == 65536:
         assert big.max() > 2 ** 22
@@ -98,7 +103,8 @@ def test_e4m3_partial_sums_cross_2_20_to_2_24_mid_chunk(sq, K):
     assert_y_close(g_y, y16, terms, f"E4M3 crossing K={K}")
 
 
-def test_e4m3_and_fp16_groups_both_extreme(sq):
+@PATHS
+def test_e4m3_and_fp16_groups_both_extreme(sq, flags):
     """A 4-bit group and an 8-bit group side by side, both at their extremes
     over a long K: the 8-bit group needs exact segments, the 4-bit one runs
     unsegmented on the E4M3 pipe."""
@@ -113,7 +119,7 @@ def test_e4m3_and_fp16_groups_both_extreme(sq):
     J[1::2, :K0] = -8
     J[0::2, K0:] = -128
     J[1::2, K0:] = 127
-    g_acc, g_y, r_acc, y16, terms = _run_codes(sq, U, J, [K0, K1], [4, 8], [4, 8], flags=2)
+    g_acc, g_y, r_acc, y16, terms = _run_codes(sq, U, J, [K0, K1], [4, 8], [4, 8], flags=flags)
     assert np.abs(r_acc[1]).max() > 2 ** 24
     assert np.array_equal(g_acc, r_acc)
     assert_y_close(g_y, y16, terms, "E4M3 + fp16 extremes")

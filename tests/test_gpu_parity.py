@@ -172,12 +172,25 @@ def test_pack_weights_bytes(sq, taps, mode, bits):
 GEMM_BITS = [(1, 4), (1, 8), (2, 6), (2, 8), (3, 5), (3, 8), (4, 4), (4, 6), (4, 8), (2, 2), (8, 8), (5, 7)]
 
 
+# tensor-core paths: staged (expand into scratch, then GEMM) and fused (expand on chip)
+STAGED, FUSED = 2, 2 | 4
+
+
+@pytest.mark.parametrize("path", [STAGED, FUSED], ids=["staged", "fused"])
 @pytest.mark.parametrize("bits", GEMM_BITS)
-def test_gemm_small_all_bit_pairs(sq, bits):
+def test_gemm_small_all_bit_pairs(sq, bits, path):
     # several 128x128 tiles plus ragged tails in M, N and K
     d = wl.random_linear(100 + bits[0] * 10 + bits[1], M=300, K=333, N=264, bits_lo=bits[0],
                          bits_hi=bits[1], frac_hi=0.3, n_outliers=2)
-    check_linear(sq, d, flags=2, what=f"gemm{bits}")
+    check_linear(sq, d, flags=path, what=f"gemm{bits}")
+
+
+def test_gemm_paths_reported(sq):
+    d = wl.random_linear(5, M=300, K=333, N=264, bits_lo=2, bits_hi=8, frac_hi=0.3)
+    lay = sq.Layout(d["perm"], d["count"], d["bits"])
+    assert sq.gemm_path(lay, 300, 264) == sq.PATH_NAMES[2]
+    assert sq.gemm_path(lay, 300, 264, FUSED) == sq.PATH_NAMES[1]
+    assert sq.gemm_path(lay, 8, 264) == sq.PATH_NAMES[0]
 
 
 @pytest.mark.parametrize("pad", [32, 128])
@@ -221,7 +234,8 @@ def test_gemm_zero_group(sq):
     assert not g["acc"][1].any()
 
 
-def test_gemm_exactness_segments(sq):
+@pytest.mark.parametrize("path", [STAGED, FUSED], ids=["staged", "fused"])
+def test_gemm_exactness_segments(sq, path):
     """Worst-case 8-bit codes over a long K: every partial sum is the extreme
     255 * -128, so a single fp32 accumulator would leave the exact-integer
     range after 514 codes.  The segmented accumulation must stay exact."""
@@ -233,7 +247,7 @@ def test_gemm_exactness_segments(sq):
     W[::3, :] = 0.5                          # j = 127 on some rows
     A[1::2, ::7] = 0                         # some rows with fewer terms
     d = dict(A=A, W=W, perm=perm, count=count, bits=[4, 8])
-    g, r = check_linear(sq, d, flags=2, what="segments")
+    g, r = check_linear(sq, d, flags=path, what="segments")
     assert np.abs(r["acc"]).max() > 2 ** 24
 
 
@@ -297,7 +311,7 @@ def test_gemv_matches_mma(sq):
 # implicit-GEMM convolution
 # ---------------------------------------------------------------------------
 
-def run_conv(sq, spec, pad_unit=32):
+def run_conv(sq, spec, pad_unit=32, flags=0):
     d = wl.make_conv(spec)
     lay = sq.Layout(d["perm"], d["count"], d["bits"], pad_unit=pad_unit)
     X = _dev(d["X"]).reshape(-1, spec.C)
@@ -305,15 +319,15 @@ def run_conv(sq, spec, pad_unit=32):
     Xp, s_a = sq.quantize_act(lay, X)
     cd = sq.conv_desc(spec.batch, spec.H, spec.W, spec.C_out, spec.R, spec.S, spec.stride, spec.pad)
     acc = torch.zeros((2, spec.M, spec.C_out), dtype=torch.int32, device="cuda")
-    Y = sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, acc_dbg=acc)
+    Y = sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, acc_dbg=acc, flags=flags)
     assert sq.sync_status() == 0
     return d, dict(Xp=Xp.cpu().numpy(), s_a=s_a.cpu().numpy(), Wp=Wp.cpu().numpy(),
                    s_w=s_w.cpu().numpy(), acc=acc.cpu().numpy(),
                    Y=Y.float().cpu().numpy().reshape(spec.M, spec.C_out))
 
 
-def check_conv(sq, spec, pad_unit=32, pix=None, what="conv"):
-    d, g = run_conv(sq, spec, pad_unit)
+def check_conv(sq, spec, pad_unit=32, pix=None, what="conv", flags=0):
+    d, g = run_conv(sq, spec, pad_unit, flags)
     r = oracle.conv2d(d["X"], d["W"], d["perm"], d["count"], d["bits"], d["bits"], spec.R, spec.S,
                       stride=spec.stride, pad=spec.pad, pad_unit=pad_unit, pix=pix)
     assert np.array_equal(g["s_a"], r["s_a"]) and np.array_equal(g["s_w"], r["s_w"])
@@ -325,13 +339,14 @@ def check_conv(sq, spec, pad_unit=32, pix=None, what="conv"):
     assert_y_close(g["Y"][sel], r["Y16"], terms, what)
 
 
+@pytest.mark.parametrize("flags", [0, 4], ids=["staged", "fused"])
 @pytest.mark.parametrize("bits", [(4, 8), (1, 4), (2, 6)])
 @pytest.mark.parametrize("geom", [((1, 1), (1, 1)), ((2, 2), (0, 0)), ((1, 2), (1, 0))])
-def test_conv_small(sq, bits, geom):
+def test_conv_small(sq, bits, geom, flags):
     stride, pad = geom
     spec = wl.ConvSpec("t", batch=3, H=9, W=7, C=70, C_out=40, R=3, S=3, stride=stride, pad=pad,
                        bits_lo=bits[0], bits_hi=bits[1], frac_hi=0.3, seed=bits[0] + 7 * stride[0])
-    check_conv(sq, spec, what=f"conv{bits}{geom}")
+    check_conv(sq, spec, what=f"conv{bits}{geom}", flags=flags)
 
 
 def test_conv_1x1_and_5x5_pad128(sq):
@@ -371,10 +386,11 @@ def test_full_linear_64x512x512(sq):
     check_linear(sq, d, what="linear 64x512x512")
 
 
+@pytest.mark.parametrize("flags", [0, 4], ids=["staged", "fused"])
 @pytest.mark.parametrize("spec", [wl.CONV_RESNET, wl.CONV_RESNET_1B4B], ids=lambda s: s.name)
-def test_full_conv_resnet(sq, spec):
+def test_full_conv_resnet(sq, spec, flags):
     pix = _sample_rows(spec.M, 600, 1)
-    check_conv(sq, spec, pix=pix, what=spec.name)
+    check_conv(sq, spec, pix=pix, what=spec.name, flags=flags)
 
 
 def test_full_mlp_up(sq):
@@ -400,27 +416,29 @@ def test_sweep_every_point_full_k(sq, lo, hi, frac):
     check_linear(sq, d, rows=_sample_rows(256, 24, 4), what=f"sweep lo{lo} hi{hi} f{frac}")
 
 
+@pytest.mark.parametrize("flags", [0, FUSED], ids=["default", "fused"])
 @pytest.mark.parametrize("lo,hi,frac", [(1, 8, 1.0), (2, 4, 0.1), (3, 6, 0.5), (4, 8, 0.25)])
-def test_full_sweep_points(sq, lo, hi, frac):
+def test_full_sweep_points(sq, lo, hi, frac, flags):
     spec = wl.LinearSpec("sweep", M=8192, K=4096, N=4096, bits_lo=lo, bits_hi=hi, frac_hi=frac)
     d = wl.make_linear(spec)
-    check_linear(sq, d, rows=_sample_rows(8192, 48, 3), what=f"sweep lo{lo} hi{hi} f{frac}")
+    check_linear(sq, d, rows=_sample_rows(8192, 48, 3), what=f"sweep lo{lo} hi{hi} f{frac}", flags=flags)
 
 
 # ---------------------------------------------------------------------------
 # failure reporting without a GPU fault
 # ---------------------------------------------------------------------------
 
-def test_timeout_is_reported_and_context_survives(sq):
-    d = wl.random_linear(400, M=128, K=256, N=128, bits_lo=2, bits_hi=8, frac_hi=0.25)
+@pytest.mark.parametrize("path", [STAGED, FUSED], ids=["staged", "fused"])
+def test_timeout_is_reported_and_context_survives(sq, path):
+    d = wl.random_linear(400, M=300, K=1000, N=256, bits_lo=2, bits_hi=8, frac_hi=0.25)
     lay = sq.Layout(d["perm"], d["count"], d["bits"])
     Wp, s_w = sq.pack_weights(lay, _dev(d["W"]))
     Ap, s_a = sq.quantize_act(lay, _dev(d["A"]))
     assert sq.sync_status() == 0
-    sq.mp_gemm(lay, Ap, s_a, Wp, s_w, flags=sq.FLAG_FORCE_MMA | sq.FLAG_TEST_DROP_ARRIVE)
+    sq.mp_gemm(lay, Ap, s_a, Wp, s_w, flags=path | sq.FLAG_TEST_DROP_ARRIVE)
     assert sq.sync_status() == 5            # SONIQ_ERR_TIMEOUT, then cleared
     assert sq.sync_status() == 0
-    check_linear(sq, d, flags=2, what="after timeout")
+    check_linear(sq, d, flags=path, what="after timeout")
 
 
 def test_quantize_barrier_timeout_is_reported_and_scratch_recovers(sq):
