@@ -29,14 +29,20 @@
 //     over its K range could exceed that is accumulated in segments that the
 //     epilogue warps drain into int32 registers.
 //
-// The GEMM kernel: persistent CTAs (one per SM) walk 128 x 128 output tiles.
-//   warp 0     TMA producer: per 128-byte K-stage, one A and one B box (16 KB
-//              each, 128-byte swizzle) into a 6-stage ring
-//   warp 1     TMEM owner and MMA issuer (one thread): 4 MMAs per K-stage into
-//              the tile's accumulators; two accumulator sets (2 x 2 groups x
-//              128 columns = all 512 TMEM columns), so one tile's epilogue
-//              overlaps the next tile's mainloop
-//   warps 2-9  epilogue: two warps per TMEM lane quadrant, 64 columns each
+// The GEMM kernel: persistent CTAs (one per SM) walk 128 x 256 output tiles
+// (N = 256 per MMA: with 128-column MMAs the per-instruction cost, not the
+// tensor pipe, set the pace).
+//   warp 0      TMA producer: per 128-byte K-stage, an A box (128 rows, 16 KB)
+//               and a B box (256 rows, 32 KB), 128-byte swizzle, 4-stage ring
+//   warp 1      TMEM owner and MMA issuer (one thread): 4 MMAs per K-stage.
+//               A tile's accumulation is a sequence of jobs (a group, or one
+//               exact segment of a group; the segmented group first), and job
+//               k of the CTA accumulates into TMEM region k % 2 (256 columns
+//               each), so the epilogue drains one region while the MMAs fill
+//               the other, across tile boundaries too
+//   warps 2-17  epilogue: four warps per TMEM lane quadrant, 64 columns each;
+//               earlier jobs of a tile are summed into int32 registers, the
+//               final job completes the outputs
 // Every wait is bounded (2 s); a wait that runs out records an error bit,
 // raises a CTA abort flag and the CTA winds down (copies and MMAs in flight
 // are waited for, TMEM is freed).
@@ -55,18 +61,19 @@ namespace staged {
 using namespace tc;
 
 constexpr int BM = 128;
-constexpr int BN = 128;
-constexpr int STAGES = 6;
+constexpr int BN = 256;
+constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * 128;
 constexpr int B_BYTES = BN * 128;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int NUM_EPI_WARPS = 8;
+constexpr int NUM_EPI_WARPS = 16;
 constexpr int WARP_TMA = 0, WARP_MMA = 1, WARP_EPI = 2;
 constexpr int NUM_THREADS = (2 + NUM_EPI_WARPS) * 32;
-constexpr int BAR_FULL = 0, BAR_EMPTY = STAGES, BAR_ACC_FULL = 2 * STAGES, BAR_ACC_EMPTY = 2 * STAGES + 2,
-              BAR_SEG_FULL = 2 * STAGES + 4, BAR_SEG_FREE = 2 * STAGES + 6, BAR_TEARDOWN = 2 * STAGES + 8,
-              NUM_BARS = 2 * STAGES + 9;
-constexpr int SMEM_BAR = STAGES * STAGE_BYTES;
+constexpr int BAR_FULL = 0, BAR_EMPTY = STAGES, BAR_REG_FULL = 2 * STAGES, BAR_REG_EMPTY = 2 * STAGES + 2,
+              BAR_TEARDOWN = 2 * STAGES + 4, NUM_BARS = 2 * STAGES + 5;
+constexpr int COLS_PER_WARP = 2 * 2 * 64 * 4;           // [s_w | center * C][group][64 columns], 4 bytes each
+constexpr int SMEM_COLS = STAGES * STAGE_BYTES;
+constexpr int SMEM_BAR = SMEM_COLS + NUM_EPI_WARPS * COLS_PER_WARP;
 constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;   // tmem base, abort flag, a zero word
 constexpr int SMEM_TOTAL = SMEM_MISC + 16;
 constexpr int SMEM_ALLOC = SMEM_TOTAL + 1024;        // slack for 1024-byte alignment
@@ -264,6 +271,12 @@ __device__ __forceinline__ void store_out16(const SParams& p, int64_t m, int nb,
     }
 }
 
+// The tile's accumulation jobs, in order: the group that needs exact
+// segments (if any) first, then the other one; each segment is one job.
+// Job k of the CTA accumulates into TMEM region k % 2 (256 columns), so the
+// epilogue drains one region while the MMAs fill the other.
+__device__ __forceinline__ int first_group(const SParams& p) { return p.seg_group == 1 ? 1 : 0; }
+
 __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid_constant__ SParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -274,6 +287,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + SMEM_MISC);
     const uint32_t abort_flag = smem_u32(smem + SMEM_MISC + 4);
     const uint32_t no_abort = smem_u32(smem + SMEM_MISC + 8);   // stays 0: waits that must run to completion
+    const int g_first = first_group(p);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
@@ -281,10 +295,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
             mbar_init(bar(BAR_EMPTY + i), 1);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(bar(BAR_ACC_FULL + i), 1);
-            mbar_init(bar(BAR_ACC_EMPTY + i), NUM_EPI_WARPS);
-            mbar_init(bar(BAR_SEG_FULL + i), 1);
-            mbar_init(bar(BAR_SEG_FREE + i), NUM_EPI_WARPS);
+            mbar_init(bar(BAR_REG_FULL + i), 1);
+            mbar_init(bar(BAR_REG_EMPTY + i), NUM_EPI_WARPS);
         }
         mbar_init(bar(BAR_TEARDOWN), 1);
         set_flag(abort_flag, 0);
@@ -310,7 +322,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
             for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
                 const int m0 = (t % p.m_tiles) * BM, n0 = (t / p.m_tiles) * BN;
 #pragma unroll 1
-                for (int g = 0; g < 2 && ok; ++g) {
+                for (int gi = 0; gi < 2 && ok; ++gi) {
+                    const int g = gi == 0 ? g_first : 1 - g_first;
                     const int ns = p.g[g].stages, x0 = p.g[g].x0;
 #pragma unroll 1
                     for (int i = 0; i < ns; ++i, ++s) {
@@ -335,67 +348,51 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     } else if (warp == WARP_MMA) {
         // ------------------------------------------------------------------ MMA
         if (lane == 0) {
-            uint32_t s = 0, segq[2] = {0u, 0u};
+            uint32_t s = 0, job = 0;
             bool ok = true;
-            int tcount = 0;
-            for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x, ++tcount) {
-                const int b = tcount & 1;
-                const uint32_t use = (uint32_t)(tcount >> 1);
-                if (!wait_bounded(bar(BAR_ACC_EMPTY + b), (use & 1u) ^ 1u, abort_flag, kTimeoutNs, p.err, kErrWait))
-                    break;
-                tc_fence_after();
+            for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
 #pragma unroll 1
-                for (int g = 0; g < 2 && ok; ++g) {
+                for (int gi = 0; gi < 2 && ok; ++gi) {
+                    const int g = gi == 0 ? g_first : 1 - g_first;
                     const int ns = p.g[g].stages;
-                    if (ns == 0) continue;
                     const bool f8 = p.g[g].kind == 0;
-                    const bool segd = g == p.seg_group;
-                    const int seg_st = p.g[g].seg_stages;
-                    const uint32_t d = tmem_base + (uint32_t)((b * 2 + g) * BN);
-                    int in_seg = 0;
+                    const int per_job = g == p.seg_group ? p.g[g].seg_stages : ns;
 #pragma unroll 1
-                    for (int i = 0; i < ns; ++i, ++s) {
-                        const bool first = segd ? in_seg == 0 : i == 0;
-                        if (segd && first && i > 0) {
-                            // the previous segment of this group must be drained before it is overwritten
-                            if (!wait_bounded(bar(BAR_SEG_FREE + b), segq[b] & 1u, abort_flag, kTimeoutNs, p.err,
-                                              kErrWait)) {
-                                ok = false;
-                                break;
-                            }
-                            ++segq[b];
-                            tc_fence_after();
-                        }
-                        const uint32_t slot = s % STAGES, ph = (s / STAGES) & 1u;
-                        if (!wait_bounded(bar(BAR_FULL + slot), ph, abort_flag, kTimeoutNs, p.err, kErrWait)) {
+                    for (int i = 0; i < ns && ok; ++job) {
+                        const uint32_t r = job & 1u, use = job >> 1;
+                        if (!wait_bounded(bar(BAR_REG_EMPTY + r), (use & 1u) ^ 1u, abort_flag, kTimeoutNs, p.err,
+                                          kErrWait)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t a_addr = sbase + slot * STAGE_BYTES, b_addr = a_addr + A_BYTES;
-                        if (f8) {
-#pragma unroll
-                            for (int k = 0; k < 4; ++k)
-                                mma_f8<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
-                                              (first && k == 0) ? 0u : 1u);
-                        } else {
-#pragma unroll
-                            for (int k = 0; k < 4; ++k)
-                                mma_f16<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
-                                               (first && k == 0) ? 0u : 1u);
-                        }
-                        mma_commit(bar(BAR_EMPTY + slot));
-                        if (segd) {
-                            if (++in_seg == seg_st || i == ns - 1) {
-                                mma_commit(bar(BAR_SEG_FULL + b));
-                                in_seg = 0;
+                        const uint32_t d = tmem_base + r * BN;
+                        const int jn = per_job < ns - i ? per_job : ns - i;
+#pragma unroll 1
+                        for (int q = 0; q < jn; ++q, ++i, ++s) {
+                            const uint32_t slot = s % STAGES, ph = (s / STAGES) & 1u;
+                            if (!wait_bounded(bar(BAR_FULL + slot), ph, abort_flag, kTimeoutNs, p.err, kErrWait)) {
+                                ok = false;
+                                break;
                             }
+                            tc_fence_after();
+                            const uint32_t a_addr = sbase + slot * STAGE_BYTES, b_addr = a_addr + A_BYTES;
+                            if (f8) {
+#pragma unroll
+                                for (int k = 0; k < 4; ++k)
+                                    mma_f8<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
+                                                  (q == 0 && k == 0) ? 0u : 1u);
+                            } else {
+#pragma unroll
+                                for (int k = 0; k < 4; ++k)
+                                    mma_f16<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
+                                                   (q == 0 && k == 0) ? 0u : 1u);
+                            }
+                            mma_commit(bar(BAR_EMPTY + slot));
                         }
+                        if (ok) mma_commit(bar(BAR_REG_FULL + r));
                     }
-                    // the drain of this tile's last segment completes a phase nobody here waits for
-                    if (segd) ++segq[b];
                 }
-                if (ok) mma_commit(bar(BAR_ACC_FULL + b));
             }
             // every issued MMA completes before TMEM and shared memory are released
             mma_commit(bar(BAR_TEARDOWN));
@@ -403,111 +400,110 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
         }
     } else {
         // ------------------------------------------------------------- epilogue
+        // Warp w reads TMEM lane quadrant w % 4 (rows 32*(w%4) .. +31 of the
+        // tile) and the 64 columns cgrp*64 .. +63, cgrp = (w - 2) / 4.
         const int ew = warp - WARP_EPI;
-        const int quad = warp & 3;              // TMEM lane quadrant this warp may read
-        const int half = ew >> 2;               // columns [64 * half, 64 * half + 64) of the tile
+        const int quad = warp & 3;
+        const int cgrp = ew >> 2;
         const int row = quad * 32 + lane;
-        const uint32_t lane_base = tmem_base + ((uint32_t)(quad * 32) << 16);
-        const int gs = p.seg_group;
-        uint32_t segf[2] = {0u, 0u};
-        int tcount = 0;
+        const uint32_t lane_base = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(cgrp * 64);
+        // this warp's copy of the tile's column constants: s_w * inv_levels and
+        // center * (weight code sum), [group][64 columns]
+        float* sw_w = reinterpret_cast<float*>(smem + SMEM_COLS + ew * COLS_PER_WARP);
+        int32_t* cs_w = reinterpret_cast<int32_t*>(smem + SMEM_COLS + ew * COLS_PER_WARP + 2 * 64 * 4);
+        uint32_t job = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x, ++tcount) {
-            const int b = tcount & 1;
-            const uint32_t use = (uint32_t)(tcount >> 1);
+        for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
             const int64_t m0 = (int64_t)(t % p.m_tiles) * BM;
-            const int n0 = (t / p.m_tiles) * BN;
-            int32_t sacc[64];
+            const int nc0 = (t / p.m_tiles) * BN + cgrp * 64;    // this warp's first column
+            __syncwarp();
 #pragma unroll
-            for (int j = 0; j < 64; ++j) sacc[j] = 0;
-            if (gs >= 0) {
-                const int nseg = gs == 0 ? p.g[0].n_seg : p.g[1].n_seg;
-                const uint32_t col = (uint32_t)((b * 2 + gs) * BN + half * 64);
-                for (int j = 0; j < nseg; ++j) {
-                    if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_SEG_FULL + b), segf[b] & 1u, abort_flag,
-                                                              kTimeoutNs, p.err, kErrWait))) {
-                        ok = false;
-                        break;
-                    }
-                    ++segf[b];
-                    tc_fence_after();
+            for (int h = 0; h < 2; ++h) {
+                const int c = lane + 32 * h;
+                const int n = nc0 + c < p.N ? nc0 + c : p.N - 1;
 #pragma unroll
-                    for (int cc = 0; cc < 4; ++cc) {
-                        uint32_t v[16];
-                        tmem_ld16(lane_base + col + cc * 16, v);
-#pragma unroll
-                        for (int q = 0; q < 16; ++q) sacc[cc * 16 + q] += __float2int_rn(__uint_as_float(v[q]));
-                    }
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(bar(BAR_SEG_FREE + b));
+                for (int g = 0; g < 2; ++g) {
+                    sw_w[g * 64 + c] = __ldg(p.s_w + (int64_t)n * 2 + g) * p.g[g].inv_levels;
+                    cs_w[g * 64 + c] = p.g[g].center ? p.g[g].center * __ldg(p.colsum + (int64_t)n * 2 + g) : 0;
                 }
-                if (!ok) break;
             }
-            if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_ACC_FULL + b), use & 1u, abort_flag, kTimeoutNs, p.err,
-                                                      kErrWait)))
-                break;
-            tc_fence_after();
+            __syncwarp();
             const int64_t m = m0 + row;
             float sa[2];
 #pragma unroll
             for (int g = 0; g < 2; ++g)
                 sa[g] = m < p.M ? (p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g)) : 0.0f;
+            // part: the exact accumulator of the first group (or the running
+            // sum of the segments of the tile's only group)
+            int32_t part[64];
 #pragma unroll
-            for (int cc = 0; cc < 4; ++cc) {
-                const int nb = n0 + half * 64 + cc * 16;
-                uint32_t v[2][16];
-                tmem_ld16x2(lane_base + (uint32_t)((b * 2 + 0) * BN + half * 64 + cc * 16),
-                            lane_base + (uint32_t)((b * 2 + 1) * BN + half * 64 + cc * 16), v[0], v[1]);
-                int32_t acc[2][16];
-#pragma unroll
-                for (int g = 0; g < 2; ++g) {
-                    const SGroup& G = p.g[g];
-                    if (G.stages == 0) {
-#pragma unroll
-                        for (int q = 0; q < 16; ++q) acc[g][q] = 0;
-                        continue;
-                    }
-                    if (g == gs) {
-#pragma unroll
-                        for (int q = 0; q < 16; ++q) acc[g][q] = sacc[cc * 16 + q];
-                    } else {
-#pragma unroll
-                        for (int q = 0; q < 16; ++q)
-                            acc[g][q] = __float2int_rn(__uint_as_float(v[g][q]) * G.acc_scale);
-                    }
-                    if (G.center) {
-#pragma unroll
-                        for (int q = 0; q < 16; ++q) {
-                            const int n = nb + q;
-                            acc[g][q] += n < p.N ? G.center * __ldg(p.colsum + (int64_t)n * 2 + g) : 0;
-                        }
-                    }
+            for (int j = 0; j < 64; ++j) part[j] = 0;
+            const int gA = g_first, gB = 1 - g_first;
+            const int nA = p.g[gA].stages > 0 ? (gA == p.seg_group ? p.g[gA].n_seg : 1) : 0;
+            const int nB = p.g[gB].stages > 0 ? (gB == p.seg_group ? p.g[gB].n_seg : 1) : 0;
+            const int njobs = nA + nB;
+            const int g_last = nB > 0 ? gB : gA;        // group of the final job
+            const bool part_is_other = nA > 0 && nB > 0;
+#pragma unroll 1
+            for (int jj = 0; jj < njobs; ++jj, ++job) {
+                const uint32_t r = job & 1u, use = job >> 1;
+                if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_REG_FULL + r), use & 1u, abort_flag, kTimeoutNs,
+                                                          p.err, kErrWait))) {
+                    ok = false;
+                    break;
                 }
-                if (m < p.M) {
-                    if (p.acc_dbg != nullptr) {
+                tc_fence_after();
+                const uint32_t taddr = lane_base + r * BN;
+                if (jj < njobs - 1) {
+                    // accumulate: a whole first group, or a segment
+                    const int gj = jj < nA ? gA : gB;
+                    const float sc = p.g[gj].acc_scale;
 #pragma unroll
-                        for (int g = 0; g < 2; ++g) {
-                            int32_t* dst = p.acc_dbg + ((int64_t)g * p.M + m) * p.N;
+                    for (int cc = 0; cc < 4; ++cc) {
+                        uint32_t v[16];
+                        tmem_ld16(taddr + cc * 16, v);
 #pragma unroll
-                            for (int q = 0; q < 16; ++q)
-                                if (nb + q < p.N) dst[nb + q] = acc[g][q];
-                        }
+                        for (int q = 0; q < 16; ++q) part[cc * 16 + q] += __float2int_rn(__uint_as_float(v[q]) * sc);
                     }
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar(BAR_REG_EMPTY + r));
+                    if (jj == nA - 1 && part_is_other) {
+                        // the first group is complete: add back its centring
+#pragma unroll
+                        for (int j = 0; j < 64; ++j) part[j] += cs_w[gA * 64 + j];
+                    }
+                    continue;
+                }
+                // the final job: finish the tile's outputs, 16 columns at a time
+                const float sc = p.g[g_last].acc_scale;
+                const bool dbg = p.acc_dbg != nullptr && m < p.M;
+#pragma unroll
+                for (int cc = 0; cc < 4; ++cc) {
+                    uint32_t v[16];
+                    tmem_ld16(taddr + cc * 16, v);
+                    const int nb = nc0 + cc * 16;
                     float y[16];
 #pragma unroll
                     for (int q = 0; q < 16; ++q) {
-                        const int n = nb + q < p.N ? nb + q : p.N - 1;
-                        const float sw0 = __ldg(p.s_w + (int64_t)n * 2) * p.g[0].inv_levels;
-                        const float sw1 = __ldg(p.s_w + (int64_t)n * 2 + 1) * p.g[1].inv_levels;
-                        y[q] = fmaf(sa[1] * sw1, (float)acc[1][q], sa[0] * sw0 * (float)acc[0][q]);
+                        const int j = cc * 16 + q;
+                        const int32_t x = __float2int_rn(__uint_as_float(v[q]) * sc) + cs_w[g_last * 64 + j];
+                        const int32_t last = part_is_other ? x : part[j] + x;     // the final job's group
+                        const int32_t other = part_is_other ? part[j] : 0;
+                        const int32_t a0 = g_last == 0 ? last : other;
+                        const int32_t a1 = g_last == 0 ? other : last;
+                        y[q] = fmaf(sa[1] * sw_w[64 + j], (float)a1, sa[0] * sw_w[j] * (float)a0);
+                        if (dbg && nb + q < p.N) {
+                            p.acc_dbg[m * p.N + nb + q] = a0;
+                            p.acc_dbg[(p.M + m) * p.N + nb + q] = a1;
+                        }
                     }
-                    store_out16(p, m, nb, y);
+                    if (m < p.M) store_out16(p, m, nb, y);
                 }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(BAR_REG_EMPTY + r));
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(BAR_ACC_EMPTY + b));
         }
     }
 
@@ -543,11 +539,12 @@ EncodeTiledFn encode_fn() {
 }
 
 // 2-D map over expanded rows [rows][row_bytes] with a box of one 128-byte
-// K-stage by 128 rows, 128-byte swizzle (the layout the MMA descriptors read).
-bool encode_rows(EncodeTiledFn enc, CUtensorMap* map, const uint8_t* base, int64_t row_bytes, int64_t rows) {
+// K-stage by box_rows rows, 128-byte swizzle (the layout the MMA descriptors read).
+bool encode_rows(EncodeTiledFn enc, CUtensorMap* map, const uint8_t* base, int64_t row_bytes, int64_t rows,
+                 int box_rows) {
     cuuint64_t dims[2] = {(cuuint64_t)row_bytes, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
-    cuuint32_t box[2] = {128u, 128u};
+    cuuint32_t box[2] = {128u, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -666,7 +663,7 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     memset(&p, 0, sizeof(p));
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;
-    if (!encode_rows(enc, &p.tma_a, xa, sp.eb, rows_a) || !encode_rows(enc, &p.tma_b, xw, sp.eb, a.N))
+    if (!encode_rows(enc, &p.tma_a, xa, sp.eb, rows_a, BM) || !encode_rows(enc, &p.tma_b, xw, sp.eb, a.N, BN))
         return cudaErrorInvalidValue;
     p.s_a = a.s_a;
     p.s_w = a.s_w;
