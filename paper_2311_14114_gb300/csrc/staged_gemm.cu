@@ -40,9 +40,11 @@
 //               k of the CTA accumulates into TMEM region k % 2 (256 columns
 //               each), so the epilogue drains one region while the MMAs fill
 //               the other, across tile boundaries too
-//   warps 2-17  epilogue: four warps per TMEM lane quadrant, 64 columns each;
+//   warps 2-9   epilogue: two warps per TMEM lane quadrant, 128 columns each;
 //               earlier jobs of a tile are summed into int32 registers, the
-//               final job completes the outputs
+//               final job completes the outputs, which leave through shared
+//               memory and TMA stores (ten warps in all, so that each thread
+//               can hold 128 partial sums in registers)
 // Every wait is bounded (2 s); a wait that runs out records an error bit,
 // raises a CTA abort flag and the CTA winds down (copies and MMAs in flight
 // are waited for, TMEM is freed).
@@ -62,17 +64,20 @@ using namespace tc;
 
 constexpr int BM = 128;
 constexpr int BN = 256;
-constexpr int STAGES = 4;
+constexpr int STAGES = 3;
 constexpr int A_BYTES = BM * 128;
 constexpr int B_BYTES = BN * 128;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int NUM_EPI_WARPS = 16;
+constexpr int NUM_EPI_WARPS = 8;
 constexpr int WARP_TMA = 0, WARP_MMA = 1, WARP_EPI = 2;
 constexpr int NUM_THREADS = (2 + NUM_EPI_WARPS) * 32;
 constexpr int BAR_FULL = 0, BAR_EMPTY = STAGES, BAR_REG_FULL = 2 * STAGES, BAR_REG_EMPTY = 2 * STAGES + 2,
               BAR_TEARDOWN = 2 * STAGES + 4, NUM_BARS = 2 * STAGES + 5;
-constexpr int COLS_PER_WARP = 2 * 2 * 64 * 4;           // [s_w | center * C][group][64 columns], 4 bytes each
-constexpr int SMEM_COLS = STAGES * STAGE_BYTES;
+constexpr int EPI_COLS = BN / (NUM_EPI_WARPS / 4);     // columns per epilogue warp (128)
+constexpr int COLS_PER_WARP = EPI_COLS * 16;            // float4 per column: s_w0', s_w1', center*C0, center*C1
+constexpr int OUT_PER_WARP = 32 * EPI_COLS * 2;         // a warp's 32 x 128 outputs: two 64-column boxes, 128-byte swizzled
+constexpr int SMEM_OUT = STAGES * STAGE_BYTES;
+constexpr int SMEM_COLS = SMEM_OUT + NUM_EPI_WARPS * OUT_PER_WARP;
 constexpr int SMEM_BAR = SMEM_COLS + NUM_EPI_WARPS * COLS_PER_WARP;
 constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;   // tmem base, abort flag, a zero word
 constexpr int SMEM_TOTAL = SMEM_MISC + 16;
@@ -94,6 +99,7 @@ struct SGroup {
 struct SParams {
     CUtensorMap tma_a;     // expanded activations [rows][eb]
     CUtensorMap tma_b;     // expanded weights [N][eb]
+    CUtensorMap tma_y;     // outputs [M][N] (2-byte elements), 64 x 32 boxes, when y_tma
     const float* s_a;
     const float* s_w;
     const int32_t* colsum; // [N][2] weight code sums
@@ -107,6 +113,7 @@ struct SParams {
     int32_t out_bf16;
     int32_t seg_group;     // group accumulated in drained segments, or -1
     int32_t drop_first;    // test hook: the producer never issues the first K-stage
+    int32_t y_tma;         // 1: outputs leave through shared memory and TMA stores
     SGroup g[2];
 };
 
@@ -232,6 +239,39 @@ __global__ void __launch_bounds__(256) expand_kernel(const ExpandParams p) {
 // The persistent GEMM over expanded operands
 // ---------------------------------------------------------------------------
 
+// 8 consecutive outputs of row m from column nb (one 16-byte store when aligned).
+__device__ __forceinline__ void store_out8(const SParams& p, int64_t m, int nb, const float (&y)[8]) {
+    const bool vec = nb + 8 <= p.N && (p.N & 7) == 0;
+    uint32_t wv[4];
+    if (p.out_bf16) {
+        __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(p.Y) + m * p.N;
+        if (vec) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                __nv_bfloat162 h2 = __floats2bfloat162_rn(y[2 * e], y[2 * e + 1]);
+                wv[e] = *reinterpret_cast<uint32_t*>(&h2);
+            }
+            *reinterpret_cast<uint4*>(dst + nb) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+        } else {
+            for (int j = 0; j < 8; ++j)
+                if (nb + j < p.N) dst[nb + j] = __float2bfloat16_rn(y[j]);
+        }
+    } else {
+        __half* dst = reinterpret_cast<__half*>(p.Y) + m * p.N;
+        if (vec) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                __half2 h2 = __floats2half2_rn(y[2 * e], y[2 * e + 1]);
+                wv[e] = *reinterpret_cast<uint32_t*>(&h2);
+            }
+            *reinterpret_cast<uint4*>(dst + nb) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+        } else {
+            for (int j = 0; j < 8; ++j)
+                if (nb + j < p.N) dst[nb + j] = __float2half_rn(y[j]);
+        }
+    }
+}
+
 __device__ __forceinline__ void store_out16(const SParams& p, int64_t m, int nb, const float (&y)[16]) {
     const bool vec = nb + 16 <= p.N && (p.N & 7) == 0;
     if (p.out_bf16) {
@@ -277,6 +317,7 @@ __device__ __forceinline__ void store_out16(const SParams& p, int64_t m, int nb,
 // epilogue drains one region while the MMAs fill the other.
 __device__ __forceinline__ int first_group(const SParams& p) { return p.seg_group == 1 ? 1 : 0; }
 
+template <bool DBG>
 __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid_constant__ SParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -401,43 +442,45 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     } else {
         // ------------------------------------------------------------- epilogue
         // Warp w reads TMEM lane quadrant w % 4 (rows 32*(w%4) .. +31 of the
-        // tile) and the 64 columns cgrp*64 .. +63, cgrp = (w - 2) / 4.
+        // tile) and the 128 columns cgrp*128 .. +127, cgrp = (w - 2) / 4.
         const int ew = warp - WARP_EPI;
         const int quad = warp & 3;
         const int cgrp = ew >> 2;
         const int row = quad * 32 + lane;
-        const uint32_t lane_base = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(cgrp * 64);
-        // this warp's copy of the tile's column constants: s_w * inv_levels and
-        // center * (weight code sum), [group][64 columns]
-        float* sw_w = reinterpret_cast<float*>(smem + SMEM_COLS + ew * COLS_PER_WARP);
-        int32_t* cs_w = reinterpret_cast<int32_t*>(smem + SMEM_COLS + ew * COLS_PER_WARP + 2 * 64 * 4);
+        const uint32_t lane_base = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(cgrp * EPI_COLS);
+        // this warp's copy of the tile's column constants: {s_w0 * inv_levels0,
+        // s_w1 * inv_levels1, center0 * C0, center1 * C1} per column
+        float4* colc = reinterpret_cast<float4*>(smem + SMEM_COLS + ew * COLS_PER_WARP);
+        const uint32_t out_s = sbase + (uint32_t)(SMEM_OUT + ew * OUT_PER_WARP);   // 1024-aligned
         uint32_t job = 0;
         bool ok = true;
         for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
             const int64_t m0 = (int64_t)(t % p.m_tiles) * BM;
-            const int nc0 = (t / p.m_tiles) * BN + cgrp * 64;    // this warp's first column
+            const int nc0 = (t / p.m_tiles) * BN + cgrp * EPI_COLS;    // this warp's first column
             __syncwarp();
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
+            for (int h = 0; h < EPI_COLS / 32; ++h) {
                 const int c = lane + 32 * h;
                 const int n = nc0 + c < p.N ? nc0 + c : p.N - 1;
-#pragma unroll
-                for (int g = 0; g < 2; ++g) {
-                    sw_w[g * 64 + c] = __ldg(p.s_w + (int64_t)n * 2 + g) * p.g[g].inv_levels;
-                    cs_w[g * 64 + c] = p.g[g].center ? p.g[g].center * __ldg(p.colsum + (int64_t)n * 2 + g) : 0;
-                }
+                float4 k;
+                k.x = __ldg(p.s_w + (int64_t)n * 2) * p.g[0].inv_levels;
+                k.y = __ldg(p.s_w + (int64_t)n * 2 + 1) * p.g[1].inv_levels;
+                k.z = __int_as_float(p.g[0].center ? p.g[0].center * __ldg(p.colsum + (int64_t)n * 2) : 0);
+                k.w = __int_as_float(p.g[1].center ? p.g[1].center * __ldg(p.colsum + (int64_t)n * 2 + 1) : 0);
+                colc[c] = k;
             }
             __syncwarp();
             const int64_t m = m0 + row;
-            float sa[2];
-#pragma unroll
-            for (int g = 0; g < 2; ++g)
-                sa[g] = m < p.M ? (p.s_a_per_row ? __ldg(p.s_a + m * 2 + g) : __ldg(p.s_a + g)) : 0.0f;
+            float sa0 = 0.0f, sa1 = 0.0f;
+            if (m < p.M) {
+                sa0 = p.s_a_per_row ? __ldg(p.s_a + m * 2) : __ldg(p.s_a);
+                sa1 = p.s_a_per_row ? __ldg(p.s_a + m * 2 + 1) : __ldg(p.s_a + 1);
+            }
             // part: the exact accumulator of the first group (or the running
             // sum of the segments of the tile's only group)
-            int32_t part[64];
+            int32_t part[EPI_COLS];
 #pragma unroll
-            for (int j = 0; j < 64; ++j) part[j] = 0;
+            for (int j = 0; j < EPI_COLS; ++j) part[j] = 0;
             const int gA = g_first, gB = 1 - g_first;
             const int nA = p.g[gA].stages > 0 ? (gA == p.seg_group ? p.g[gA].n_seg : 1) : 0;
             const int nB = p.g[gB].stages > 0 ? (gB == p.seg_group ? p.g[gB].n_seg : 1) : 0;
@@ -459,11 +502,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     const int gj = jj < nA ? gA : gB;
                     const float sc = p.g[gj].acc_scale;
 #pragma unroll
-                    for (int cc = 0; cc < 4; ++cc) {
-                        uint32_t v[16];
-                        tmem_ld16(taddr + cc * 16, v);
+                    for (int cc = 0; cc < EPI_COLS / 8; ++cc) {
+                        uint32_t v[8];
+                        tmem_ld8(taddr + cc * 8, v);
 #pragma unroll
-                        for (int q = 0; q < 16; ++q) part[cc * 16 + q] += __float2int_rn(__uint_as_float(v[q]) * sc);
+                        for (int q = 0; q < 8; ++q) part[cc * 8 + q] += __float2int_rn(__uint_as_float(v[q]) * sc);
                     }
                     tc_fence_before();
                     __syncwarp();
@@ -471,40 +514,82 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     if (jj == nA - 1 && part_is_other) {
                         // the first group is complete: add back its centring
 #pragma unroll
-                        for (int j = 0; j < 64; ++j) part[j] += cs_w[gA * 64 + j];
+                        for (int j = 0; j < EPI_COLS; ++j) {
+                            const float4 k = colc[j];
+                            part[j] += __float_as_int(gA == 0 ? k.z : k.w);
+                        }
                     }
                     continue;
                 }
-                // the final job: finish the tile's outputs, 16 columns at a time
+                // the final job: finish the tile's outputs, 8 columns at a time
                 const float sc = p.g[g_last].acc_scale;
-                const bool dbg = p.acc_dbg != nullptr && m < p.M;
+                const bool dbg = DBG && m < p.M;
+                if (p.y_tma) {
+                    // the previous tile's store must have read the staging buffer
+                    if (lane == 0) bulk_wait_read0();
+                    __syncwarp();
+                }
 #pragma unroll
-                for (int cc = 0; cc < 4; ++cc) {
-                    uint32_t v[16];
-                    tmem_ld16(taddr + cc * 16, v);
-                    const int nb = nc0 + cc * 16;
-                    float y[16];
+                for (int cc = 0; cc < EPI_COLS / 8; ++cc) {
+                    uint32_t v[8];
+                    tmem_ld8(taddr + cc * 8, v);
+                    const int nb = nc0 + cc * 8;
+                    float y[8];
 #pragma unroll
-                    for (int q = 0; q < 16; ++q) {
-                        const int j = cc * 16 + q;
-                        const int32_t x = __float2int_rn(__uint_as_float(v[q]) * sc) + cs_w[g_last * 64 + j];
+                    for (int q = 0; q < 8; ++q) {
+                        const int j = cc * 8 + q;
+                        const float4 k = colc[j];
+                        const int32_t x = __float2int_rn(__uint_as_float(v[q]) * sc) +
+                                          __float_as_int(g_last == 0 ? k.z : k.w);
                         const int32_t last = part_is_other ? x : part[j] + x;     // the final job's group
                         const int32_t other = part_is_other ? part[j] : 0;
                         const int32_t a0 = g_last == 0 ? last : other;
                         const int32_t a1 = g_last == 0 ? other : last;
-                        y[q] = fmaf(sa[1] * sw_w[64 + j], (float)a1, sa[0] * sw_w[j] * (float)a0);
+                        y[q] = fmaf(sa1 * k.y, (float)a1, sa0 * k.x * (float)a0);
                         if (dbg && nb + q < p.N) {
                             p.acc_dbg[m * p.N + nb + q] = a0;
                             p.acc_dbg[(p.M + m) * p.N + nb + q] = a1;
                         }
                     }
-                    if (m < p.M) store_out16(p, m, nb, y);
+                    if (p.y_tma) {
+                        uint32_t w[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            if (p.out_bf16) {
+                                __nv_bfloat162 h2 = __floats2bfloat162_rn(y[2 * e], y[2 * e + 1]);
+                                w[e] = *reinterpret_cast<uint32_t*>(&h2);
+                            } else {
+                                __half2 h2 = __floats2half2_rn(y[2 * e], y[2 * e + 1]);
+                                w[e] = *reinterpret_cast<uint32_t*>(&h2);
+                            }
+                        }
+                        // box cc / 8 (64 columns), row `lane`, 16-byte chunk cc % 8, 128-byte swizzle
+                        // (the TMA store map's layout)
+                        const uint32_t dst = out_s + (uint32_t)(cc >> 3) * 4096u + (uint32_t)lane * 128u +
+                                             ((((uint32_t)cc & 7u) ^ ((uint32_t)lane & 7u)) << 4);
+                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w[0]), "r"(w[1]),
+                                     "r"(w[2]), "r"(w[3])
+                                     : "memory");
+                    } else if (m < p.M) {
+                        store_out8(p, m, nb, y);
+                    }
                 }
                 tc_fence_before();
+                if (p.y_tma) fence_proxy_async_shared();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(bar(BAR_REG_EMPTY + r));
+                if (lane == 0) {
+                    mbar_arrive(bar(BAR_REG_EMPTY + r));
+                    if (p.y_tma) {
+                        // rows and columns beyond M and N are clipped by the store
+#pragma unroll
+                        for (int bx = 0; bx < EPI_COLS / 64; ++bx)
+                            tma_store_2d(&p.tma_y, nc0 + bx * 64, (int)(m0 + quad * 32), out_s + bx * 4096u);
+                        bulk_commit();
+                    }
+                }
             }
         }
+        if (p.y_tma && lane == 0) bulk_wait0();   // stores complete before the CTA exits
     }
 
     tc_fence_before();
@@ -681,6 +766,19 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     p.out_bf16 = a.out_bf16;
     p.seg_group = sp.seg_group;
     p.drop_first = (a.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) != 0 ? 1 : 0;
+    // outputs through TMA stores when the row pitch allows a tensor map (N * 2 bytes a multiple of 16)
+    p.y_tma = 0;
+    if (a.N % 8 == 0 && (uintptr_t)a.Y % 16 == 0) {
+        cuuint64_t dims[2] = {(cuuint64_t)a.N, (cuuint64_t)a.M};
+        cuuint64_t strides[1] = {(cuuint64_t)a.N * 2};
+        cuuint32_t box[2] = {64u, 32u};
+        cuuint32_t estr[2] = {1, 1};
+        if (enc(&p.tma_y, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, a.Y, dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        p.y_tma = 1;
+    }
     for (int g = 0; g < 2; ++g) {
         const GroupGeom& G = geo.g[g];
         SGroup& S = p.g[g];
@@ -697,14 +795,21 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        if ((err = cudaFuncSetAttribute(staged_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
-            cudaSuccess)
+        if ((err = cudaFuncSetAttribute(staged_mma_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        SMEM_ALLOC)) != cudaSuccess ||
+            (err = cudaFuncSetAttribute(staged_mma_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        SMEM_ALLOC)) != cudaSuccess)
             return err;
         attr_done[dev] = true;
     }
-    if ((err = prefer_max_shared((const void*)staged_mma_kernel)) != cudaSuccess) return err;
     const int grid = p.total_tiles < num_sms() ? p.total_tiles : num_sms();
-    staged_mma_kernel<<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
+    if (a.acc_dbg != nullptr) {
+        if ((err = prefer_max_shared((const void*)staged_mma_kernel<true>)) != cudaSuccess) return err;
+        staged_mma_kernel<true><<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
+    } else {
+        if ((err = prefer_max_shared((const void*)staged_mma_kernel<false>)) != cudaSuccess) return err;
+        staged_mma_kernel<false><<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
+    }
     note_launch();
     return cudaGetLastError();
 }
