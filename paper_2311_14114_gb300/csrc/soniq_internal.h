@@ -115,7 +115,7 @@ cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st)
 // then a persistent tcgen05 GEMM runs over them.
 struct StagedGroup {
     int32_t kind;          // 0: E4M3, 1: fp16
-    int32_t stages;        // 128-byte K-stages
+    int32_t stages;        // K-stages of the ring (128 bytes of K each)
     int32_t x0;            // byte offset of the group in an expanded row
     int32_t seg_stages;    // K-stages per exact fp32 segment
     int32_t n_seg;         // segments (> 1: drained to int32)

@@ -64,9 +64,10 @@ using namespace tc;
 
 constexpr int BM = 128;
 constexpr int BN = 256;
+constexpr int KSTAGE = 128;                          // bytes of K per ring stage (128-byte swizzle)
 constexpr int STAGES = 3;
-constexpr int A_BYTES = BM * 128;
-constexpr int B_BYTES = BN * 128;
+constexpr int A_BYTES = BM * KSTAGE;
+constexpr int B_BYTES = BN * KSTAGE;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int WARP_TMA = 0, WARP_MMA = 1, WARP_EPI = 2;
@@ -376,8 +377,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                         if (p.drop_first && s == 0) continue;   // the MMA's wait for it runs out
                         const uint32_t dst = sbase + slot * STAGE_BYTES;
                         mbar_arrive_expect_tx(bar(BAR_FULL + slot), STAGE_BYTES);
-                        tma_load_2d(dst, &p.tma_a, x0 + i * 128, m0, bar(BAR_FULL + slot));
-                        tma_load_2d(dst + A_BYTES, &p.tma_b, x0 + i * 128, n0, bar(BAR_FULL + slot));
+                        tma_load_2d(dst, &p.tma_a, x0 + i * KSTAGE, m0, bar(BAR_FULL + slot));
+                        tma_load_2d(dst + A_BYTES, &p.tma_b, x0 + i * KSTAGE, n0, bar(BAR_FULL + slot));
                     }
                 }
             }
@@ -391,6 +392,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
         if (lane == 0) {
             uint32_t s = 0, job = 0;
             bool ok = true;
+            const uint64_t a_desc0 = KSTAGE == 128 ? sw128_desc(sbase) : sw64_desc(sbase);
             for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
 #pragma unroll 1
                 for (int gi = 0; gi < 2 && ok; ++gi) {
@@ -417,17 +419,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                                 break;
                             }
                             tc_fence_after();
-                            const uint32_t a_addr = sbase + slot * STAGE_BYTES, b_addr = a_addr + A_BYTES;
+                            // descriptors of this stage; +32 bytes of K is +2 in the start-address field
+                            const uint64_t ad = a_desc0 + (uint64_t)((slot * STAGE_BYTES) >> 4);
+                            const uint64_t bd = ad + (uint64_t)(A_BYTES >> 4);
                             if (f8) {
 #pragma unroll
-                                for (int k = 0; k < 4; ++k)
-                                    mma_f8<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
-                                                  (q == 0 && k == 0) ? 0u : 1u);
+                                for (int k = 0; k < KSTAGE / 32; ++k)
+                                    mma_f8<IDESC>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
                             } else {
 #pragma unroll
-                                for (int k = 0; k < 4; ++k)
-                                    mma_f16<IDESC>(d, sw128_desc(a_addr + 32 * k), sw128_desc(b_addr + 32 * k),
-                                                   (q == 0 && k == 0) ? 0u : 1u);
+                                for (int k = 0; k < KSTAGE / 32; ++k)
+                                    mma_f16<IDESC>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
                             }
                             mma_commit(bar(BAR_EMPTY + slot));
                         }
@@ -629,10 +631,11 @@ bool encode_rows(EncodeTiledFn enc, CUtensorMap* map, const uint8_t* base, int64
                  int box_rows) {
     cuuint64_t dims[2] = {(cuuint64_t)row_bytes, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
-    cuuint32_t box[2] = {128u, (cuuint32_t)box_rows};
+    cuuint32_t box[2] = {(cuuint32_t)KSTAGE, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, KSTAGE == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -649,12 +652,12 @@ bool staged_plan(const LayoutGeom& geo, StagedPlan* sp) {
         StagedGroup& S = sp->g[g];
         S.kind = (G.bits_a <= 4 && G.bits_w <= 4) ? 0 : 1;
         const int64_t bytes = (int64_t)G.pw * (S.kind == 0 ? 1 : 2);
-        S.stages = (int32_t)(bytes / 128);
+        S.stages = (int32_t)(bytes / staged::KSTAGE);
         S.x0 = (int32_t)x0;
         x0 += bytes;
         const int64_t maxprod = S.kind == 0 ? (int64_t)((1 << G.bits_a) - 1) * (1 << (G.bits_w - 1))
                                             : (int64_t)(1 << (G.bits_a - 1)) * (1 << (G.bits_w - 1));
-        const int64_t codes_per_stage = S.kind == 0 ? 128 : 64;
+        const int64_t codes_per_stage = S.kind == 0 ? staged::KSTAGE : staged::KSTAGE / 2;
         const int64_t seg_stages = ((int64_t)1 << 24) / maxprod / codes_per_stage;
         if (seg_stages < 1) return false;
         S.seg_stages = (int32_t)(seg_stages < S.stages ? seg_stages : (S.stages > 0 ? S.stages : 1));

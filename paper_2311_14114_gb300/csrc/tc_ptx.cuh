@@ -112,6 +112,17 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
     return d;
 }
 
+// 64-byte-swizzle K-major shared-memory matrix descriptor: 8-row x 64-byte
+// atoms stacked along M/N every 512 bytes.
+__device__ __forceinline__ uint64_t sw64_desc(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;              // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(512 >> 4) << 32;     // stride byte offset: next 8-row atom
+    d |= (uint64_t)1 << 46;              // descriptor version
+    d |= (uint64_t)4 << 61;              // SWIZZLE_64B
+    return d;
+}
+
 // Instruction descriptor: fp32 accumulator, A/B format 0 (E4M3 for
 // kind::f8f6f4, F16 for kind::f16), both K-major, N x M = bn x bm.
 __host__ __device__ constexpr uint32_t idesc(int bm, int bn) {
