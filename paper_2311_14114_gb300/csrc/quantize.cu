@@ -2,7 +2,8 @@
 // Operations" steps 1-3 with the channel permutation and padding of Sec. 4.1.
 //
 //   act_absmax_kernel     per-(tensor, group) max |a|            (step 1)
-//   quantize_act_kernel   gather by perm, unsigned codes, pack    (steps 1-2)
+//   quantize_tiles_kernel permute, unsigned codes, pack            (steps 1-2)
+//   quantize_fused_kernel per-tensor scale, codes and pack in one pass (steps 1-2)
 //   weight_absmax_kernel  per-(tensor, group) max |w|             (step 1)
 //   pack_weights_kernel   per-(row, group) scale, Eq. (1) codes, pack (steps 1, 3)
 //
@@ -114,15 +115,25 @@ __global__ void __launch_bounds__(kThreads) act_absmax_kernel(const uint4* __res
 #pragma unroll
             for (int q = 0; q < 4; ++q)
                 m1[q] = (grp[8 * j + 2 * q] ? 0x0000FFFFu : 0u) | (grp[8 * j + 2 * q + 1] ? 0xFFFF0000u : 0u);
-            for (int64_t m = (int64_t)blockIdx.x * rpar + tr; m < rows; m += (int64_t)gridDim.x * rpar) {
-                const uint4 v = __ldg(X + m * KV + j);
-                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+            // eight rows' loads in flight before they are reduced
+            const int64_t rstep = (int64_t)gridDim.x * rpar;
+            for (int64_t m0 = (int64_t)blockIdx.x * rpar + tr; m0 < rows; m0 += 8 * rstep) {
+                uint4 v[8];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint32_t x = w[q] & 0x7FFF7FFFu;
-                    x &= __vcmpleu2(x, 0x7C007C00u);          // NaN -> 0
-                    g1 = __vmaxu2(g1, x & m1[q]);
-                    g0 = __vmaxu2(g0, x & ~m1[q]);
+                for (int u = 0; u < 8; ++u) {
+                    const int64_t m = m0 + u * rstep;
+                    v[u] = m < rows ? __ldg(X + m * KV + j) : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int u = 0; u < 8; ++u) {
+                    const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint32_t x = w[q] & 0x7FFF7FFFu;
+                        x &= __vcmpleu2(x, 0x7C007C00u);          // NaN -> 0
+                        g1 = __vmaxu2(g1, x & m1[q]);
+                        g0 = __vmaxu2(g0, x & ~m1[q]);
+                    }
                 }
             }
         }
@@ -138,31 +149,6 @@ __global__ void __launch_bounds__(kThreads) act_absmax_kernel(const uint4* __res
         atomicMax(s_bits + 1, __float_as_uint(mx1));
     }
 }
-
-// ---------------------------------------------------------------------------
-// Activation quantize-and-pack.  A CTA stages a tile of rows in shared memory
-// already permuted and padded (packed position order, group g starting at
-// g ? pa0 : 0), so that each 32-code block is 64 contiguous bytes.  Four
-// consecutive threads share a block, one quarter (8 codes, 16 bytes) each:
-// they quantize (Sec. 3 step 2), build their part of each bit slice, and
-// combine the 2-bit and 1-bit slice words with two width-4 shuffles.
-// ---------------------------------------------------------------------------
-struct QuantActParams {
-    const uint16_t* A;
-    uint8_t* Ap;
-    float* s_a;
-    const int32_t* perm;
-    int64_t M;
-    int32_t K;
-    int32_t a_row_bytes;
-    int32_t scale_mode;
-    int32_t vec_ok;
-    int32_t tile_rows;       // rows staged per CTA
-    int32_t row_halves;      // pa0 + pa1: staged row length
-    int32_t nblk0;           // 32-code blocks of group 0 per row
-    int32_t nblk;            // blocks of both groups per row
-    GroupGeom g[2];
-};
 
 // The code of Sec. 3 step 2, t = (a / s) * (2^n - 1) rounded half to even and
 // clipped to [0, 2^n - 1].  The quotient is formed by Markstein's correction
@@ -217,125 +203,6 @@ __device__ __forceinline__ void quarter_codes(const uint4 x, int valid, const QC
             v |= (u0 | (u1 << 8)) << (16 * e);
         }
         o[i] = v;
-    }
-}
-
-__global__ void __launch_bounds__(256) quantize_act_kernel(const QuantActParams p) {
-    extern __shared__ __align__(16) uint8_t smem[];
-    uint16_t* pos_s = reinterpret_cast<uint16_t*>(smem);              // original channel -> staged position
-    const int pos_bytes = (p.K * 2 + 15) & ~15;
-    float* scale_s = reinterpret_cast<float*>(smem + pos_bytes);      // [tile_rows][2]
-    const int scale_bytes = (p.tile_rows * 8 + 15) & ~15;
-    __half* rows_s = reinterpret_cast<__half*>(smem + pos_bytes + scale_bytes);   // [tile_rows][RH]
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-    const int RH = p.row_halves;
-
-    const int c0 = p.g[0].count, pa0 = p.g[0].pa;
-    for (int j = threadIdx.x; j < p.K; j += blockDim.x) pos_s[p.perm[j]] = (uint16_t)(j < c0 ? j : pa0 + (j - c0));
-    const bool per_row = p.scale_mode == SONIQ_SCALE_PER_ROW;
-    const QConst tk0 = make_qconst(per_row ? 0.0f : p.s_a[0], p.g[0].bits_a);
-    const QConst tk1 = make_qconst(per_row ? 0.0f : p.s_a[1], p.g[1].bits_a);
-    // staging map: thread -> (row offset, 16-byte column); no division in the loop
-    const int kv = p.K >> 3;
-    const int scols = kv < (int)blockDim.x ? kv : (int)blockDim.x;
-    const int srows = blockDim.x / scols;
-    const int s_tc = threadIdx.x % scols, s_tr = threadIdx.x / scols;
-    __syncthreads();
-
-    for (int64_t m0 = (int64_t)blockIdx.x * p.tile_rows; m0 < p.M; m0 += (int64_t)gridDim.x * p.tile_rows) {
-        const int nr = p.M - m0 < p.tile_rows ? (int)(p.M - m0) : p.tile_rows;
-        // stage: row r, original channel c -> rows_s[r * RH + pos(c)]
-        if (p.vec_ok) {
-            const uint4* src = reinterpret_cast<const uint4*>(p.A + m0 * p.K);
-            if (s_tr < srows) {
-                for (int j = s_tc; j < kv; j += scols) {
-                    const uint4 ps = *reinterpret_cast<const uint4*>(pos_s + 8 * j);
-                    const uint32_t pw[4] = {ps.x, ps.y, ps.z, ps.w};
-                    for (int r = s_tr; r < nr; r += srows) {
-                        const uint4 v = __ldg(src + (int64_t)r * kv + j);
-                        const uint32_t vw[4] = {v.x, v.y, v.z, v.w};
-                        uint16_t* dst = reinterpret_cast<uint16_t*>(rows_s) + r * RH;
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            dst[pw[q] & 0xFFFFu] = (uint16_t)(vw[q] & 0xFFFFu);
-                            dst[pw[q] >> 16] = (uint16_t)(vw[q] >> 16);
-                        }
-                    }
-                }
-            }
-        } else {
-            const uint16_t* src = p.A + m0 * p.K;
-            for (int i = threadIdx.x; i < nr * p.K; i += blockDim.x) {
-                const int r = i / p.K, c = i - r * p.K;
-                reinterpret_cast<uint16_t*>(rows_s)[r * RH + pos_s[c]] = src[i];
-            }
-        }
-        __syncthreads();
-        if (per_row) {
-            // max |a| of each staged row and group (the group's channels are contiguous here)
-            for (int r = warp; r < nr; r += nwarps) {
-                const __half* row = rows_s + r * RH;
-#pragma unroll
-                for (int g = 0; g < 2; ++g) {
-                    const int base = g ? pa0 : 0;
-                    float mx = 0.0f;
-                    for (int j = lane; j < p.g[g].count; j += 32) mx = fmaxf(mx, fabsf(__half2float(row[base + j])));
-                    mx = warp_max(mx);
-                    if (lane == 0) {
-                        scale_s[2 * r + g] = mx;
-                        p.s_a[(m0 + r) * 2 + g] = mx;
-                    }
-                }
-            }
-            __syncthreads();
-        }
-        // quarter-block tasks, whole warps at a time so that the shuffles see all lanes
-        const int tasks = nr * p.nblk * 4;
-        for (int base = warp * 32; base < tasks; base += nwarps * 32) {
-            const int t = base + lane;
-            const bool live = t < tasks;                   // whole 4-lane groups are live or not
-            const int blk = (live ? t : 0) >> 2, qq = t & 3;
-            const int r = blk / p.nblk;
-            const int kb = blk - r * p.nblk;
-            const int g = kb >= p.nblk0;
-            const int kbg = kb - (g ? p.nblk0 : 0);
-            const int n = p.g[g].bits_a;
-            const QConst k = per_row ? make_qconst(scale_s[2 * r + g], n) : (g ? tk1 : tk0);
-            const int valid = p.g[g].count - kbg * 32 - 8 * qq;   // channels of this quarter; the rest is padding
-            const uint4 x = *reinterpret_cast<const uint4*>(rows_s + r * RH + (g ? pa0 : 0) + kbg * 32 + 8 * qq);
-            uint32_t o[2];
-            if (k.mode == 1) quarter_codes<true>(x, valid, k, o);
-            else if (k.mode == 2) quarter_codes<false>(x, valid, k, o);
-            else o[0] = o[1] = 0u;                          // no positive scale: every code is 0
-            // this quarter's share of each slice word
-            const uint32_t p4 = (o[0] & 0x0F0F0F0Fu) | ((o[1] & 0x0F0F0F0Fu) << 4);
-            const int off2 = (n & 4) ? 4 : 0, off1 = off2 + ((n & 2) ? 2 : 0);
-            const int j2 = 2 * (qq & 1);
-            uint32_t p2 = (((o[0] >> off2) & 0x03030303u) << (2 * j2)) | (((o[1] >> off2) & 0x03030303u) << (2 * j2 + 2));
-            uint32_t p1 = (((o[0] >> off1) & 0x01010101u) << (2 * qq)) | (((o[1] >> off1) & 0x01010101u) << (2 * qq + 1));
-            p2 |= __shfl_xor_sync(0xffffffffu, p2, 1, 4);
-            p1 |= __shfl_xor_sync(0xffffffffu, p1, 1, 4);
-            p1 |= __shfl_xor_sync(0xffffffffu, p1, 2, 4);
-            if (!live) continue;
-            uint32_t* dst = reinterpret_cast<uint32_t*>(p.Ap + (m0 + r) * (int64_t)p.a_row_bytes + p.g[g].a_off +
-                                                        kbg * 4 * n);
-            if (n == 8) {
-                dst[2 * qq] = o[0];
-                dst[2 * qq + 1] = o[1];
-            } else {
-                int w = 0;
-                if (n & 4) {
-                    dst[qq] = p4;
-                    w = 4;
-                }
-                if (n & 2) {
-                    if ((qq & 1) == 0) dst[w + (qq >> 1)] = p2;
-                    w += 2;
-                }
-                if ((n & 1) && qq == 0) dst[w] = p1;
-            }
-        }
-        __syncthreads();   // the tile is overwritten next
     }
 }
 
@@ -686,6 +553,194 @@ __global__ void __launch_bounds__(128) pack_weights_kernel(const PackWParams p) 
     }
 }
 
+// ---------------------------------------------------------------------------
+// Activation quantize-and-pack over tiles of rows (persistent CTAs of 1024
+// threads).  A tile of rows is staged in shared memory already permuted and
+// padded (Sec. 3 "Dynamic channel re-ordering"; the padding slots are zeroed
+// once and never written again), so every 32-code block is 64 contiguous
+// bytes, and one thread turns a block into its packed words (Sec. 3 step 2).
+// While a tile is quantized, the next tile's input is already loading into
+// registers.  Scales: given (per tensor after the max-abs pass, or
+// calibrated), per row (found from the staged row), or per tensor within a
+// single CTA that holds every row (tensor_in_cta, small inputs).
+// ---------------------------------------------------------------------------
+struct TileQuantParams {
+    const uint16_t* A;
+    uint8_t* Ap;
+    float* s_a;
+    const int32_t* perm;
+    int64_t M;
+    int32_t K;
+    int32_t a_row_bytes;
+    int32_t scale_mode;
+    int32_t tensor_in_cta;
+    int32_t vec_ok;          // rows load as 16-byte vectors
+    int32_t tile_rows;       // rows per tile
+    int32_t row_halves;      // pa0 + pa1: staged row length
+    int32_t nblk0, nblk;     // 32-code blocks of group 0 / of both groups per row
+    GroupGeom g[2];
+};
+constexpr int kTileThreads = 1024;
+constexpr int kTilePrefetch = 4;   // 16-byte vectors per thread held in registers for the next tile
+
+// Per-group max |a| of staged rows r0 .. r1-1 (sign cleared, NaN dropped as
+// fmaxf drops it, two halves per instruction); block-wide, all threads.
+__device__ __forceinline__ void staged_group_max(const __half* rows_s, int RH, int pa0, int r0, int r1, float* red,
+                                                 float& f0, float& f1) {
+    uint32_t mx0 = 0u, mx1 = 0u;
+    const int vpr = RH / 8, v0 = pa0 / 8;
+    const uint32_t rs = (uint32_t)__cvta_generic_to_shared(rows_s);
+    for (int i = threadIdx.x; i < (r1 - r0) * vpr; i += blockDim.x) {
+        const int r = r0 + i / vpr, v = i - (i / vpr) * vpr;
+        const uint4 x = lds128q(rs + 16u * (uint32_t)(r * vpr + v));
+        const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
+        uint32_t m = 0u;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t a = xw[q] & 0x7FFF7FFFu;
+            a &= __vcmpleu2(a, 0x7C007C00u);
+            m = __vmaxu2(m, a);
+        }
+        if (v < v0) mx0 = __vmaxu2(mx0, m);
+        else mx1 = __vmaxu2(mx1, m);
+    }
+    mx0 = max(mx0 & 0xFFFFu, mx0 >> 16);
+    mx1 = max(mx1 & 0xFFFFu, mx1 >> 16);
+    f0 = __half2float(__ushort_as_half((unsigned short)mx0));
+    f1 = __half2float(__ushort_as_half((unsigned short)mx1));
+    block_max2(f0, f1, red);
+}
+
+__global__ void __launch_bounds__(kTileThreads, 1) quantize_tiles_kernel(const TileQuantParams p) {
+    extern __shared__ __align__(16) uint8_t smem[];
+    uint16_t* pos_s = reinterpret_cast<uint16_t*>(smem);                  // original channel -> staged position
+    const int pos_bytes = (p.K * 2 + 15) & ~15;
+    float* scale_s = reinterpret_cast<float*>(smem + pos_bytes);          // [tile_rows][2] (per-row scales)
+    const int scale_bytes = (p.tile_rows * 8 + 15) & ~15;
+    __half* rows_s = reinterpret_cast<__half*>(smem + pos_bytes + scale_bytes);
+    __shared__ float red[64];
+    const int RH = p.row_halves, TR = p.tile_rows;
+    const int c0 = p.g[0].count, pa0 = p.g[0].pa;
+    for (int j = threadIdx.x; j < p.K; j += blockDim.x) pos_s[p.perm[j]] = (uint16_t)(j < c0 ? j : pa0 + (j - c0));
+    {
+        uint4* z = reinterpret_cast<uint4*>(rows_s);
+        for (int i = threadIdx.x; i < TR * RH / 8; i += blockDim.x) z[i] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    const bool per_row = p.scale_mode == SONIQ_SCALE_PER_ROW;
+    QConst k0, k1;
+    if (!per_row && !p.tensor_in_cta) {
+        k0 = make_qconst(p.s_a[0], p.g[0].bits_a);
+        k1 = make_qconst(p.s_a[1], p.g[1].bits_a);
+    }
+    __syncthreads();
+    const uint32_t rows_a = (uint32_t)__cvta_generic_to_shared(rows_s);
+    const int KV = p.K >> 3;
+    const int64_t tstep = (int64_t)gridDim.x * TR;
+    // staging map: vector v of a tile is row v / KV, column v % KV; this thread
+    // takes v = tid + u * blockDim for u < kTilePrefetch
+    const int tile_vecs = TR * KV;
+    uint4 nxt[kTilePrefetch];
+    auto load_tile = [&](int64_t m0) {
+        const int nr = p.M - m0 < TR ? (int)(p.M - m0) : TR;
+        const uint4* src = reinterpret_cast<const uint4*>(p.A + m0 * p.K);
+#pragma unroll
+        for (int u = 0; u < kTilePrefetch; ++u) {
+            const int v = threadIdx.x + u * blockDim.x;
+            if (v < tile_vecs && v < nr * KV) nxt[u] = __ldg(src + v);
+        }
+    };
+    auto store_tile = [&](int64_t m0) {
+        const int nr = p.M - m0 < TR ? (int)(p.M - m0) : TR;
+#pragma unroll
+        for (int u = 0; u < kTilePrefetch; ++u) {
+            const int v = threadIdx.x + u * blockDim.x;
+            if (v < tile_vecs && v < nr * KV) {
+                const int r = v / KV, j = v - r * KV;
+                const uint4 ps = *reinterpret_cast<const uint4*>(pos_s + 8 * j);
+                const uint32_t pw[4] = {ps.x, ps.y, ps.z, ps.w};
+                const uint32_t vw[4] = {nxt[u].x, nxt[u].y, nxt[u].z, nxt[u].w};
+                uint16_t* dst = reinterpret_cast<uint16_t*>(rows_s) + r * RH;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    dst[pw[q] & 0xFFFFu] = (uint16_t)(vw[q] & 0xFFFFu);
+                    dst[pw[q] >> 16] = (uint16_t)(vw[q] >> 16);
+                }
+            }
+        }
+    };
+    int64_t m0 = (int64_t)blockIdx.x * TR;
+    if (p.vec_ok && m0 < p.M) load_tile(m0);
+    for (; m0 < p.M; m0 += tstep) {
+        const int nr = p.M - m0 < TR ? (int)(p.M - m0) : TR;
+        // ---- stage this tile (from the registers), then start the next tile's loads ----
+        if (p.vec_ok) {
+            store_tile(m0);
+            if (m0 + tstep < p.M) load_tile(m0 + tstep);
+        } else {
+            const uint16_t* src = p.A + m0 * p.K;
+            for (int i = threadIdx.x; i < nr * p.K; i += blockDim.x) {
+                const int r = i / p.K, c = i - r * p.K;
+                reinterpret_cast<uint16_t*>(rows_s)[r * RH + pos_s[c]] = __ldg(src + i);
+            }
+        }
+        __syncthreads();
+        if (p.tensor_in_cta) {
+            float f0, f1;
+            staged_group_max(rows_s, RH, pa0, 0, nr, red, f0, f1);
+            if (threadIdx.x < 2) p.s_a[threadIdx.x] = threadIdx.x ? f1 : f0;
+            k0 = make_qconst(f0, p.g[0].bits_a);
+            k1 = make_qconst(f1, p.g[1].bits_a);
+        } else if (per_row) {
+            // max |a| of each staged row and group (the group's channels are contiguous here)
+            const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+            for (int r = warp; r < nr; r += nwarps) {
+                const __half* row = rows_s + r * RH;
+#pragma unroll
+                for (int g = 0; g < 2; ++g) {
+                    const int base = g ? pa0 : 0;
+                    float mx = 0.0f;
+                    for (int j = lane; j < p.g[g].count; j += 32) mx = fmaxf(mx, fabsf(__half2float(row[base + j])));
+                    mx = warp_max(mx);
+                    if (lane == 0) {
+                        scale_s[2 * r + g] = mx;
+                        p.s_a[(m0 + r) * 2 + g] = mx;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+        // ---- quantize: thread per (row, 32-code block) ----
+        const int tasks = nr * p.nblk;
+        int t = threadIdx.x;
+        int r = t / p.nblk, kb = t - r * p.nblk;
+        const int dr = blockDim.x / p.nblk, dk = blockDim.x - dr * p.nblk;
+        for (; t < tasks; t += blockDim.x) {
+            const int g = kb >= p.nblk0;
+            const GroupGeom& G = p.g[g];
+            const int kbg = kb - (g ? p.nblk0 : 0);
+            const QConst k = per_row ? make_qconst(scale_s[2 * r + g], G.bits_a) : (g ? k1 : k0);
+            uint32_t o[8];
+            if (k.mode == 1) {
+                block_codes_fast(rows_a + 2u * (uint32_t)(r * RH + (g ? pa0 : 0) + kbg * 32), k.s, k.r, k.levels,
+                                 k.top, o);
+            } else if (k.mode == 2) {
+                block_codes<false>(rows_s + r * RH + (g ? pa0 : 0) + kbg * 32, G.count - kbg * 32, k, o);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 8; ++q) o[q] = 0u;
+            }
+            store_block32_n(G.bits_a, o, p.Ap + (m0 + r) * (int64_t)p.a_row_bytes + G.a_off + kbg * 4 * G.bits_a);
+            r += dr;
+            kb += dk;
+            if (kb >= p.nblk) {
+                kb -= p.nblk;
+                ++r;
+            }
+        }
+        __syncthreads();   // the tile is overwritten next
+    }
+}
+
 int grid_for(int64_t work_items, int per_cta) {
     int64_t ctas = (work_items + per_cta - 1) / per_cta;
     int64_t cap = (int64_t)num_sms() * 8;
@@ -703,8 +758,8 @@ cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const 
     if (geo.K % 8 == 0 && (uintptr_t)A % 16 == 0) {
         const int KV = geo.K / 8;
         const int rpar = kThreads / (KV < kThreads ? KV : kThreads);
-        // enough CTAs that each thread streams a handful of rows
-        int64_t ctas = (M + 4 * rpar - 1) / (4 * rpar);
+        // enough CTAs that each thread streams a handful of rows (eight loads in flight)
+        int64_t ctas = (M + 8 * rpar - 1) / (8 * rpar);
         const int64_t cap = (int64_t)num_sms() * 8;
         if (ctas > cap) ctas = cap;
         if (ctas < 1) ctas = 1;
@@ -720,10 +775,12 @@ cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const 
     return cudaGetLastError();
 }
 
-cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
-                                int64_t M, int32_t scale_mode, float* s_a, uint8_t* Ap,
-                                cudaStream_t st) {
-    QuantActParams p;
+// Tiled quantize (quantize_tiles_kernel).  tensor_in_cta: one CTA holds every
+// row in one tile and finds the per-tensor scale itself; returns
+// cudaErrorNotSupported when the rows do not fit that way.
+cudaError_t launch_quantize_rows(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
+                                 int32_t scale_mode, bool tensor_in_cta, float* s_a, uint8_t* Ap, cudaStream_t st) {
+    TileQuantParams p;
     p.A = A;
     p.Ap = Ap;
     p.s_a = s_a;
@@ -732,31 +789,48 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
     p.K = geo.K;
     p.a_row_bytes = geo.a_row_bytes;
     p.scale_mode = scale_mode;
+    p.tensor_in_cta = tensor_in_cta ? 1 : 0;
     p.vec_ok = (geo.K % 8 == 0) && ((uintptr_t)A % 16 == 0);
     p.g[0] = geo.g[0];
     p.g[1] = geo.g[1];
     p.nblk0 = geo.g[0].pa / 32;
     p.nblk = p.nblk0 + geo.g[1].pa / 32;
     p.row_halves = geo.g[0].pa + geo.g[1].pa;
-    const int row_bytes = p.row_halves * 2;
-    // about 16 KB of staged rows per CTA, several CTAs per SM
-    int tr = (16 * 1024) / row_bytes;
-    if (tr > 64) tr = 64;
-    if (tr < 1) tr = 1;
-    p.tile_rows = tr;
-    const size_t smem = (size_t)((geo.K * 2 + 15) & ~15) + (size_t)((tr * 8 + 15) & ~15) + (size_t)tr * row_bytes;
-    if (smem > 227 * 1024) return cudaErrorInvalidValue;
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(quantize_act_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
-        if (e != cudaSuccess) return e;
+    if (p.nblk == 0) return cudaErrorNotSupported;
+    const size_t pos_bytes = (size_t)((geo.K * 2 + 15) & ~15);
+    const size_t row_bytes = (size_t)p.row_halves * 2;
+    const size_t budget = 200 * 1024;
+    // rows per tile: what the register prefetch covers (kTilePrefetch vectors per
+    // thread) and shared memory holds
+    const int64_t KV = geo.K / 8 > 0 ? geo.K / 8 : 1;
+    int64_t tr = (int64_t)kTileThreads * kTilePrefetch / KV;
+    const int64_t tr_smem = (int64_t)((budget - pos_bytes - 4096) / row_bytes);
+    if (tr > tr_smem) tr = tr_smem;
+    if (tr > 256) tr = 256;
+    if (!p.vec_ok && tr > 64) tr = 64;
+    if (tensor_in_cta) {
+        // every row in the single CTA's one tile
+        if (M > tr) return cudaErrorNotSupported;
+        tr = M;
     }
-    int64_t ctas = (M + tr - 1) / tr;
-    const int64_t cap = (int64_t)num_sms() * 8;
+    if (tr < 1) return cudaErrorNotSupported;
+    p.tile_rows = (int32_t)tr;
+    const size_t smem = pos_bytes + (size_t)((tr * 8 + 15) & ~15) + (size_t)tr * row_bytes;
+    if (smem > budget) return cudaErrorNotSupported;
+    static int attr_dev = -1;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (attr_dev != dev) {
+        cudaError_t e = cudaFuncSetAttribute(quantize_tiles_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)budget);
+        if (e == cudaSuccess) e = prefer_max_shared((const void*)quantize_tiles_kernel);
+        if (e != cudaSuccess) return e;
+        attr_dev = dev;
+    }
+    int64_t ctas = tensor_in_cta ? 1 : (M + tr - 1) / tr;
+    const int64_t cap = (int64_t)num_sms();
     if (ctas > cap) ctas = cap;
-    cudaError_t ec = prefer_max_shared((const void*)quantize_act_kernel);
-    if (ec != cudaSuccess) return ec;
-    quantize_act_kernel<<<(int)ctas, 256, smem, st>>>(p);
+    quantize_tiles_kernel<<<(int)ctas, kTileThreads, smem, st>>>(p);
     note_launch();
     return cudaGetLastError();
 }

@@ -278,6 +278,12 @@ soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M,
     cudaStream_t s = as_stream(stream);
     const uint16_t* A16 = static_cast<const uint16_t*>(A);
     if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
+        // a small input (up to 16K values): one CTA finds the scale and quantizes, no scratch needed
+        if (M * (int64_t)L->K <= 16384) {
+            cudaError_t e0 = launch_quantize_rows(geo, L->perm, A16, M, scale_mode, true, s_a, Ap, s);
+            if (e0 == cudaSuccess) return SONIQ_OK;
+            if (e0 != cudaErrorNotSupported) return cuda_status(e0);
+        }
         if (scratch != nullptr && scratch_bytes >= (size_t)kQuantScratchBytes) {
             // one pass: barrier words at the start of the scratch, per-CTA maxima after 256 bytes
             unsigned* bar = static_cast<unsigned*>(scratch);
@@ -290,7 +296,7 @@ soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M,
         cudaError_t e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);   // two passes
         if (e != cudaSuccess) return cuda_status(e);
     }
-    return cuda_status(launch_quantize_act(geo, L->perm, A16, M, scale_mode, s_a, Ap, s));
+    return cuda_status(launch_quantize_rows(geo, L->perm, A16, M, scale_mode, false, s_a, Ap, s));
 }
 
 soniq_status soniq_quantize_act_oneshot(const soniq_layout* L, const void* A, int64_t M, float* s_a, uint8_t* Ap,

@@ -57,9 +57,6 @@ cudaError_t prefer_max_shared(const void* func);
 
 cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
                               int64_t M, float* s_out, cudaStream_t st);
-cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
-                                int64_t M, int32_t scale_mode, float* s_a, uint8_t* Ap,
-                                cudaStream_t st);
 // One-pass per-tensor quantize (cooperative launch); its grid barrier (two
 // words, zero between launches) and per-CTA maxima [max_ctas][2] are `bar` and
 // `part`; a barrier wait that runs out ORs `err_bit` into the error word.
@@ -67,6 +64,11 @@ cudaError_t launch_quantize_act(const LayoutGeom& geo, const int32_t* perm, cons
 cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
                                   float* s_a, uint8_t* Ap, cudaStream_t st, unsigned* bar, float* part,
                                   int max_ctas, unsigned err_bit);
+// Tiled quantize-and-pack (per-tensor scale given in s_a, calibrated, or per
+// row); with tensor_in_cta a single CTA holds every row and computes the
+// per-tensor scale itself (cudaErrorNotSupported if M is too large).
+cudaError_t launch_quantize_rows(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
+                                 int32_t scale_mode, bool tensor_in_cta, float* s_a, uint8_t* Ap, cudaStream_t st);
 cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, const float* W,
                                  int32_t N, float* s_out, cudaStream_t st);
 cudaError_t launch_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W,
