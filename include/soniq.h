@@ -110,6 +110,10 @@ enum {
     SONIQ_FLAG_FORCE_MMA = 2u,           /* soniq_mp_gemm: use a tensor-core kernel for any M */
     SONIQ_FLAG_FORCE_FUSED = 4u,         /* tensor-core work takes the fused kernel even when
                                             scratch for the staged path is given */
+    SONIQ_FLAG_FORCE_STAGED = 8u,        /* tensor-core work takes the staged path whenever the
+                                            scratch suffices, however small the problem (without
+                                            it the staged path is used from about 2^30
+                                            multiply-adds) */
     SONIQ_FLAG_TEST_DROP_ARRIVE = 0x100u /* test hook: the tensor-core kernels' operand producer
                                             skips its first arrival (fused) or its first K-stage
                                             (staged), so the consumer's bounded wait runs out and
@@ -134,6 +138,30 @@ typedef struct soniq_conv_desc {
     int32_t stride_h, stride_w;
     int32_t pad_h, pad_w;
 } soniq_conv_desc;
+
+/*
+ * Quantize-in-epilogue: the next layer's activation quantization fused into
+ * this layer's GEMM / convolution epilogue (Sec. 4.1: the CPU back-end fuses
+ * Conv2D + BatchNorm + Quantize so the next layer receives its codes
+ * directly).  The next layer's codes are those soniq_quantize_act computes
+ * with SONIQ_SCALE_CALIBRATED on the fp16 outputs of this call: every output
+ * y is rounded to fp16 first, then u = clip(round_half_even(fp32(y16 / s) *
+ * (2^n - 1)), 0, 2^n - 1) with the next layer's scale s and bits n.
+ *
+ * Convention: this call's output column j is packed position j of the next
+ * layer's activation rows, so N must equal PA_0' + PA_1' of its layout (the
+ * padded row length) and the caller arranges this layer's weight rows once,
+ * offline, in that order: the rows of the next layer's group-0 channels in
+ * its permutation order, zero rows up to PA_0', then its group-1 channels and
+ * zero rows up to PA_1'.  The next layer's permutation is thereby folded into
+ * this layer's output order and needs no gather at run time.  Codes at pad
+ * positions are 0.
+ */
+typedef struct soniq_next_layer {
+    const soniq_layout *layout;  /* the next layer's layout; layout->perm is not read */
+    const float *s_a;            /* device fp32 [2]: its calibrated activation scales */
+    uint8_t *Ap;                 /* device out [M][soniq_packed_row_bytes(layout, 0, 1)], 4-byte aligned */
+} soniq_next_layer;
 
 /* ---- sizes and checks (host only, no CUDA calls) ------------------------ */
 
@@ -268,6 +296,11 @@ SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, co
  *   Wp, s_w    from soniq_pack_weights with the same layout and taps = 1.
  *   Y          device out [M][N], fp16 or bf16 per out_dtype, 16-byte aligned.
  *   acc_dbg    NULL, or device out int32 [2][M][N]: the exact Acc_g.
+ *   next       NULL, or the next layer whose codes the epilogue also writes
+ *              (soniq_next_layer above; out_dtype must be SONIQ_OUT_F16, Y may
+ *              then be NULL).  Needs the staged path: scratch of at least
+ *              soniq_mp_gemm_scratch_bytes(..., flags | SONIQ_FLAG_FORCE_STAGED),
+ *              else SONIQ_ERR_UNSUPPORTED.
  *   Limits (SONIQ_ERR_UNSUPPORTED otherwise): K <= 65536.  The tensor-core
  *   kernel accumulates integer codes in fp32, exact while every partial sum
  *   stays within 2^24; a group whose worst-case sum over its K range could
@@ -278,7 +311,7 @@ SONIQ_API soniq_status soniq_mp_gemm(const soniq_layout *layout, const uint8_t *
                            int32_t scale_mode, int64_t M, const uint8_t *Wp, const float *s_w,
                            int32_t N, void *Y, int32_t out_dtype, int32_t *acc_dbg,
                            uint32_t flags, void *scratch, size_t scratch_bytes,
-                           soniq_stream_t stream);
+                           const soniq_next_layer *next, soniq_stream_t stream);
 
 /* Scratch of soniq_mp_gemm and soniq_mp_conv2d.  With scratch (256-byte
  * aligned) of at least the *_scratch_bytes() size, the tensor-core work takes
@@ -313,12 +346,14 @@ SONIQ_API int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout *layout, int64_
  *   Wp, s_w    soniq_pack_weights of OHWI weights with taps = R*S.
  *   Y          device out NHWC [batch][P][Q][C_out], 16-byte aligned.
  *   acc_dbg    NULL or device out int32 [2][batch*P*Q][C_out].
+ *   next       NULL, or the next layer whose codes the epilogue also writes,
+ *              as for soniq_mp_gemm (C_out = PA_0' + PA_1').
  */
 SONIQ_API soniq_status soniq_mp_conv2d(const soniq_layout *layout, const soniq_conv_desc *cd,
                              const uint8_t *Xp, const float *s_a, int32_t scale_mode,
                              const uint8_t *Wp, const float *s_w, void *Y, int32_t out_dtype,
                              int32_t *acc_dbg, uint32_t flags, void *scratch, size_t scratch_bytes,
-                             soniq_stream_t stream);
+                             const soniq_next_layer *next, soniq_stream_t stream);
 
 /* Scratch bytes soniq_mp_conv2d can use for these arguments (0: none).  Host
  * only; -1 on a bad argument. */

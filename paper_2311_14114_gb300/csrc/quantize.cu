@@ -150,43 +150,6 @@ __global__ void __launch_bounds__(kThreads) act_absmax_kernel(const uint4* __res
     }
 }
 
-// The code of Sec. 3 step 2, t = (a / s) * (2^n - 1) rounded half to even and
-// clipped to [0, 2^n - 1].  The quotient is formed by Markstein's correction
-// step: q0 = a * r, q = q0 + (a - q0 * s) * r with r = RN(1 / s), both
-// products fused; for |a| <= 65504 and s in [2^-60, 2^60] this is the
-// correctly rounded quotient (checked exhaustively over every fp16 a); other
-// scales take the IEEE division.  Rounding to an unsigned integer saturates
-// negative values (and NaN) at 0, which is the clip at 0.
-template <bool FAST>
-__device__ __forceinline__ uint32_t act_code_q(float a, float s, float r, float levels, uint32_t top) {
-    float q;
-    if constexpr (FAST) {
-        const float q0 = a * r;
-        q = fmaf(fmaf(-q0, s, a), r, q0);
-    } else {
-        q = __fdiv_rn(a, s);
-    }
-    return min(__float2uint_rn(__fmul_rn(q, levels)), top);
-}
-
-// Quantizer constants of one (row or tensor, group): scale, its reciprocal,
-// the level count and the largest code.
-struct QConst {
-    float s, r, levels;
-    uint32_t top;
-    int mode;   // 0: every code is 0 (no positive scale); 1: Markstein quotient; 2: IEEE division
-};
-
-__device__ __forceinline__ QConst make_qconst(float s, int n) {
-    QConst q;
-    q.s = s;
-    q.levels = (float)((1 << n) - 1);
-    q.top = (1u << n) - 1u;
-    q.mode = (s >= 0x1p-60f && s <= 0x1p60f) ? 1 : (s > 0.0f ? 2 : 0);
-    q.r = q.mode == 1 ? __frcp_rn(s) : 0.0f;
-    return q;
-}
-
 // Quantizes 8 halves (x) into two words of bytes: byte b of o[i] is code 4i+b.
 template <bool FAST>
 __device__ __forceinline__ void quarter_codes(const uint4 x, int valid, const QConst& k, uint32_t o[2]) {
@@ -234,42 +197,6 @@ struct FusedParams {
     long long timeout_ns;
     GroupGeom g[2];
 };
-
-template <int N>
-__device__ __forceinline__ void store_block32(const uint32_t* o, uint8_t* dst) {
-    uint32_t w[N];
-    bytes_to_block<N>(o, w);
-    if constexpr (N % 4 == 0) {
-        if ((reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
-#pragma unroll
-            for (int q = 0; q < N; q += 4)
-                *reinterpret_cast<uint4*>(dst + 4 * q) = make_uint4(w[q], w[q + 1], w[q + 2], w[q + 3]);
-            return;
-        }
-    }
-    if constexpr (N % 2 == 0) {
-        if ((reinterpret_cast<uintptr_t>(dst) & 7u) == 0) {
-#pragma unroll
-            for (int q = 0; q < N; q += 2) *reinterpret_cast<uint2*>(dst + 4 * q) = make_uint2(w[q], w[q + 1]);
-            return;
-        }
-    }
-#pragma unroll
-    for (int q = 0; q < N; ++q) reinterpret_cast<uint32_t*>(dst)[q] = w[q];
-}
-
-__device__ __forceinline__ void store_block32_n(int n, const uint32_t* o, uint8_t* dst) {
-    switch (n) {
-        case 1: store_block32<1>(o, dst); break;
-        case 2: store_block32<2>(o, dst); break;
-        case 3: store_block32<3>(o, dst); break;
-        case 4: store_block32<4>(o, dst); break;
-        case 5: store_block32<5>(o, dst); break;
-        case 6: store_block32<6>(o, dst); break;
-        case 7: store_block32<7>(o, dst); break;
-        default: store_block32<8>(o, dst); break;
-    }
-}
 
 __device__ __forceinline__ uint4 lds128q(uint32_t addr) {
     uint4 v;

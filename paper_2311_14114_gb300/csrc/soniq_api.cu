@@ -160,6 +160,15 @@ namespace {
 
 cudaStream_t as_stream(soniq_stream_t s) { return reinterpret_cast<cudaStream_t>(s); }
 
+// The staged path pays for its expansion passes and a persistent launch; below
+// about 2^30 multiply-adds the fused kernel is faster (measured: a 64 x 512 x
+// 512 layer 37 vs 17 us, decode M = 16 x 11008 x 4096 62 vs 41.5 us), unless
+// the call needs an epilogue only the staged kernel has.
+bool staged_worthwhile(const LayoutGeom& geo, int64_t M, int64_t N, uint32_t flags) {
+    if (flags & SONIQ_FLAG_FORCE_STAGED) return true;
+    return (double)M * (double)N * (double)geo.K * (double)geo.taps >= 1073741824.0;
+}
+
 // The kernel soniq_mp_gemm runs: a SONIQ_PATH_* value, -1 when the
 // tensor-core kernel would be chosen but cannot take the layout (mma_check
 // says why), -2 when the GEMV was forced but cannot take the shape.
@@ -170,12 +179,23 @@ int gemm_path(const LayoutGeom& geo, int64_t M, int32_t N, uint32_t flags, size_
         (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= SONIQ_GEMV_MAX_M && !(flags & SONIQ_FLAG_FORCE_MMA));
     if (want_gemv && gemv_supported(geo, M, N)) return SONIQ_PATH_GEMV;
     if (flags & SONIQ_FLAG_FORCE_GEMV) return -2;
-    if (!(flags & SONIQ_FLAG_FORCE_FUSED)) {
+    if (!(flags & SONIQ_FLAG_FORCE_FUSED) && staged_worthwhile(geo, M, N, flags)) {
         const int64_t need = staged_scratch_bytes(geo, M, N);
         if (need > 0 && (int64_t)scratch_bytes >= need) return SONIQ_PATH_TENSOR_STAGED;
     }
     if (mma_check(geo) != SONIQ_OK) return -1;
     return SONIQ_PATH_TENSOR;
+}
+
+// Checks a quantize-in-epilogue descriptor against this call's output width N.
+soniq_status check_next(const soniq_next_layer* next, int64_t N, int32_t out_dtype, LayoutGeom* geo_next) {
+    if (next->layout == nullptr || next->s_a == nullptr || next->Ap == nullptr) return SONIQ_ERR_INVALID_ARG;
+    soniq_status st = make_geom(next->layout, 1, geo_next);
+    if (st != SONIQ_OK) return st;
+    if (out_dtype != SONIQ_OUT_F16) return SONIQ_ERR_INVALID_ARG;   // the next layer reads fp16 activations
+    if ((int64_t)geo_next->g[0].pa + geo_next->g[1].pa != N) return SONIQ_ERR_INVALID_ARG;
+    if (!aligned(next->s_a, 4) || !aligned(next->Ap, 4)) return SONIQ_ERR_ALIGNMENT;
+    return SONIQ_OK;
 }
 
 int64_t conv_rows(const soniq_conv_desc* cd) {
@@ -321,7 +341,7 @@ soniq_status soniq_quantize_act_oneshot(const soniq_layout* L, const void* A, in
 soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float* s_a, int32_t scale_mode,
                            int64_t M, const uint8_t* Wp, const float* s_w, int32_t N, void* Y,
                            int32_t out_dtype, int32_t* acc_dbg, uint32_t flags, void* scratch,
-                           size_t scratch_bytes, soniq_stream_t stream) {
+                           size_t scratch_bytes, const soniq_next_layer* next, soniq_stream_t stream) {
     LayoutGeom geo;
     soniq_status st = make_geom(L, 1, &geo);
     if (st != SONIQ_OK) return st;
@@ -329,8 +349,11 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     if ((st = check_scale_mode_act(scale_mode)) != SONIQ_OK) return st;
     if (out_dtype != SONIQ_OUT_F16 && out_dtype != SONIQ_OUT_BF16) return SONIQ_ERR_INVALID_ARG;
     if ((flags & SONIQ_FLAG_FORCE_GEMV) && (flags & SONIQ_FLAG_FORCE_MMA)) return SONIQ_ERR_INVALID_ARG;
+    if ((flags & SONIQ_FLAG_FORCE_FUSED) && (flags & SONIQ_FLAG_FORCE_STAGED)) return SONIQ_ERR_INVALID_ARG;
+    LayoutGeom geo_next;
+    if (next != nullptr && (st = check_next(next, N, out_dtype, &geo_next)) != SONIQ_OK) return st;
     if (M == 0 || N == 0) return SONIQ_OK;
-    if (Ap == nullptr || s_a == nullptr || Wp == nullptr || s_w == nullptr || Y == nullptr)
+    if (Ap == nullptr || s_a == nullptr || Wp == nullptr || s_w == nullptr || (Y == nullptr && next == nullptr))
         return SONIQ_ERR_INVALID_ARG;
     if (!aligned(Ap, 4) || !aligned(Wp, 16) || !aligned(Y, 16) || !aligned(s_a, 4) || !aligned(s_w, 4) ||
         (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
@@ -338,7 +361,9 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     // K <= 65536 keeps |Acc| < 2^31 and the GEMV's unsigned offset sums below 2^32
     const int per_row = scale_mode == SONIQ_SCALE_PER_ROW;
     cudaStream_t s = as_stream(stream);
+    if (next != nullptr) flags = (flags & ~(uint32_t)SONIQ_FLAG_FORCE_GEMV) | SONIQ_FLAG_FORCE_MMA | SONIQ_FLAG_FORCE_STAGED;
     const int path = gemm_path(geo, M, N, flags, scratch != nullptr ? scratch_bytes : 0);
+    if (next != nullptr && path != SONIQ_PATH_TENSOR_STAGED) return SONIQ_ERR_UNSUPPORTED;
     if (path < 0) return path == -2 ? SONIQ_ERR_UNSUPPORTED : mma_check(geo);
     if (path == SONIQ_PATH_GEMV) {
         GemvArgs a{Ap, Wp, s_a, s_w, Y, acc_dbg, (int32_t)M, N, per_row, out_dtype == SONIQ_OUT_BF16};
@@ -358,6 +383,11 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     a.out_bf16 = out_dtype == SONIQ_OUT_BF16;
     a.flags = flags;
     a.conv = 0;
+    if (next != nullptr) {
+        a.next = &geo_next;
+        a.next_s_a = next->s_a;
+        a.next_Ap = next->Ap;
+    }
     if (path == SONIQ_PATH_TENSOR_STAGED) return cuda_status(launch_staged(geo, a, scratch, scratch_bytes, s));
     return cuda_status(launch_mma(geo, a, s));
 }
@@ -365,7 +395,8 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
 soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, const uint8_t* Xp,
                              const float* s_a, int32_t scale_mode, const uint8_t* Wp, const float* s_w,
                              void* Y, int32_t out_dtype, int32_t* acc_dbg, uint32_t flags,
-                             void* scratch, size_t scratch_bytes, soniq_stream_t stream) {
+                             void* scratch, size_t scratch_bytes, const soniq_next_layer* next,
+                             soniq_stream_t stream) {
     if (cd == nullptr) return SONIQ_ERR_INVALID_ARG;
     if (cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->pad_h < 0 || cd->pad_w < 0 ||
         cd->batch < 0 || cd->H < 1 || cd->W < 1 || cd->C_out < 0)
@@ -380,16 +411,20 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
     if (cd->H + 2 * cd->pad_h < cd->R || cd->W + 2 * cd->pad_w < cd->S || P < 1 || Q < 1)
         return SONIQ_ERR_INVALID_ARG;
     const int64_t M = (int64_t)cd->batch * P * Q;
+    LayoutGeom geo_next;
+    if (next != nullptr && (st = check_next(next, cd->C_out, out_dtype, &geo_next)) != SONIQ_OK) return st;
+    if (next != nullptr) flags |= SONIQ_FLAG_FORCE_STAGED;
     if (M == 0 || cd->C_out == 0) return SONIQ_OK;
-    if (Xp == nullptr || s_a == nullptr || Wp == nullptr || s_w == nullptr || Y == nullptr)
+    if (Xp == nullptr || s_a == nullptr || Wp == nullptr || s_w == nullptr || (Y == nullptr && next == nullptr))
         return SONIQ_ERR_INVALID_ARG;
     if (!aligned(Xp, 4) || !aligned(Wp, 16) || !aligned(Y, 16) || !aligned(s_a, 4) || !aligned(s_w, 4) ||
         (acc_dbg != nullptr && !aligned(acc_dbg, 4)))
         return SONIQ_ERR_ALIGNMENT;
     const bool staged = !(flags & SONIQ_FLAG_FORCE_FUSED) && scratch != nullptr &&
-                        staged_scratch_bytes(geo, M, cd->C_out) > 0 &&
+                        staged_worthwhile(geo, M, cd->C_out, flags) && staged_scratch_bytes(geo, M, cd->C_out) > 0 &&
                         (int64_t)scratch_bytes >= staged_scratch_bytes(geo, M, cd->C_out);
     if (staged && !aligned(scratch, 256)) return SONIQ_ERR_ALIGNMENT;
+    if (next != nullptr && !staged) return SONIQ_ERR_UNSUPPORTED;
     if (!staged && (st = mma_check(geo)) != SONIQ_OK) return st;
     MmaArgs a{};
     a.Ap = Xp;
@@ -414,6 +449,11 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
     a.sw = cd->stride_w;
     a.ph = cd->pad_h;
     a.pw = cd->pad_w;
+    if (next != nullptr) {
+        a.next = &geo_next;
+        a.next_s_a = next->s_a;
+        a.next_Ap = next->Ap;
+    }
     if (staged) return cuda_status(launch_staged(geo, a, scratch, scratch_bytes, as_stream(stream)));
     return cuda_status(launch_mma(geo, a, as_stream(stream)));
 }
@@ -434,7 +474,7 @@ int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout* L, int64_t M, int32_t N,
     const bool want_gemv =
         (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= SONIQ_GEMV_MAX_M && !(flags & SONIQ_FLAG_FORCE_MMA));
     if (want_gemv) return 0;
-    return staged_scratch_bytes(geo, M, N);
+    return staged_worthwhile(geo, M, N, flags) ? staged_scratch_bytes(geo, M, N) : 0;
 }
 
 int64_t soniq_mp_conv2d_scratch_bytes(const soniq_layout* L, const soniq_conv_desc* cd, uint32_t flags) {
@@ -443,7 +483,7 @@ int64_t soniq_mp_conv2d_scratch_bytes(const soniq_layout* L, const soniq_conv_de
         cd->C_out < 0 || make_geom(L, cd->R * cd->S, &geo) != SONIQ_OK)
         return -1;
     if (cd->H + 2 * cd->pad_h < cd->R || cd->W + 2 * cd->pad_w < cd->S) return -1;
-    if (flags & SONIQ_FLAG_FORCE_FUSED) return 0;
+    if (flags & SONIQ_FLAG_FORCE_FUSED || !staged_worthwhile(geo, conv_rows(cd), cd->C_out, flags)) return 0;
     return staged_scratch_bytes(geo, conv_rows(cd), cd->C_out);
 }
 

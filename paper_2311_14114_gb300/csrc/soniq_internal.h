@@ -106,6 +106,10 @@ struct MmaArgs {
     // convolution geometry; conv = 0 for a plain GEMM
     int32_t conv;
     int32_t H, W, P, Q, R, S, sh, sw, ph, pw;
+    // quantize-in-epilogue (staged path only): the next layer's geometry, scales and codes
+    const LayoutGeom* next;
+    const float* next_s_a;
+    uint8_t* next_Ap;
 };
 // Host-side planning of the tensor-core kernel (exactness segments etc.).
 soniq_status mma_check(const LayoutGeom& geo);

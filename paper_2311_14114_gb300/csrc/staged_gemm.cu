@@ -115,6 +115,14 @@ struct SParams {
     int32_t seg_group;     // group accumulated in drained segments, or -1
     int32_t drop_first;    // test hook: the producer never issues the first K-stage
     int32_t y_tma;         // 1: outputs leave through shared memory and TMA stores
+    int32_t write_y;       // 0: Y is not written (only the next layer's codes)
+    // quantize-in-epilogue: output column j is packed position j of the next layer
+    int32_t has_next;
+    const float* s_next;   // the next layer's calibrated activation scales [2]
+    uint8_t* Ap_next;      // its packed activation rows
+    int32_t next_row_bytes;
+    int32_t next_pa0;      // first packed position of its group 1
+    int32_t next_count[2], next_bits[2], next_off[2];
     SGroup g[2];
 };
 
@@ -531,6 +539,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     if (lane == 0) bulk_wait_read0();
                     __syncwarp();
                 }
+                QConst kn0, kn1;              // the next layer's quantizers
+                if (p.has_next) {
+                    kn0 = make_qconst(__ldg(p.s_next), p.next_bits[0]);
+                    kn1 = make_qconst(__ldg(p.s_next + 1), p.next_bits[1]);
+                }
+                uint32_t nq[8];               // the next layer's codes of the current 32-column block
 #pragma unroll
                 for (int cc = 0; cc < EPI_COLS / 8; ++cc) {
                     uint32_t v[8];
@@ -553,7 +567,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                             p.acc_dbg[(p.M + m) * p.N + nb + q] = a1;
                         }
                     }
-                    if (p.y_tma) {
+                    if (p.has_next) {
+                        // quantize fp16(y) for the next layer (Sec. 3 step 2 with its calibrated
+                        // scale), 8 codes of the block whose 32 columns end at chunk cc | 3
+                        const int cb = (nc0 + (cc & ~3) * 8);             // first column of the block
+                        const int gn = cb >= p.next_pa0;
+                        const int jg = cb - (gn ? p.next_pa0 : 0);        // position within the group
+                        const QConst& kn = gn ? kn1 : kn0;
+                        const int cnt = gn ? p.next_count[1] : p.next_count[0];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            uint32_t word = 0u;
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const int q = 4 * h + e;
+                                const float a = __half2float(__float2half_rn(y[q]));
+                                uint32_t u = 0u;
+                                if (jg + (cc & 3) * 8 + q < cnt && kn.mode != 0)
+                                    u = kn.mode == 1 ? act_code_q<true>(a, kn.s, kn.r, kn.levels, kn.top)
+                                                     : act_code_q<false>(a, kn.s, kn.r, kn.levels, kn.top);
+                                word |= u << (8 * e);
+                            }
+                            nq[2 * (cc & 3) + h] = word;
+                        }
+                        if ((cc & 3) == 3 && m < p.M && cb < p.N) {
+                            const int nb = gn ? p.next_bits[1] : p.next_bits[0];
+                            store_block32_n(nb, nq, p.Ap_next + m * (int64_t)p.next_row_bytes +
+                                                        (gn ? p.next_off[1] : p.next_off[0]) + (jg >> 5) * 4 * nb);
+                        }
+                    }
+                    if (!p.write_y) {
+                        // no fp16/bf16 outputs requested
+                    } else if (p.y_tma) {
                         uint32_t w[4];
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
@@ -581,7 +626,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 __syncwarp();
                 if (lane == 0) {
                     mbar_arrive(bar(BAR_REG_EMPTY + r));
-                    if (p.y_tma) {
+                    if (p.y_tma && p.write_y) {
                         // rows and columns beyond M and N are clipped by the store
 #pragma unroll
                         for (int bx = 0; bx < EPI_COLS / 64; ++bx)
@@ -769,9 +814,22 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     p.out_bf16 = a.out_bf16;
     p.seg_group = sp.seg_group;
     p.drop_first = (a.flags & SONIQ_FLAG_TEST_DROP_ARRIVE) != 0 ? 1 : 0;
+    p.write_y = a.Y != nullptr;
+    if (a.next != nullptr) {
+        p.has_next = 1;
+        p.s_next = a.next_s_a;
+        p.Ap_next = a.next_Ap;
+        p.next_row_bytes = a.next->a_row_bytes;
+        p.next_pa0 = a.next->g[0].pa;
+        for (int g = 0; g < 2; ++g) {
+            p.next_count[g] = a.next->g[g].count;
+            p.next_bits[g] = a.next->g[g].bits_a;
+            p.next_off[g] = a.next->g[g].a_off;
+        }
+    }
     // outputs through TMA stores when the row pitch allows a tensor map (N * 2 bytes a multiple of 16)
     p.y_tma = 0;
-    if (a.N % 8 == 0 && (uintptr_t)a.Y % 16 == 0) {
+    if (p.write_y && a.N % 8 == 0 && (uintptr_t)a.Y % 16 == 0) {
         cuuint64_t dims[2] = {(cuuint64_t)a.N, (cuuint64_t)a.M};
         cuuint64_t strides[1] = {(cuuint64_t)a.N * 2};
         cuuint32_t box[2] = {64u, 32u};

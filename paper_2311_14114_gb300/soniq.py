@@ -22,7 +22,7 @@ STATUS_NAMES = {0: "SONIQ_OK", 1: "SONIQ_ERR_INVALID_ARG", 2: "SONIQ_ERR_UNSUPPO
                 3: "SONIQ_ERR_ALIGNMENT", 4: "SONIQ_ERR_CUDA", 5: "SONIQ_ERR_TIMEOUT"}
 SCALE_PER_TENSOR, SCALE_PER_ROW, SCALE_CALIBRATED = 0, 1, 2
 OUT_F16, OUT_BF16 = 0, 1
-FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_FORCE_FUSED, FLAG_TEST_DROP_ARRIVE = 1, 2, 4, 0x100
+FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_FORCE_FUSED, FLAG_FORCE_STAGED, FLAG_TEST_DROP_ARRIVE = 1, 2, 4, 8, 0x100
 PATH_NAMES = {0: "CUDA-core GEMV", 1: "tensor-core fused kernel", 2: "tensor-core staged (expand + GEMM)"}
 
 EXPORTED = ["soniq_abi_version", "soniq_status_string", "soniq_group_codes",
@@ -46,6 +46,10 @@ class CLayout(ctypes.Structure):
                 ("count", ctypes.c_int32 * 2), ("bits_w", ctypes.c_int32 * 2),
                 ("bits_a", ctypes.c_int32 * 2), ("perm", ctypes.c_void_p),
                 ("pad_unit", ctypes.c_int32)]
+
+
+class CNextLayer(ctypes.Structure):
+    _fields_ = [("layout", ctypes.c_void_p), ("s_a", ctypes.c_void_p), ("Ap", ctypes.c_void_p)]
 
 
 class CConvDesc(ctypes.Structure):
@@ -84,13 +88,13 @@ def lib() -> ctypes.CDLL:
         L.soniq_quantize_act_scratch_bytes.restype = i64
         L.soniq_quantize_act_oneshot.argtypes = [P, P, i64, P, P, P]
         L.soniq_quantize_act_oneshot.restype = i32
-        L.soniq_mp_gemm.argtypes = [P, P, P, i32, i64, P, P, i32, P, i32, P, u32, P, ctypes.c_size_t, P]
+        L.soniq_mp_gemm.argtypes = [P, P, P, i32, i64, P, P, i32, P, i32, P, u32, P, ctypes.c_size_t, P, P]
         L.soniq_mp_gemm.restype = i32
         L.soniq_mp_gemm_path.argtypes = [P, i64, i32, u32, ctypes.c_size_t]
         L.soniq_mp_gemm_path.restype = i32
         L.soniq_mp_gemm_scratch_bytes.argtypes = [P, i64, i32, u32]
         L.soniq_mp_gemm_scratch_bytes.restype = i64
-        L.soniq_mp_conv2d.argtypes = [P, P, P, P, i32, P, P, P, i32, P, u32, P, ctypes.c_size_t, P]
+        L.soniq_mp_conv2d.argtypes = [P, P, P, P, i32, P, P, P, i32, P, u32, P, ctypes.c_size_t, P, P]
         L.soniq_mp_conv2d.restype = i32
         L.soniq_mp_conv2d_scratch_bytes.argtypes = [P, P, u32]
         L.soniq_mp_conv2d_scratch_bytes.restype = i64
@@ -175,6 +179,7 @@ class Layout:
         _check(lib().soniq_validate_layout(ctypes.byref(host),
                                            perm_t.numpy().ctypes.data_as(ctypes.c_void_p)),
                "soniq_validate_layout")
+        self.perm_host = perm_t.numpy().copy()
         self.perm = perm_t.to(device if device is not None else "cuda")
         host.perm = ctypes.c_void_p(self.perm.data_ptr())
         self.c = host
@@ -187,6 +192,34 @@ class Layout:
 
     def group_codes(self, g: int, is_weight: bool = False, taps: int = 1) -> int:
         return int(lib().soniq_group_codes(ctypes.byref(self.c), int(g), int(is_weight), int(taps)))
+
+
+def next_layer_row_order(next_layout: Layout):
+    """Row order of a layer whose epilogue quantizes for `next_layout`
+    (soniq_next_layer): entry j is the output channel placed at column j, the
+    next layer's packed position j, or -1 for a padding position (a zero row).
+    Index bookkeeping on the host for the one-time arrangement of weights."""
+    import numpy as np
+    pa0 = next_layout.group_codes(0)
+    pa1 = next_layout.group_codes(1)
+    c0, c1 = next_layout.count
+    order = np.full(pa0 + pa1, -1, dtype=np.int64)
+    order[:c0] = next_layout.perm_host[:c0]
+    order[pa0:pa0 + c1] = next_layout.perm_host[c0:c0 + c1]
+    return order
+
+
+class NextLayer:
+    """The next layer's codes written by a GEMM / conv epilogue (soniq_next_layer)."""
+
+    def __init__(self, layout: Layout, s_a: torch.Tensor, Ap: Optional[torch.Tensor] = None, M: Optional[int] = None):
+        _need(s_a, torch.float32, "s_a")
+        self.layout = layout
+        self.s_a = s_a
+        if Ap is None:
+            Ap = torch.empty((M, layout.row_bytes(False)), dtype=torch.uint8, device=s_a.device)
+        self.Ap = Ap
+        self.c = CNextLayer(ctypes.cast(ctypes.byref(layout.c), ctypes.c_void_p), s_a.data_ptr(), Ap.data_ptr())
 
 
 def pack_weights(layout: Layout, W: torch.Tensor, scale_mode: str = "row",
@@ -250,17 +283,23 @@ def quantize_act_oneshot(layout: Layout, A: torch.Tensor, s_a: Optional[torch.Te
 def mp_gemm(layout: Layout, Ap: torch.Tensor, s_a: torch.Tensor, Wp: torch.Tensor,
             s_w: torch.Tensor, scale_mode: str = "tensor", out_dtype=torch.float16,
             Y: Optional[torch.Tensor] = None, acc_dbg: Optional[torch.Tensor] = None,
-            flags: int = 0, stream=None) -> torch.Tensor:
-    """soniq_mp_gemm: Y[M][N] = dequantized (A W^T) from packed codes."""
+            flags: int = 0, stream=None, next: Optional[NextLayer] = None,
+            write_y: bool = True) -> torch.Tensor:
+    """soniq_mp_gemm: Y[M][N] = dequantized (A W^T) from packed codes; with
+    `next`, the epilogue also writes the next layer's packed codes (next.Ap)."""
     M, N = Ap.shape[0], Wp.shape[0]
-    if Y is None:
+    if Y is None and write_y:
         Y = torch.empty((M, N), dtype=out_dtype, device=Ap.device)
-    od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
-    need = int(lib().soniq_mp_gemm_scratch_bytes(ctypes.byref(layout.c), M, N, int(flags)))
+    od = OUT_BF16 if (Y is not None and Y.dtype == torch.bfloat16) or (Y is None and out_dtype == torch.bfloat16) \
+        else OUT_F16
+    qflags = int(flags) | (FLAG_FORCE_STAGED if next is not None else 0)
+    need = int(lib().soniq_mp_gemm_scratch_bytes(ctypes.byref(layout.c), M, N, qflags))
     scratch = _get_scratch(need, Ap.device, stream, "gemm")
     _check(lib().soniq_mp_gemm(ctypes.byref(layout.c), _ptr(Ap), _ptr(s_a), _SCALE[scale_mode], M,
                                _ptr(Wp), _ptr(s_w), N, _ptr(Y), od, _ptr(acc_dbg), int(flags),
-                               _ptr(scratch), max(need, 0), _stream(stream)), "soniq_mp_gemm")
+                               _ptr(scratch), max(need, 0),
+                               ctypes.byref(next.c) if next is not None else None, _stream(stream)),
+           "soniq_mp_gemm")
     return Y
 
 
@@ -286,17 +325,22 @@ def conv_out_hw(cd: CConvDesc) -> Tuple[int, int]:
 def mp_conv2d(layout: Layout, cd: CConvDesc, Xp: torch.Tensor, s_a: torch.Tensor,
               Wp: torch.Tensor, s_w: torch.Tensor, scale_mode: str = "tensor",
               out_dtype=torch.float16, Y: Optional[torch.Tensor] = None,
-              acc_dbg: Optional[torch.Tensor] = None, flags: int = 0, stream=None) -> torch.Tensor:
-    """soniq_mp_conv2d: NHWC implicit-GEMM convolution from packed codes."""
+              acc_dbg: Optional[torch.Tensor] = None, flags: int = 0, stream=None,
+              next: Optional[NextLayer] = None, write_y: bool = True) -> torch.Tensor:
+    """soniq_mp_conv2d: NHWC implicit-GEMM convolution from packed codes; with
+    `next`, the epilogue also writes the next layer's packed codes."""
     P, Q = conv_out_hw(cd)
-    if Y is None:
+    if Y is None and write_y:
         Y = torch.empty((cd.batch, P, Q, cd.C_out), dtype=out_dtype, device=Xp.device)
-    od = OUT_BF16 if Y.dtype == torch.bfloat16 else OUT_F16
-    need = int(lib().soniq_mp_conv2d_scratch_bytes(ctypes.byref(layout.c), ctypes.byref(cd), int(flags)))
+    od = OUT_BF16 if (Y is not None and Y.dtype == torch.bfloat16) or (Y is None and out_dtype == torch.bfloat16) \
+        else OUT_F16
+    qflags = int(flags) | (FLAG_FORCE_STAGED if next is not None else 0)
+    need = int(lib().soniq_mp_conv2d_scratch_bytes(ctypes.byref(layout.c), ctypes.byref(cd), qflags))
     scratch = _get_scratch(need, Xp.device, stream, "gemm")
     _check(lib().soniq_mp_conv2d(ctypes.byref(layout.c), ctypes.byref(cd), _ptr(Xp), _ptr(s_a),
                                  _SCALE[scale_mode], _ptr(Wp), _ptr(s_w), _ptr(Y), od,
                                  _ptr(acc_dbg), int(flags), _ptr(scratch), max(need, 0),
+                                 ctypes.byref(next.c) if next is not None else None,
                                  _stream(stream)), "soniq_mp_conv2d")
     return Y
 

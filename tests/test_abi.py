@@ -98,22 +98,41 @@ def test_host_side_argument_errors_need_no_gpu(L):
     # misaligned scratch
     assert L.soniq_quantize_act(ctypes.byref(lay), fake, 10, 0, fake, fake, ctypes.c_void_p(4100), 9000,
                                 None) == 3
-    assert L.soniq_mp_gemm(ctypes.byref(lay), None, None, 0, 0, None, None, 5, None, 0, None, 0, None, 0, None) == 0
+    assert L.soniq_mp_gemm(ctypes.byref(lay), None, None, 0, 0, None, None, 5, None, 0, None, 0, None, 0, None, None) == 0
     # both dispatch overrides at once
-    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 3, None, 0, None) == 1
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 3, None, 0, None, None) == 1
     # bad output dtype
-    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 9, None, 0, None, 0, None) == 1
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 4, fake, fake, 8, fake, 9, None, 0, None, 0, None, None) == 1
     # conv: per-row activation scales are rejected (a dot product spans pixels)
     cd = soniq.conv_desc(1, 8, 8, 16)
     assert L.soniq_mp_conv2d(ctypes.byref(lay), ctypes.byref(cd), fake, fake, 1, fake, fake, fake, 0,
-                             None, 0, None, 0, None) == 1
+                             None, 0, None, 0, None, None) == 1
     # conv: filter larger than the padded image
     cd = soniq.conv_desc(1, 2, 2, 16, R=5, S=5, pad=(0, 0))
     assert L.soniq_mp_conv2d(ctypes.byref(lay), ctypes.byref(cd), fake, fake, 0, fake, fake, fake, 0,
-                             None, 0, None, 0, None) == 1
+                             None, 0, None, 0, None, None) == 1
     # K beyond the supported range
     big = _layout(soniq, K=70000, count=(70000, 0), bits=(2, 2), perm=ctypes.c_void_p(16))
-    assert L.soniq_mp_gemm(ctypes.byref(big), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 0, None, 0, None) == 2
+    assert L.soniq_mp_gemm(ctypes.byref(big), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 0, None, 0, None, None) == 2
+
+
+def test_next_layer_descriptor_checks(L):
+    """The quantize-in-epilogue descriptor is checked on the host: the output
+    width must be the next layer's padded row length, outputs fp16."""
+    from paper_2311_14114_gb300 import soniq
+    lay = _layout(soniq, perm=ctypes.c_void_p(16))
+    nxt_lay = _layout(soniq, K=40, count=(30, 10), bits=(2, 8), pad=32, perm=ctypes.c_void_p(16))
+    fake = ctypes.c_void_p(4096)
+    nxt = soniq.CNextLayer(ctypes.cast(ctypes.byref(nxt_lay), ctypes.c_void_p).value, 4096, 4096)
+    # N = 64 = 32 + 32 (pad 32) is accepted up to the missing scratch; 8 is not the padded width
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 300, fake, fake, 8, fake, 0, None, 0, None, 0,
+                           ctypes.byref(nxt), None) == 1
+    # bf16 outputs cannot feed the next layer's fp16 quantizer
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 300, fake, fake, 64, fake, 1, None, 0, None, 0,
+                           ctypes.byref(nxt), None) == 1
+    # without staged scratch the fused epilogue is unavailable
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 300, fake, fake, 64, fake, 0, None, 0, None, 0,
+                           ctypes.byref(nxt), None) == 2
 
 
 def test_scratch_size_queries(L):

@@ -67,7 +67,7 @@ def _max_codes(M, N, K, na, nw):
     return U, J
 
 
-PATHS = pytest.mark.parametrize("flags", [2, 2 | 4], ids=["staged", "fused"])
+PATHS = pytest.mark.parametrize("flags", [2 | 8, 2 | 4], ids=["staged", "fused"])
 
 
 @PATHS

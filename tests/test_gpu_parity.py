@@ -173,7 +173,7 @@ GEMM_BITS = [(1, 4), (1, 8), (2, 6), (2, 8), (3, 5), (3, 8), (4, 4), (4, 6), (4,
 
 
 # tensor-core paths: staged (expand into scratch, then GEMM) and fused (expand on chip)
-STAGED, FUSED = 2, 2 | 4
+STAGED, FUSED = 2 | 8, 2 | 4
 
 
 @pytest.mark.parametrize("path", [STAGED, FUSED], ids=["staged", "fused"])
@@ -188,7 +188,9 @@ def test_gemm_small_all_bit_pairs(sq, bits, path):
 def test_gemm_paths_reported(sq):
     d = wl.random_linear(5, M=300, K=333, N=264, bits_lo=2, bits_hi=8, frac_hi=0.3)
     lay = sq.Layout(d["perm"], d["count"], d["bits"])
-    assert sq.gemm_path(lay, 300, 264) == sq.PATH_NAMES[2]
+    assert sq.gemm_path(lay, 300, 264, STAGED) == sq.PATH_NAMES[2]
+    assert sq.gemm_path(lay, 300, 264) == sq.PATH_NAMES[1]          # small: the fused kernel
+    assert sq.gemm_path(lay, 8192, 4096) == sq.PATH_NAMES[2]        # large: staged
     assert sq.gemm_path(lay, 300, 264, FUSED) == sq.PATH_NAMES[1]
     assert sq.gemm_path(lay, 8, 264) == sq.PATH_NAMES[0]
 
@@ -339,7 +341,7 @@ def check_conv(sq, spec, pad_unit=32, pix=None, what="conv", flags=0):
     assert_y_close(g["Y"][sel], r["Y16"], terms, what)
 
 
-@pytest.mark.parametrize("flags", [0, 4], ids=["staged", "fused"])
+@pytest.mark.parametrize("flags", [8, 4], ids=["staged", "fused"])
 @pytest.mark.parametrize("bits", [(4, 8), (1, 4), (2, 6)])
 @pytest.mark.parametrize("geom", [((1, 1), (1, 1)), ((2, 2), (0, 0)), ((1, 2), (1, 0))])
 def test_conv_small(sq, bits, geom, flags):
@@ -386,7 +388,7 @@ def test_full_linear_64x512x512(sq):
     check_linear(sq, d, what="linear 64x512x512")
 
 
-@pytest.mark.parametrize("flags", [0, 4], ids=["staged", "fused"])
+@pytest.mark.parametrize("flags", [8, 4], ids=["staged", "fused"])
 @pytest.mark.parametrize("spec", [wl.CONV_RESNET, wl.CONV_RESNET_1B4B], ids=lambda s: s.name)
 def test_full_conv_resnet(sq, spec, flags):
     pix = _sample_rows(spec.M, 600, 1)
