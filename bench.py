@@ -432,7 +432,48 @@ def run_suite(args, sq, wl, pk, flush, head):
                      "quantize_GBps": round(qb / (qms * 1e-3) / 1e9, 1),
                      "quantize_frac_hbm": round(qb / (qms * 1e-3) / 1e9 / pk["hbm"], 4)})
 
+    def fused_quant_case(spec, bits2, frac2):
+        """The layer's epilogue writing the next layer's packed codes (quantize-in-
+        epilogue) against the unfused pair: fp16 outputs, then soniq_quantize_act
+        with the next layer's calibrated scales."""
+        d = wl.make_linear(spec)
+        perm2, count2, _ = wl.assignment(np.random.default_rng(spec.seed + 1), spec.N, frac2, 0)
+        lay2 = sq.Layout(perm2, count2, bits2)
+        order = sq.next_layer_row_order(lay2)
+        Wa = np.zeros((len(order), spec.K), np.float32)
+        Wa[order >= 0] = d["W"][order[order >= 0]]
+        lay = sq.Layout(d["perm"], d["count"], d["bits"])
+        Wp, s_w = sq.pack_weights(lay, torch.from_numpy(Wa).cuda())
+        A = torch.from_numpy(d["A"]).cuda()
+        Ap, s_a = sq.quantize_act(lay, A)
+        s2 = torch.tensor([0.6, 1.8], dtype=torch.float32, device="cuda")
+        nxt = sq.NextLayer(lay2, s2, M=spec.M)
+        Y = torch.empty((spec.M, len(order)), dtype=torch.float16, device="cuda")
+        X2 = torch.empty((spec.M, spec.N), dtype=torch.float16, device="cuda")
+        Ap2 = torch.empty_like(nxt.Ap)
+        cols = torch.from_numpy(np.flatnonzero(order >= 0)).cuda()
+        chans = torch.from_numpy(order[order >= 0]).cuda()
+
+        def unfused():
+            sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y)
+            X2[:, chans] = Y[:, cols]          # the next layer's input in channel order (not timed below)
+            sq.quantize_act(lay2, X2, "calibrated", s_a=s2, Ap=Ap2)
+
+        gemm_ms = _time_fn(lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y), steps, flush, stream)
+        unfused()
+        q_ms = _time_fn(lambda: sq.quantize_act(lay2, X2, "calibrated", s_a=s2, Ap=Ap2), steps, flush, stream)
+        fused_ms = _time_fn(lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y, next=nxt), steps, flush, stream)
+        codes_ms = _time_fn(lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, next=nxt, write_y=False), steps, flush,
+                            stream)
+        same = bool(torch.equal(nxt.Ap, Ap2))
+        rows.append({"workload": spec.name + "_then_next_layer_quantize", "M": spec.M, "N": len(order),
+                     "K": spec.K, "bits": d["bits"], "next_bits": bits2, "next_count": count2,
+                     "gemm_us": round(gemm_ms * 1e3, 2), "separate_quantize_us": round(q_ms * 1e3, 2),
+                     "unfused_us": round((gemm_ms + q_ms) * 1e3, 2), "fused_us": round(fused_ms * 1e3, 2),
+                     "fused_codes_only_us": round(codes_ms * 1e3, 2), "codes_identical": same})
+
     linear_case(wl.LINEAR_SMALL)
+    fused_quant_case(wl.MLP_UP, [2, 8], 0.2)
     conv_case(wl.CONV_RESNET)
     conv_case(wl.CONV_RESNET_1B4B)
     linear_case(wl.MLP_UP)
