@@ -326,7 +326,10 @@ __device__ __forceinline__ void store_out16(const SParams& p, int64_t m, int nb,
 // epilogue drains one region while the MMAs fill the other.
 __device__ __forceinline__ int first_group(const SParams& p) { return p.seg_group == 1 ? 1 : 0; }
 
-template <bool DBG>
+// GENERAL = false: the common case compiled lean (no debug accumulators, no
+// next-layer codes, outputs through TMA stores), which keeps the unrolled
+// epilogue small enough for the instruction cache; GENERAL = true handles the rest.
+template <bool GENERAL>
 __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid_constant__ SParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -533,14 +536,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 }
                 // the final job: finish the tile's outputs, 8 columns at a time
                 const float sc = p.g[g_last].acc_scale;
-                const bool dbg = DBG && m < p.M;
-                if (p.y_tma) {
+                const bool dbg = GENERAL && p.acc_dbg != nullptr && m < p.M;
+                const bool has_next = GENERAL && p.has_next;
+                const bool y_tma = GENERAL ? p.y_tma != 0 : true;
+                const bool write_y = GENERAL ? p.write_y != 0 : true;
+                if (y_tma) {
                     // the previous tile's store must have read the staging buffer
                     if (lane == 0) bulk_wait_read0();
                     __syncwarp();
                 }
                 QConst kn0, kn1;              // the next layer's quantizers
-                if (p.has_next) {
+                if (has_next) {
                     kn0 = make_qconst(__ldg(p.s_next), p.next_bits[0]);
                     kn1 = make_qconst(__ldg(p.s_next + 1), p.next_bits[1]);
                 }
@@ -567,7 +573,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                             p.acc_dbg[(p.M + m) * p.N + nb + q] = a1;
                         }
                     }
-                    if (p.has_next) {
+                    if (has_next) {
                         // quantize fp16(y) for the next layer (Sec. 3 step 2 with its calibrated
                         // scale), 8 codes of the block whose 32 columns end at chunk cc | 3
                         const int cb = (nc0 + (cc & ~3) * 8);             // first column of the block
@@ -596,9 +602,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                                                         (gn ? p.next_off[1] : p.next_off[0]) + (jg >> 5) * 4 * nb);
                         }
                     }
-                    if (!p.write_y) {
+                    if (!write_y) {
                         // no fp16/bf16 outputs requested
-                    } else if (p.y_tma) {
+                    } else if (y_tma) {
                         uint32_t w[4];
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
@@ -622,11 +628,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     }
                 }
                 tc_fence_before();
-                if (p.y_tma) fence_proxy_async_shared();
+                if (y_tma) fence_proxy_async_shared();
                 __syncwarp();
                 if (lane == 0) {
                     mbar_arrive(bar(BAR_REG_EMPTY + r));
-                    if (p.y_tma && p.write_y) {
+                    if (y_tma && write_y) {
                         // rows and columns beyond M and N are clipped by the store
 #pragma unroll
                         for (int bx = 0; bx < EPI_COLS / 64; ++bx)
@@ -636,7 +642,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 }
             }
         }
-        if (p.y_tma && lane == 0) bulk_wait0();   // stores complete before the CTA exits
+        if ((GENERAL ? p.y_tma && p.write_y : true) && lane == 0) bulk_wait0();   // stores complete before the CTA exits
     }
 
     tc_fence_before();
@@ -864,7 +870,7 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         attr_done[dev] = true;
     }
     const int grid = p.total_tiles < num_sms() ? p.total_tiles : num_sms();
-    if (a.acc_dbg != nullptr) {
+    if (a.acc_dbg != nullptr || p.has_next || !p.y_tma || !p.write_y) {
         if ((err = prefer_max_shared((const void*)staged_mma_kernel<true>)) != cudaSuccess) return err;
         staged_mma_kernel<true><<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
     } else {
