@@ -143,6 +143,8 @@ struct ExpandParams {
     // channel block kb % cpt[g] of the input pixel that tap reads
     int32_t conv, H, W, P, Q, R, S, sh, sw, ph, pw;
     int32_t cpt[2];
+    uint64_t cpt_magic[2];     // ceil(2^32 / cpt): tap = (kb * magic) >> 32, exact for kb < 2^32 / cpt
+    int32_t vec16[2];          // source blocks of the group can be read as 16-byte vectors
 };
 
 // n-bit two's-complement patterns in the bytes of x -> E4M3 sign-magnitude bytes.
@@ -153,9 +155,31 @@ __device__ __forceinline__ uint32_t twos_to_e4m3(uint32_t x) {
     return (x & ~neg) | ((mag | 0x80808080u) & neg);
 }
 
+// This block's N packed words from src (16-byte loads when the group allows).
+template <int N>
+__device__ __forceinline__ void load_block_words(const uint8_t* src, bool vec16, uint32_t (&words)[N]) {
+    if constexpr (N % 4 == 0) {
+        if (vec16) {
+#pragma unroll
+            for (int i = 0; i < N; i += 4) {
+                const uint4 v = __ldg(reinterpret_cast<const uint4*>(src) + i / 4);
+                words[i] = v.x;
+                words[i + 1] = v.y;
+                words[i + 2] = v.z;
+                words[i + 3] = v.w;
+            }
+            return;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < N; ++i) words[i] = __ldg(reinterpret_cast<const uint32_t*>(src) + i);
+}
+
 template <int N>
 __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int g, int lane) {
     const int kind = p.kind[g];
+    const bool vec16 = p.vec16[g] != 0;
+    const uint64_t magic = p.cpt_magic[g];
     uint8_t* drow = p.dst + r * p.dst_row_bytes + p.dst_off[g];
     int64_t img = 0;
     int hp = 0, wq = 0;
@@ -176,7 +200,7 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
         if (!p.conv) {
             if (kb < p.blk_src[g]) src = p.src + r * p.src_row_bytes + p.src_off[g] + kb * 4 * N;
         } else {
-            const int tap = kb / p.cpt[g];
+            const int tap = (int)(((uint64_t)kb * magic) >> 32);
             const int cb = kb - tap * p.cpt[g];
             if (tap < p.R * p.S) {
                 const int rr = tap / p.S, ss = tap - rr * p.S;
@@ -186,8 +210,12 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
             }
         }
         uint32_t words[N];
+        if (src != nullptr) {
+            load_block_words<N>(src, vec16, words);
+        } else {
 #pragma unroll
-        for (int i = 0; i < N; ++i) words[i] = src ? __ldg(reinterpret_cast<const uint32_t*>(src) + i) : 0u;
+            for (int i = 0; i < N; ++i) words[i] = 0u;
+        }
         uint32_t o[8];
         block_to_bytes<N>(words, o);
         if (kind == 0) {
@@ -223,7 +251,7 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
     }
 }
 
-__global__ void __launch_bounds__(256) expand_kernel(const ExpandParams p) {
+__global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ ExpandParams p) {
     const int lane = threadIdx.x & 31;
     const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -757,6 +785,8 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         e.blk_dst[g] = G.pw / 32;
         e.center[g] = sp.g[g].center;
         e.cpt[g] = G.pa / 32 > 0 ? G.pa / 32 : 1;
+        e.cpt_magic[g] = (((uint64_t)1 << 32) + (uint64_t)e.cpt[g] - 1) / (uint64_t)e.cpt[g];
+        e.vec16[g] = (G.a_off % 16 == 0 && geo.a_row_bytes % 16 == 0 && (uintptr_t)a.Ap % 16 == 0) ? 1 : 0;
     }
     e.src = a.Ap;
     e.src_row_bytes = geo.a_row_bytes;
@@ -785,6 +815,7 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         w.src_off[g] = G.w_off;
         w.blk_src[g] = G.pw / 32;
         w.center[g] = 0;
+        w.vec16[g] = (G.w_off % 16 == 0 && geo.w_row_bytes % 16 == 0 && (uintptr_t)a.Wp % 16 == 0) ? 1 : 0;
     }
     w.src = a.Wp;
     w.src_row_bytes = geo.w_row_bytes;
