@@ -39,10 +39,11 @@ import numpy as np  # noqa: E402
 
 METRIC = "mixed-precision GEMM effective TOPS (and GEMV GB/s) and % of roofline on 1 GB300"
 L2_FLUSH_BYTES = 256 << 20       # > 129 MB L2
-KERNEL_SOURCES = ("paper_2311_14114_gb300/csrc/mma_gemm.cu",)
-# dram__bytes_read.sum + dram__bytes_write.sum of one launch of the dominant
-# kernel on the headline workload, from one ncu capture, keyed by the sha256 of
-# the kernel sources it was captured with: a different source reports null.
+KERNEL_SOURCES = ("paper_2311_14114_gb300/csrc/staged_gemm.cu", "paper_2311_14114_gb300/csrc/tc_ptx.cuh")
+# dram__bytes_read.sum + dram__bytes_write.sum of one soniq_mp_gemm call on the
+# headline workload (its three kernels: activation expand, weight expand,
+# staged tcgen05 GEMM), from one ncu capture, keyed by the sha256 of the
+# kernel sources it was captured with: a different source reports null.
 TRAFFIC = {"sha256": None, "bytes": None, "capture": None}
 
 
@@ -186,8 +187,10 @@ def _time_graph(g, steps, flush, stream, warm=3):
 
 
 def _time_fn(fn, steps, flush, stream):
-    """Median device time (ms) of a library call replayed as a CUDA graph."""
-    return statistics.median(_time_graph(_graph(fn, stream), steps, flush, stream))
+    """Mean device time (ms) of a library call replayed as a CUDA graph (the
+    mean, not the median: event timestamps here tick in steps of about 2 us,
+    which a median of short calls would keep)."""
+    return statistics.mean(_time_graph(_graph(fn, stream), steps, flush, stream))
 
 
 def run_gpu(args):
@@ -331,7 +334,7 @@ def run_gpu(args):
     peak = mixed_peak(linear_ops(spec.M, spec.N, d["count"]), kinds, pk)
     sha = kernel_sha()
     traffic = TRAFFIC["bytes"] if TRAFFIC["sha256"] == sha else None
-    roofline = {"kernel": "soniq_mp_gemm tensor-core path", "bound": "tensor",
+    roofline = {"kernel": "soniq_mp_gemm call (operand expand + staged tcgen05 GEMM)", "bound": "tensor",
                 "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": "TFLOP/s",
                 "frac": round(achieved / peak, 4), "traffic": traffic,
                 "peak_source": f"{pk['src']}: bf16 {pk['bf16']} TFLOP/s burst; E4M3 = 2x bf16 "
@@ -610,7 +613,8 @@ def run_reference(args):
 
 def run_case(args):
     """One kernel family on one workload, for profiling (ncu) and tuning:
-    headline | quant_headline | conv_4b8b | conv_1b4b | quant_conv | gemm:MxNxK:lo:hi:frac | gemv:M."""
+    headline | quant_headline | conv_4b8b | conv_1b4b | quant_conv | mlp_next | mlp_next_codes |
+    gemm:MxNxK:lo:hi:frac | gemv:M."""
     import torch
     from paper_2311_14114_gb300 import soniq as sq
     from paper_2311_14114_gb300 import workloads as wl
@@ -648,6 +652,22 @@ def run_case(args):
             fn, ops = (lambda: sq.quantize_act(lay, A, "tensor", s_a=s_a, Ap=Ap)), 0
         else:
             fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y, flags=args.flags)), spec.ops
+    elif name in ("mlp_next", "mlp_next_codes"):
+        # the MLP up-projection whose epilogue writes the next layer's codes
+        spec = wl.MLP_UP
+        d = wl.make_linear(spec)
+        perm2, count2, _ = wl.assignment(np.random.default_rng(spec.seed + 1), spec.N, 0.2, 0)
+        lay2 = sq.Layout(perm2, count2, [2, 8])
+        order = sq.next_layer_row_order(lay2)
+        Wa = np.zeros((len(order), spec.K), np.float32)
+        Wa[order >= 0] = d["W"][order[order >= 0]]
+        lay = sq.Layout(d["perm"], d["count"], d["bits"])
+        Wp, s_w = sq.pack_weights(lay, torch.from_numpy(Wa).cuda())
+        Ap, s_a = sq.quantize_act(lay, torch.from_numpy(d["A"]).cuda())
+        nxt = sq.NextLayer(lay2, torch.tensor([0.6, 1.8], dtype=torch.float32, device="cuda"), M=spec.M)
+        Y = torch.empty((spec.M, len(order)), dtype=torch.float16, device="cuda")
+        wy = name == "mlp_next"
+        fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y if wy else None, next=nxt, write_y=wy)), spec.ops
     elif name.startswith("gemv:"):
         spec = wl.DECODE[int(name.split(":")[1])]
         d = wl.make_linear(spec)

@@ -206,6 +206,41 @@ __device__ __forceinline__ void store_block32_n(int n, const uint32_t* o, uint8_
     }
 }
 
+// One packed block from 8 words of code bytes (byte b of o[t] is code
+// 4*t + b), for a width n known only at run time: the slice words of every
+// width are formed and the n output words selected from them, so the code is
+// short and indexes no register array by a run-time value.  dst is 4-byte
+// aligned.
+__device__ __forceinline__ void store_block32_rt(int n, const uint32_t (&o)[8], uint8_t* dst) {
+    uint32_t* d = reinterpret_cast<uint32_t*>(dst);
+    if (n == 8) {
+#pragma unroll
+        for (int t = 0; t < 8; ++t) d[t] = o[t];
+        return;
+    }
+    const int off2 = n & 4;                  // bit offset of the 2-bit slice in each code
+    const int off1 = (n & 4) + (n & 2);      // bit offset of the 1-bit slice
+    uint32_t s4[4], s2[2], s1 = 0u;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) s4[q] = (o[2 * q] & 0x0F0F0F0Fu) | ((o[2 * q + 1] & 0x0F0F0F0Fu) << 4);
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+        uint32_t v = 0u;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) v |= ((o[4 * q + j] >> off2) & 0x03030303u) << (2 * j);
+        s2[q] = v;
+    }
+#pragma unroll
+    for (int t = 0; t < 8; ++t) s1 |= ((o[t] >> off1) & 0x01010101u) << t;
+    const int b2 = (n & 4) ? 4 : 0;          // first word of the 2-bit slice
+    const int b1 = b2 + ((n & 2) ? 2 : 0);   // the word of the 1-bit slice
+#pragma unroll
+    for (int q = 0; q < 7; ++q) {
+        const uint32_t w = q < b2 ? s4[q & 3] : (q < b1 ? (((q - b2) & 1) ? s2[1] : s2[0]) : s1);
+        if (q < n) d[q] = w;
+    }
+}
+
 // Byte-wise sign-bit flip: n-bit two's complement j -> offset binary j + 2^(n-1).
 __device__ __forceinline__ uint32_t sign_flip_mask(int n) { return 0x01010101u << (n - 1); }
 

@@ -354,10 +354,67 @@ __device__ __forceinline__ void store_out16(const SParams& p, int64_t m, int nb,
 // epilogue drains one region while the MMAs fill the other.
 __device__ __forceinline__ int first_group(const SParams& p) { return p.seg_group == 1 ? 1 : 0; }
 
-// GENERAL = false: the common case compiled lean (no debug accumulators, no
-// next-layer codes, outputs through TMA stores), which keeps the unrolled
-// epilogue small enough for the instruction cache; GENERAL = true handles the rest.
-template <bool GENERAL>
+// Quantize-in-epilogue (Sec. 4.1, Conv2D + BatchNorm + Quantize fused): the
+// next layer's packed codes of this lane's row from the fp16 outputs in the
+// warp's staging tile (row `lane`, 128 columns from nc0, 64-column boxes of
+// 128-byte-swizzled rows).  The columns are the next layer's packed
+// positions, so each 32-column block is one packed block of its group (Sec. 3
+// step 2 with the next layer's calibrated scale).  Kept out of the unrolled
+// output loop, with run-time widths, so that the kernel's code stays small.
+__device__ __forceinline__ void next_layer_codes(const SParams& p, uint32_t out_s, int lane, int m, int nc0) {
+    const QConst kn0 = make_qconst(__ldg(p.s_next), p.next_bits[0]);
+    const QConst kn1 = make_qconst(__ldg(p.s_next + 1), p.next_bits[1]);
+#pragma unroll 1
+    for (int b = 0; b < EPI_COLS / 32; ++b) {
+        const int cb = nc0 + 32 * b;                       // first column of the block
+        if (cb >= p.N) break;
+        const int gn = cb >= p.next_pa0;
+        const int jg = cb - (gn ? p.next_pa0 : 0);         // position within the group
+        const QConst kn = gn ? kn1 : kn0;
+        const int valid = (gn ? p.next_count[1] : p.next_count[0]) - jg;   // real channels in the block
+        uint32_t o[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int cc = 4 * b + i;                      // 8-column chunk of the staging tile
+            const uint32_t src = out_s + (uint32_t)(cc >> 3) * 4096u + (uint32_t)lane * 128u +
+                                 ((((uint32_t)cc & 7u) ^ ((uint32_t)lane & 7u)) << 4);
+            uint32_t h[4];
+            asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(h[0]), "=r"(h[1]), "=r"(h[2]), "=r"(h[3])
+                         : "r"(src)
+                         : "memory");
+            uint32_t u[8];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&h[e]));
+                u[2 * e] = act_code_q<true>(f.x, kn.s, kn.r, kn.levels, kn.top);
+                u[2 * e + 1] = act_code_q<true>(f.y, kn.s, kn.r, kn.levels, kn.top);
+            }
+            if (kn.mode != 1) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&h[e]));
+                    u[2 * e] = kn.mode == 0 ? 0u : act_code_q<false>(f.x, kn.s, kn.r, kn.levels, kn.top);
+                    u[2 * e + 1] = kn.mode == 0 ? 0u : act_code_q<false>(f.y, kn.s, kn.r, kn.levels, kn.top);
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (8 * i + q >= valid) u[q] = 0u;         // padding positions hold code 0
+            o[2 * i] = u[0] | (u[1] << 8) | (u[2] << 16) | (u[3] << 24);
+            o[2 * i + 1] = u[4] | (u[5] << 8) | (u[6] << 16) | (u[7] << 24);
+        }
+        const int nb = gn ? p.next_bits[1] : p.next_bits[0];
+        store_block32_rt(nb, o, p.Ap_next + m * (int64_t)p.next_row_bytes + (gn ? p.next_off[1] : p.next_off[0]) +
+                                    (jg >> 5) * 4 * nb);
+    }
+}
+
+// Instantiations: GENERAL = false compiles the common epilogue lean (no debug
+// accumulators, outputs through TMA stores), which keeps the unrolled output
+// loop small enough for the instruction cache; GENERAL = true handles the
+// rest.  NEXT adds the next layer's codes (quantize-in-epilogue).
+template <bool GENERAL, bool NEXT>
 __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid_constant__ SParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -565,20 +622,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 // the final job: finish the tile's outputs, 8 columns at a time
                 const float sc = p.g[g_last].acc_scale;
                 const bool dbg = GENERAL && p.acc_dbg != nullptr && m < p.M;
-                const bool has_next = GENERAL && p.has_next;
+                constexpr bool has_next = NEXT;
                 const bool y_tma = GENERAL ? p.y_tma != 0 : true;
-                const bool write_y = GENERAL ? p.write_y != 0 : true;
-                if (y_tma) {
+                const bool write_y = (GENERAL || NEXT) ? p.write_y != 0 : true;
+                // fp16 outputs go through the staging tile for the TMA store and
+                // for the next layer's quantizer
+                const bool staged_out = y_tma || has_next;
+                if (staged_out) {
                     // the previous tile's store must have read the staging buffer
                     if (lane == 0) bulk_wait_read0();
                     __syncwarp();
                 }
-                QConst kn0, kn1;              // the next layer's quantizers
-                if (has_next) {
-                    kn0 = make_qconst(__ldg(p.s_next), p.next_bits[0]);
-                    kn1 = make_qconst(__ldg(p.s_next + 1), p.next_bits[1]);
-                }
-                uint32_t nq[8];               // the next layer's codes of the current 32-column block
 #pragma unroll
                 for (int cc = 0; cc < EPI_COLS / 8; ++cc) {
                     uint32_t v[8];
@@ -601,38 +655,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                             p.acc_dbg[(p.M + m) * p.N + nb + q] = a1;
                         }
                     }
-                    if (has_next) {
-                        // quantize fp16(y) for the next layer (Sec. 3 step 2 with its calibrated
-                        // scale), 8 codes of the block whose 32 columns end at chunk cc | 3
-                        const int cb = (nc0 + (cc & ~3) * 8);             // first column of the block
-                        const int gn = cb >= p.next_pa0;
-                        const int jg = cb - (gn ? p.next_pa0 : 0);        // position within the group
-                        const QConst& kn = gn ? kn1 : kn0;
-                        const int cnt = gn ? p.next_count[1] : p.next_count[0];
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            uint32_t word = 0u;
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const int q = 4 * h + e;
-                                const float a = __half2float(__float2half_rn(y[q]));
-                                uint32_t u = 0u;
-                                if (jg + (cc & 3) * 8 + q < cnt && kn.mode != 0)
-                                    u = kn.mode == 1 ? act_code_q<true>(a, kn.s, kn.r, kn.levels, kn.top)
-                                                     : act_code_q<false>(a, kn.s, kn.r, kn.levels, kn.top);
-                                word |= u << (8 * e);
-                            }
-                            nq[2 * (cc & 3) + h] = word;
-                        }
-                        if ((cc & 3) == 3 && m < p.M && cb < p.N) {
-                            const int nb = gn ? p.next_bits[1] : p.next_bits[0];
-                            store_block32_n(nb, nq, p.Ap_next + m * (int64_t)p.next_row_bytes +
-                                                        (gn ? p.next_off[1] : p.next_off[0]) + (jg >> 5) * 4 * nb);
-                        }
-                    }
-                    if (!write_y) {
-                        // no fp16/bf16 outputs requested
-                    } else if (y_tma) {
+                    if (staged_out) {
                         uint32_t w[4];
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
@@ -651,12 +674,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                         asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w[0]), "r"(w[1]),
                                      "r"(w[2]), "r"(w[3])
                                      : "memory");
-                    } else if (m < p.M) {
-                        store_out8(p, m, nb, y);
                     }
+                    if (write_y && !y_tma && m < p.M) store_out8(p, m, nb, y);
                 }
                 tc_fence_before();
-                if (y_tma) fence_proxy_async_shared();
+                if (staged_out) fence_proxy_async_shared();
                 __syncwarp();
                 if (lane == 0) {
                     mbar_arrive(bar(BAR_REG_EMPTY + r));
@@ -668,9 +690,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                         bulk_commit();
                     }
                 }
+                if (has_next && m < p.M) next_layer_codes(p, out_s, lane, m, nc0);
             }
         }
-        if ((GENERAL ? p.y_tma && p.write_y : true) && lane == 0) bulk_wait0();   // stores complete before the CTA exits
+        if (((GENERAL || NEXT) ? p.y_tma && p.write_y : true) && lane == 0) bulk_wait0();   // stores complete before the CTA exits
     }
 
     tc_fence_before();
@@ -889,25 +912,24 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         S.acc_scale = S.kind == 0 ? 262144.0f : 1.0f;   // 2^18
         S.inv_levels = (float)(1.0 / ((double)((1 << G.bits_a) - 1) * (double)(1 << (G.bits_w - 1))));
     }
-    static bool attr_done[64] = {};
+    // kernel instantiation: debug accumulators, outputs that cannot leave by
+    // TMA stores, or no outputs at all take the general epilogue
+    const bool general = a.acc_dbg != nullptr || (p.write_y && !p.y_tma) || (!p.write_y && !p.has_next);
+    void (*kern)(SParams) = general ? (p.has_next ? staged_mma_kernel<true, true> : staged_mma_kernel<true, false>)
+                                    : (p.has_next ? staged_mma_kernel<false, true> : staged_mma_kernel<false, false>);
+    static bool attr_done[64][4] = {};
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-        if ((err = cudaFuncSetAttribute(staged_mma_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        SMEM_ALLOC)) != cudaSuccess ||
-            (err = cudaFuncSetAttribute(staged_mma_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        SMEM_ALLOC)) != cudaSuccess)
+    const int kidx = (general ? 2 : 0) + (p.has_next ? 1 : 0);
+    if (dev >= 0 && dev < 64 && !attr_done[dev][kidx]) {
+        if ((err = cudaFuncSetAttribute((const void*)kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
+            cudaSuccess)
             return err;
-        attr_done[dev] = true;
+        if ((err = prefer_max_shared((const void*)kern)) != cudaSuccess) return err;
+        attr_done[dev][kidx] = true;
     }
     const int grid = p.total_tiles < num_sms() ? p.total_tiles : num_sms();
-    if (a.acc_dbg != nullptr || p.has_next || !p.y_tma || !p.write_y) {
-        if ((err = prefer_max_shared((const void*)staged_mma_kernel<true>)) != cudaSuccess) return err;
-        staged_mma_kernel<true><<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
-    } else {
-        if ((err = prefer_max_shared((const void*)staged_mma_kernel<false>)) != cudaSuccess) return err;
-        staged_mma_kernel<false><<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
-    }
+    kern<<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
     note_launch();
     return cudaGetLastError();
 }

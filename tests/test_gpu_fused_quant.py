@@ -87,7 +87,7 @@ def _check_codes(sq, lay2, perm2, count2, bits2, pad2, s2, order, Ap2_gpu, Y16_g
     assert bad_blocks <= max(2, Ap2_gpu.shape[0] // 50), f"{what}: {bad_blocks} blocks with differing outputs"
 
 
-@pytest.mark.parametrize("bits2,pad2", [((2, 8), 128), ((3, 6), 32), ((4, 4), 32), ((1, 8), 128)])
+@pytest.mark.parametrize("bits2,pad2", [((2, 8), 128), ((3, 6), 32), ((4, 4), 32), ((1, 8), 128), ((5, 7), 32)])
 def test_gemm_epilogue_writes_next_layer_codes(sq, bits2, pad2):
     d = wl.random_linear(600 + bits2[0], M=300, K=333, N=8, bits_lo=2, bits_hi=8, frac_hi=0.3, n_outliers=2)
     K2 = 200
