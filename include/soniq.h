@@ -114,20 +114,26 @@ enum {
                                             scratch suffices, however small the problem (without
                                             it the staged path is used from about 2^30
                                             multiply-adds) */
+    SONIQ_FLAG_FORCE_SKINNY = 16u,       /* tensor-core work takes the skinny swap-AB kernel
+                                            (M <= 32, taps = 1, groups padded to 128 codes) */
     SONIQ_FLAG_TEST_DROP_ARRIVE = 0x100u /* test hook: the tensor-core kernels' operand producer
                                             skips its first arrival (fused) or its first K-stage
-                                            (staged), so the consumer's bounded wait runs out and
-                                            the call reports SONIQ_ERR_TIMEOUT */
+                                            (staged, skinny), so the consumer's bounded wait runs
+                                            out and the call reports SONIQ_ERR_TIMEOUT */
 };
 
 /* Kernels behind soniq_mp_gemm (see soniq_mp_gemm_path). */
 enum {
     SONIQ_PATH_GEMV = 0,           /* CUDA-core GEMV streaming the packed weights (small M) */
     SONIQ_PATH_TENSOR = 1,         /* tcgen05 kernel expanding packed tiles on chip (no scratch) */
-    SONIQ_PATH_TENSOR_STAGED = 2   /* codes expanded once into scratch, then a tcgen05 GEMM */
+    SONIQ_PATH_TENSOR_STAGED = 2,  /* codes expanded once into scratch, then a tcgen05 GEMM */
+    SONIQ_PATH_TENSOR_SKINNY = 3   /* swap-AB tcgen05 kernel for few rows: packed weight rows
+                                      are the MMA's M = 128 side, converted on chip */
 };
-/* Without flags, soniq_mp_gemm runs the GEMV for M <= SONIQ_GEMV_MAX_M. */
+/* Without flags, soniq_mp_gemm runs the GEMV for M <= SONIQ_GEMV_MAX_M and the
+ * skinny tensor-core kernel for M <= SONIQ_SKINNY_MAX_M. */
 #define SONIQ_GEMV_MAX_M 12
+#define SONIQ_SKINNY_MAX_M 32
 
 /* Convolution geometry.  Input NHWC [batch][H][W][C_in], output NHWC
  * [batch][P][Q][C_out], P = (H + 2*pad_h - R)/stride_h + 1, Q likewise. */
@@ -287,9 +293,10 @@ SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, co
  *   Acc_g[m][n] = sum over k in group g of u[m][k] * j[n][k]   (exact int32)
  *   Y[m][n]     = sum_g s_a(m,g) * s_w[n][g] / ((2^na_g - 1) * 2^(nw_g - 1)) * Acc_g[m][n]
  * computed in fp32 and rounded to nearest fp16 (or bf16).  M <= SONIQ_GEMV_MAX_M
- * runs a bandwidth-bound CUDA-core GEMV, larger M the tcgen05 tensor-core
- * kernel (flags can force either; the GEMV takes M <= 16); soniq_mp_gemm_path
- * tells which.
+ * runs a bandwidth-bound CUDA-core GEMV, M <= SONIQ_SKINNY_MAX_M the skinny
+ * swap-AB tensor-core kernel, larger M the tcgen05 GEMM (flags can force a
+ * kernel; the GEMV takes M <= 16, the skinny kernel M <= 32);
+ * soniq_mp_gemm_path tells which.
  *
  *   Ap, s_a    from soniq_quantize_act with the same layout (pad_unit 32 or 128);
  *              s_a [2] (PER_TENSOR / CALIBRATED) or [M][2] (PER_ROW).

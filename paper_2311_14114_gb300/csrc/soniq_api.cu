@@ -176,9 +176,15 @@ int gemm_path(const LayoutGeom& geo, int64_t M, int32_t N, uint32_t flags, size_
     // up to SONIQ_GEMV_MAX_M rows the CUDA-core GEMV is faster; above, the tensor-core
     // kernels (whose time hardly grows with M below 128) overtake it
     const bool want_gemv =
-        (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= SONIQ_GEMV_MAX_M && !(flags & SONIQ_FLAG_FORCE_MMA));
+        (flags & SONIQ_FLAG_FORCE_GEMV) ||
+        (M <= SONIQ_GEMV_MAX_M && !(flags & (SONIQ_FLAG_FORCE_MMA | SONIQ_FLAG_FORCE_SKINNY)));
     if (want_gemv && gemv_supported(geo, M, N)) return SONIQ_PATH_GEMV;
     if (flags & SONIQ_FLAG_FORCE_GEMV) return -2;
+    const bool pinned = (flags & (SONIQ_FLAG_FORCE_FUSED | SONIQ_FLAG_FORCE_STAGED)) != 0;
+    if ((flags & SONIQ_FLAG_FORCE_SKINNY) || (!pinned && M <= SONIQ_SKINNY_MAX_M)) {
+        if (skinny_supported(geo, M, N)) return SONIQ_PATH_TENSOR_SKINNY;
+        if (flags & SONIQ_FLAG_FORCE_SKINNY) return -2;
+    }
     if (!(flags & SONIQ_FLAG_FORCE_FUSED) && staged_worthwhile(geo, M, N, flags)) {
         const int64_t need = staged_scratch_bytes(geo, M, N);
         if (need > 0 && (int64_t)scratch_bytes >= need) return SONIQ_PATH_TENSOR_STAGED;
@@ -350,6 +356,9 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     if (out_dtype != SONIQ_OUT_F16 && out_dtype != SONIQ_OUT_BF16) return SONIQ_ERR_INVALID_ARG;
     if ((flags & SONIQ_FLAG_FORCE_GEMV) && (flags & SONIQ_FLAG_FORCE_MMA)) return SONIQ_ERR_INVALID_ARG;
     if ((flags & SONIQ_FLAG_FORCE_FUSED) && (flags & SONIQ_FLAG_FORCE_STAGED)) return SONIQ_ERR_INVALID_ARG;
+    if ((flags & SONIQ_FLAG_FORCE_SKINNY) && (flags & (SONIQ_FLAG_FORCE_FUSED | SONIQ_FLAG_FORCE_STAGED |
+                                                      SONIQ_FLAG_FORCE_GEMV)))
+        return SONIQ_ERR_INVALID_ARG;
     LayoutGeom geo_next;
     if (next != nullptr && (st = check_next(next, N, out_dtype, &geo_next)) != SONIQ_OK) return st;
     if (M == 0 || N == 0) return SONIQ_OK;
@@ -361,7 +370,9 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     // K <= 65536 keeps |Acc| < 2^31 and the GEMV's unsigned offset sums below 2^32
     const int per_row = scale_mode == SONIQ_SCALE_PER_ROW;
     cudaStream_t s = as_stream(stream);
-    if (next != nullptr) flags = (flags & ~(uint32_t)SONIQ_FLAG_FORCE_GEMV) | SONIQ_FLAG_FORCE_MMA | SONIQ_FLAG_FORCE_STAGED;
+    if (next != nullptr)
+        flags = (flags & ~(uint32_t)(SONIQ_FLAG_FORCE_GEMV | SONIQ_FLAG_FORCE_SKINNY)) | SONIQ_FLAG_FORCE_MMA |
+                SONIQ_FLAG_FORCE_STAGED;
     const int path = gemm_path(geo, M, N, flags, scratch != nullptr ? scratch_bytes : 0);
     if (next != nullptr && path != SONIQ_PATH_TENSOR_STAGED) return SONIQ_ERR_UNSUPPORTED;
     if (path < 0) return path == -2 ? SONIQ_ERR_UNSUPPORTED : mma_check(geo);
@@ -389,6 +400,7 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
         a.next_Ap = next->Ap;
     }
     if (path == SONIQ_PATH_TENSOR_STAGED) return cuda_status(launch_staged(geo, a, scratch, scratch_bytes, s));
+    if (path == SONIQ_PATH_TENSOR_SKINNY) return cuda_status(launch_skinny(geo, a, s));
     return cuda_status(launch_mma(geo, a, s));
 }
 
@@ -472,8 +484,13 @@ int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout* L, int64_t M, int32_t N,
     if (M == 0 || N == 0 || (flags & SONIQ_FLAG_FORCE_FUSED)) return 0;
     // the GEMV needs none
     const bool want_gemv =
-        (flags & SONIQ_FLAG_FORCE_GEMV) || (M <= SONIQ_GEMV_MAX_M && !(flags & SONIQ_FLAG_FORCE_MMA));
+        (flags & SONIQ_FLAG_FORCE_GEMV) ||
+        (M <= SONIQ_GEMV_MAX_M && !(flags & (SONIQ_FLAG_FORCE_MMA | SONIQ_FLAG_FORCE_SKINNY)));
     if (want_gemv) return 0;
+    // nor the skinny kernel
+    const bool pinned = (flags & (SONIQ_FLAG_FORCE_FUSED | SONIQ_FLAG_FORCE_STAGED)) != 0;
+    if ((flags & SONIQ_FLAG_FORCE_SKINNY) || (!pinned && M <= SONIQ_SKINNY_MAX_M && skinny_supported(geo, M, N)))
+        return 0;
     return staged_worthwhile(geo, M, N, flags) ? staged_scratch_bytes(geo, M, N) : 0;
 }
 

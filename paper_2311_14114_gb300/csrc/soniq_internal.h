@@ -115,6 +115,11 @@ struct MmaArgs {
 soniq_status mma_check(const LayoutGeom& geo);
 cudaError_t launch_mma(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st);
 
+// ---- the skinny swap-AB tensor-core path (skinny_gemm.cu) ------------------
+// M <= 32 activation rows against packed weight rows converted on chip.
+bool skinny_supported(const LayoutGeom& geo, int64_t M, int64_t N);
+cudaError_t launch_skinny(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t st);
+
 // ---- the staged tensor-core path (staged_gemm.cu) ---------------------------
 // Packed codes are expanded once into tensor-pipe operands in caller scratch
 // (E4M3 bytes for groups with <= 4-bit codes on both sides, fp16 otherwise),

@@ -22,8 +22,10 @@ STATUS_NAMES = {0: "SONIQ_OK", 1: "SONIQ_ERR_INVALID_ARG", 2: "SONIQ_ERR_UNSUPPO
                 3: "SONIQ_ERR_ALIGNMENT", 4: "SONIQ_ERR_CUDA", 5: "SONIQ_ERR_TIMEOUT"}
 SCALE_PER_TENSOR, SCALE_PER_ROW, SCALE_CALIBRATED = 0, 1, 2
 OUT_F16, OUT_BF16 = 0, 1
-FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_FORCE_FUSED, FLAG_FORCE_STAGED, FLAG_TEST_DROP_ARRIVE = 1, 2, 4, 8, 0x100
-PATH_NAMES = {0: "CUDA-core GEMV", 1: "tensor-core fused kernel", 2: "tensor-core staged (expand + GEMM)"}
+FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_FORCE_FUSED, FLAG_FORCE_STAGED = 1, 2, 4, 8
+FLAG_FORCE_SKINNY, FLAG_TEST_DROP_ARRIVE = 16, 0x100
+PATH_NAMES = {0: "CUDA-core GEMV", 1: "tensor-core fused kernel", 2: "tensor-core staged (expand + GEMM)",
+              3: "tensor-core skinny (swap-AB)"}
 
 EXPORTED = ["soniq_abi_version", "soniq_status_string", "soniq_group_codes",
             "soniq_packed_row_bytes", "soniq_validate_layout", "soniq_launch_count",
