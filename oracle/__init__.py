@@ -75,6 +75,12 @@ def _load():
             lib.orc_conv_acc.argtypes = [P, i32, i32, i32, i32, P, i32, i32, i32, i32, i32,
                                          i32, i32, P, P, i64, P]
             lib.orc_epilogue.argtypes = [P, P, i64, i32, P, i32, P, P, P, P]
+            lib.orc_pm1_code.argtypes = [f32]
+            lib.orc_pm1_code.restype = i32
+            lib.orc_sub_scales.argtypes = [P, i64, i32, P, P, i32, i32, i32, P]
+            lib.orc_codes_variant.argtypes = [P, i64, i32, P, P, P, P, i32, i32, P, i32, P]
+            lib.orc_gemm_acc_runs.argtypes = [P, i32, P, i32, P, i32, i32, P, i64, P]
+            lib.orc_epilogue_runs.argtypes = [P, P, i64, i32, i32, P, i32, P, P, P, P, P]
             _lib = lib
     return _lib
 
@@ -335,3 +341,112 @@ def conv2d(X, W, perm, count, bits_a, bits_w, R, S, stride=(1, 1), pad=(1, 1), p
     Y = epilogue(acc, s_a, s_w, bits_a, bits_w)
     return dict(s_a=s_a, s_w=s_w, U=U, J=J, Xp=Xp, Wp=Wp, acc=acc, Y64=Y,
                 Y16=Y.astype(np.float16))
+
+
+# --------------------------------------------------------------------------
+# f3: variants (signed activations, one-bit +-1 groups, scale sub-groups along
+# K), linear layers.  kind[g]: 0 unsigned activations (default), 1 signed
+# activations (Eq. (1)), 2 +-1 codes on both sides (one-bit groups).
+# --------------------------------------------------------------------------
+
+def n_runs(count, sub_k: int) -> int:
+    """Scale runs per group array width: the larger group's run count."""
+    c = _pair(count)
+    if sub_k <= 0:
+        return 1
+    return int(max(1, max((int(x) + sub_k - 1) // sub_k for x in c)))
+
+
+def pm1_code(x: float) -> int:
+    return int(_load().orc_pm1_code(float(x)))
+
+
+def sub_scales(X, perm, count, sub_k: int, per_row: bool) -> np.ndarray:
+    X, Xp = _c(X, np.float32)
+    M, K = X.shape
+    perm, pp = _c(perm, np.int32)
+    cnt, cp = _c(_pair(count), np.int32)
+    nb = n_runs(count, sub_k)
+    s = np.zeros(((M if per_row else 1), 2, nb), dtype=np.float32)
+    _load().orc_sub_scales(Xp, M, K, pp, cp, int(sub_k), nb, int(per_row), s.ctypes.data_as(ctypes.c_void_p))
+    return s
+
+
+def codes_variant(X, perm, count, bits, kind, sub_k: int, s, per_row: bool) -> np.ndarray:
+    X, Xp = _c(X, np.float32)
+    M, K = X.shape
+    perm, pp = _c(perm, np.int32)
+    cnt, cp = _c(_pair(count), np.int32)
+    b, bp = _c(_pair(bits), np.int32)
+    kd, kp = _c(_pair(kind), np.int32)
+    s, sp = _c(s, np.float32)
+    C = np.zeros((M, K), dtype=np.int32)
+    _load().orc_codes_variant(Xp, M, K, pp, cp, bp, kp, int(sub_k), int(s.shape[-1]), sp, int(per_row),
+                              C.ctypes.data_as(ctypes.c_void_p))
+    return C
+
+
+def code_patterns(C, count, bits, kind) -> np.ndarray:
+    """The stored n-bit patterns of codes C (packed order): two's complement for
+    signed codes, bit (c + 1) / 2 for +-1 codes, the code itself otherwise."""
+    C = np.asarray(C, dtype=np.int64)
+    out = np.zeros(C.shape, dtype=np.uint8)
+    c0 = int(_pair(count)[0])
+    for g, sl in enumerate((slice(0, c0), slice(c0, C.shape[1]))):
+        n, k = int(_pair(bits)[g]), int(_pair(kind)[g])
+        x = C[:, sl]
+        out[:, sl] = ((x + 1) // 2) if k == 2 else (x & ((1 << n) - 1))
+    return out
+
+
+def gemm_acc_runs(U, J, count, sub_k: int, rows=None) -> np.ndarray:
+    """acc[2][nb][len(rows)][N] (int64)."""
+    U, Up = _c(U, np.int32)
+    J, Jp = _c(J, np.int32)
+    M, K = U.shape
+    N = J.shape[0]
+    nb = n_runs(count, sub_k)
+    rows = np.arange(M, dtype=np.int64) if rows is None else np.asarray(rows, dtype=np.int64)
+    rows, rp = _c(rows, np.int64)
+    cnt, cp = _c(_pair(count), np.int32)
+    acc = np.zeros((2, nb, rows.shape[0], N), dtype=np.int64)
+    _load().orc_gemm_acc_runs(Up, K, Jp, N, cp, int(sub_k), nb, rp, rows.shape[0],
+                              acc.ctypes.data_as(ctypes.c_void_p))
+    return acc
+
+
+def epilogue_runs(acc, s_a, s_w, bits_a, bits_w, kind, rows=None, s_a_per_row: bool = False) -> np.ndarray:
+    acc, accp = _c(acc, np.int64)
+    nb, n_rows, N = acc.shape[1], acc.shape[2], acc.shape[3]
+    rows = np.arange(n_rows, dtype=np.int64) if rows is None else np.asarray(rows, dtype=np.int64)
+    rows, rp = _c(rows, np.int64)
+    s_a, sap = _c(s_a, np.float32)
+    s_w, swp = _c(s_w, np.float32)
+    ba, bap = _c(_pair(bits_a), np.int32)
+    bw, bwp = _c(_pair(bits_w), np.int32)
+    kd, kp = _c(_pair(kind), np.int32)
+    Y = np.zeros((n_rows, N), dtype=np.float64)
+    _load().orc_epilogue_runs(accp, rp, n_rows, N, nb, sap, int(s_a_per_row), swp, bap, bwp, kp,
+                              Y.ctypes.data_as(ctypes.c_void_p))
+    return Y
+
+
+def linear_variant(A, W, perm, count, bits_a, bits_w, kind=(0, 0), sub_k: int = 0, act_mode="tensor",
+                   pad_unit: int = 128, rows=None):
+    """A linear layer under the f3 variants, all steps: scales per run, codes,
+    stored patterns, packed rows, run accumulators, fp64 and fp16 outputs.
+    Weights always take Eq. (1) (or +-1 in kind-2 groups) with per-row scales."""
+    A32 = np.asarray(A, dtype=np.float32)
+    W32 = np.asarray(W, dtype=np.float32)
+    per_row = act_mode == "row"
+    s_a = sub_scales(A32, perm, count, sub_k, per_row)
+    s_w = sub_scales(W32, perm, count, sub_k, True)
+    U = codes_variant(A32, perm, count, bits_a, kind, sub_k, s_a, per_row)
+    wkind = [2 if k == 2 else 1 for k in _pair(kind)]
+    J = codes_variant(W32, perm, count, bits_w, wkind, sub_k, s_w, True)
+    Ap = pack_act_rows(code_patterns(U, count, bits_a, kind), count, bits_a, pad_unit)
+    Wp = pack_act_rows(code_patterns(J, count, bits_w, wkind), count, bits_w, pad_unit)
+    acc = gemm_acc_runs(U, J, count, sub_k, rows=rows)
+    Y = epilogue_runs(acc, s_a, s_w, bits_a, bits_w, kind, rows=rows, s_a_per_row=per_row)
+    Yt = epilogue_runs(np.abs(acc), s_a, s_w, bits_a, bits_w, kind, rows=rows, s_a_per_row=per_row)
+    return dict(s_a=s_a, s_w=s_w, U=U, J=J, Ap=Ap, Wp=Wp, acc=acc, Y64=Y, Y16=Y.astype(np.float16), terms=Yt)

@@ -370,3 +370,102 @@ void orc_epilogue(const int64_t *acc, const int64_t *rows, int64_t n_rows, int32
             Y[i * N + n] = y;
         }
 }
+
+/* ------------------------------------------------------------------------- */
+/* f3  Variants the paper describes beside the default path (linear layers,  */
+/*     codes in packed channel order, int32).                                */
+/*  kind[g] 0: unsigned activation code, Sec. 3 step 2 (the default);         */
+/*          1: signed activation code, Eq. (1) applied to the activation     */
+/*             (u in [-2^(n-1), 2^(n-1)-1], decoded as s u / 2^(n-1)), the   */
+/*             transformer-layer reading of Sec. 3;                           */
+/*          2: one-bit +-1 code on both sides (Sec. 4.2: XNOR and POPCOUNT   */
+/*             for one-bit channels): +1 for x >= 0, else -1, decoded as     */
+/*             s * code; over m channels the dot product of two such rows is */
+/*             m - 2 popcount(bits XOR bits).                                 */
+/*  sub_k > 0: scale sub-groups along K (the fine scale groups, "GroupSize",  */
+/*     of the evaluation setup): a group's packed positions are cut into runs */
+/*     of sub_k, each with its own max-abs scale and exact accumulator; the  */
+/*     epilogue sums the runs.  sub_k = 0: one run per group (the default).  */
+/*  Scale arrays are [rows or 1][2][nb], nb = the larger group's run count.  */
+/* ------------------------------------------------------------------------- */
+int32_t orc_pm1_code(float x) { return x >= 0.0f ? 1 : -1; }
+
+static int32_t run_of(int32_t j, int32_t sub_k) { return sub_k > 0 ? j / sub_k : 0; }
+
+/* Max |x| over each run's real channels (per row, or over all rows). */
+void orc_sub_scales(const float *X, int64_t M, int32_t K, const int32_t *perm, const int32_t count[2],
+                    int32_t sub_k, int32_t nb, int32_t per_row, float *s) {
+    int32_t base[2] = {0, count[0]};
+    int64_t n_out = per_row ? M : 1;
+    for (int64_t i = 0; i < n_out * 2 * nb; ++i) s[i] = 0.0f;
+    for (int64_t m = 0; m < M; ++m)
+        for (int g = 0; g < ORC_GROUPS; ++g)
+            for (int32_t j = 0; j < count[g]; ++j) {
+                float v = fabsf(X[m * K + perm[base[g] + j]]);
+                float *t = &s[((per_row ? m : 0) * 2 + g) * nb + run_of(j, sub_k)];
+                if (v > *t) *t = v;
+            }
+}
+
+/* Codes C[M][K] of rows X[M][K] with scales s (layout above). */
+void orc_codes_variant(const float *X, int64_t M, int32_t K, const int32_t *perm, const int32_t count[2],
+                       const int32_t bits[2], const int32_t kind[2], int32_t sub_k, int32_t nb, const float *s,
+                       int32_t per_row, int32_t *C) {
+    int32_t base[2] = {0, count[0]};
+    for (int64_t m = 0; m < M; ++m)
+        for (int g = 0; g < ORC_GROUPS; ++g)
+            for (int32_t j = 0; j < count[g]; ++j) {
+                int32_t p = base[g] + j;
+                float x = X[m * K + perm[p]];
+                float sg = s[((per_row ? m : 0) * 2 + g) * nb + run_of(j, sub_k)];
+                int32_t c;
+                if (kind[g] == 2)
+                    c = orc_pm1_code(x);
+                else if (kind[g] == 1)
+                    c = orc_weight_code(x, sg, bits[g]);   /* Eq. (1), the same rule as for weights */
+                else
+                    c = orc_act_code(x, sg, bits[g]);
+                C[m * K + p] = c;
+            }
+}
+
+/* acc[2][nb][n_rows][N]: exact sums of U * J over each run of each group. */
+void orc_gemm_acc_runs(const int32_t *U, int32_t K, const int32_t *J, int32_t N, const int32_t count[2],
+                       int32_t sub_k, int32_t nb, const int64_t *rows, int64_t n_rows, int64_t *acc) {
+    int32_t base[2] = {0, count[0]};
+    for (int64_t i = 0; i < 2 * nb * n_rows * N; ++i) acc[i] = 0;
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < n_rows; ++i) {
+        int64_t m = rows[i];
+        for (int g = 0; g < ORC_GROUPS; ++g)
+            for (int32_t n = 0; n < N; ++n)
+                for (int32_t j = 0; j < count[g]; ++j) {
+                    int32_t b = run_of(j, sub_k);
+                    acc[(((int64_t)g * nb + b) * n_rows + i) * N + n] +=
+                        (int64_t)U[m * K + base[g] + j] * (int64_t)J[(int64_t)n * K + base[g] + j];
+                }
+    }
+}
+
+/* Y = sum_g sum_b s_a[g][b] s_w[n][g][b] acc[g][b] / (La_g Lw_g), fp64, with
+ * La = 2^na - 1 (kind 0), 2^(na-1) (kind 1), 1 (kind 2) and Lw = 2^(nw-1),
+ * or 1 for kind 2. */
+void orc_epilogue_runs(const int64_t *acc, const int64_t *rows, int64_t n_rows, int32_t N, int32_t nb,
+                       const float *s_a, int32_t s_a_per_row, const float *s_w, const int32_t bits_a[2],
+                       const int32_t bits_w[2], const int32_t kind[2], double *Y) {
+    for (int64_t i = 0; i < n_rows; ++i)
+        for (int32_t n = 0; n < N; ++n) {
+            double y = 0.0;
+            for (int g = 0; g < ORC_GROUPS; ++g) {
+                double la = kind[g] == 2 ? 1.0 : (kind[g] == 1 ? (double)(1 << (bits_a[g] - 1))
+                                                               : (double)((1 << bits_a[g]) - 1));
+                double lw = kind[g] == 2 ? 1.0 : (double)(1 << (bits_w[g] - 1));
+                for (int32_t b = 0; b < nb; ++b) {
+                    double sa = (double)s_a[((s_a_per_row ? rows[i] : 0) * 2 + g) * nb + b];
+                    double sw = (double)s_w[((int64_t)n * 2 + g) * nb + b];
+                    y += sa * sw * (double)acc[(((int64_t)g * nb + b) * n_rows + i) * N + n] / (la * lw);
+                }
+            }
+            Y[i * N + n] = y;
+        }
+}
