@@ -36,7 +36,7 @@
 extern "C" {
 #endif
 
-#define SONIQ_ABI_VERSION 2
+#define SONIQ_ABI_VERSION 3
 
 /* Exported symbols (the library is built with hidden default visibility). */
 #if defined(__GNUC__)
@@ -83,6 +83,24 @@ typedef void *soniq_stream_t;
  * takes w words and code i (t = i/4, b = i%4) sits in slice word t/(8/w) at
  * bit 8*b + w*(t % (8/w)).  Activation codes are unsigned, weight codes n-bit
  * two's complement.  Row strides are soniq_packed_row_bytes().
+ *
+ * Variants (all zero by default; linear layers only: taps = 1, pad_unit 128,
+ * per-row weight scales, the staged tensor-core path of soniq_mp_gemm):
+ *   act_kind[g]  SONIQ_ACT_UNSIGNED (Sec. 3 step 2), SONIQ_ACT_SIGNED (Eq. (1)
+ *              applied to the activation: codes in [-2^(n-1), 2^(n-1) - 1],
+ *              stored as n-bit two's complement, decoded as s u / 2^(n-1)),
+ *              or SONIQ_ACT_PM1 (one-bit groups, Sec. 4.2 XNOR / POPCOUNT:
+ *              both operands take code +1 for x >= 0 and -1 otherwise, stored
+ *              as the bit (code + 1) / 2 and decoded as s * code; needs
+ *              bits_w[g] = bits_a[g] = 1).
+ *   sub_k      0, or a multiple of 128: scale runs along K.  Group g's packed
+ *              positions are cut into runs of sub_k codes, each with its own
+ *              max-abs scale (activations per tensor or per row, weights per
+ *              row) and its own exact accumulator; the epilogue sums the runs.
+ *              Scale arrays then hold nb entries per (row, group):
+ *              [rows][2][nb], nb = soniq_scale_runs(layout).  Groups with
+ *              fp16 operands (codes above 4 bits) need sub_k <= 2^24 /
+ *              ((2^na - 1) 2^(nw - 1)) (512 for 8-bit groups).
  */
 typedef struct soniq_layout {
     int32_t K;
@@ -92,7 +110,11 @@ typedef struct soniq_layout {
     int32_t bits_a[2];
     const int32_t *perm;
     int32_t pad_unit;
+    int32_t act_kind[2];
+    int32_t sub_k;
 } soniq_layout;
+
+enum { SONIQ_ACT_UNSIGNED = 0, SONIQ_ACT_SIGNED = 1, SONIQ_ACT_PM1 = 2 };
 
 /* Scale granularity (Sec. 3 step 1: one max-abs scale per group; C2: one
  * scale per fused dot product).  Scale arrays are fp32 with 2 entries per
@@ -183,6 +205,10 @@ SONIQ_API int64_t soniq_group_codes(const soniq_layout *layout, int32_t group, i
  * argument. */
 SONIQ_API int64_t soniq_packed_row_bytes(const soniq_layout *layout, int32_t is_weight, int32_t taps);
 
+/* Scale runs per (row, group) in scale arrays: ceil(max PA_g / sub_k) with
+ * scale runs (layout->sub_k > 0), else 1.  -1 on a bad layout. */
+SONIQ_API int32_t soniq_scale_runs(const soniq_layout *layout);
+
 /* Checks the layout fields; if perm_host is non-NULL also checks that it is a
  * permutation of 0..K-1.  Does not read layout->perm. */
 SONIQ_API soniq_status soniq_validate_layout(const soniq_layout *layout, const int32_t *perm_host);
@@ -205,7 +231,9 @@ SONIQ_API int64_t soniq_launch_count(void);
  *   scale_mode SONIQ_SCALE_PER_ROW (one scale per (n, group) over all taps)
  *              or SONIQ_SCALE_PER_TENSOR (one per group; written to every row).
  *   Wp         device out [N][soniq_packed_row_bytes(layout, 1, taps)], 16-byte aligned.
- *   s_w        device out fp32 [N][2].
+ *   s_w        device out fp32 [N][2] ([N][2][nb] with scale runs).
+ * Layout variants (act_kind, sub_k): SONIQ_ACT_PM1 groups take code +1 / -1;
+ * scales are per row and per run; SONIQ_SCALE_PER_TENSOR is unsupported.
  */
 SONIQ_API soniq_status soniq_pack_weights(const soniq_layout *layout, const float *W, int32_t N,
                                 int32_t taps, int32_t scale_mode, uint8_t *Wp, float *s_w,
@@ -222,6 +250,9 @@ SONIQ_API soniq_status soniq_pack_weights(const soniq_layout *layout, const floa
  *   scale_mode SONIQ_SCALE_PER_TENSOR: s_a is an output [2];
  *              SONIQ_SCALE_PER_ROW:    s_a is an output [M][2];
  *              SONIQ_SCALE_CALIBRATED: s_a is an input [2].
+ *              With scale runs each entry is nb entries ([2][nb], [M][2][nb]).
+ *              Signed (SONIQ_ACT_SIGNED) groups take the Eq. (1) code, +-1
+ *              groups the sign; the variants need no scratch.
  *   s_a        device fp32, see scale_mode.
  *   Ap         device out [M][soniq_packed_row_bytes(layout, 0, 1)], 4-byte aligned.
  *   scratch, scratch_bytes

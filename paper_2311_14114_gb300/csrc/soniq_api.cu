@@ -149,6 +149,27 @@ soniq_status make_geom(const soniq_layout* L, int32_t taps, LayoutGeom* geo) {
     if (a_off > (1 << 30) || w_off > (1 << 30)) return SONIQ_ERR_UNSUPPORTED;
     geo->a_row_bytes = (int32_t)a_off;
     geo->w_row_bytes = (int32_t)w_off;
+    // variants
+    geo->variant = 0;
+    for (int g = 0; g < 2; ++g) {
+        const int k = L->act_kind[g];
+        if (k != SONIQ_ACT_UNSIGNED && k != SONIQ_ACT_SIGNED && k != SONIQ_ACT_PM1) return SONIQ_ERR_INVALID_ARG;
+        if (k == SONIQ_ACT_PM1 && g < L->n_groups && (L->bits_a[g] != 1 || L->bits_w[g] != 1))
+            return SONIQ_ERR_INVALID_ARG;
+        geo->act_kind[g] = g < L->n_groups ? k : SONIQ_ACT_UNSIGNED;
+        if (geo->act_kind[g] != SONIQ_ACT_UNSIGNED) geo->variant = 1;
+    }
+    if (L->sub_k < 0 || (L->sub_k > 0 && L->sub_k % 128 != 0)) return SONIQ_ERR_INVALID_ARG;
+    geo->sub_k = L->sub_k;
+    geo->nb = 1;
+    if (L->sub_k > 0) {
+        geo->variant = 1;
+        const int32_t pmax = geo->g[0].pa > geo->g[1].pa ? geo->g[0].pa : geo->g[1].pa;
+        geo->nb = (pmax + L->sub_k - 1) / L->sub_k;
+        if (geo->nb < 1) geo->nb = 1;
+    }
+    // the variants are implemented for linear layers with 128-code groups
+    if (geo->variant && (taps != 1 || L->pad_unit != 128)) return SONIQ_ERR_UNSUPPORTED;
     return SONIQ_OK;
 }
 
@@ -173,6 +194,12 @@ bool staged_worthwhile(const LayoutGeom& geo, int64_t M, int64_t N, uint32_t fla
 // tensor-core kernel would be chosen but cannot take the layout (mma_check
 // says why), -2 when the GEMV was forced but cannot take the shape.
 int gemm_path(const LayoutGeom& geo, int64_t M, int32_t N, uint32_t flags, size_t scratch_bytes) {
+    // the layout variants run on the staged path only
+    if (geo.variant) {
+        if (flags & (SONIQ_FLAG_FORCE_GEMV | SONIQ_FLAG_FORCE_FUSED | SONIQ_FLAG_FORCE_SKINNY)) return -2;
+        const int64_t need = staged_scratch_bytes(geo, M, N);
+        return need > 0 && (int64_t)scratch_bytes >= need ? SONIQ_PATH_TENSOR_STAGED : -2;
+    }
     // up to SONIQ_GEMV_MAX_M rows the CUDA-core GEMV is faster; above, the tensor-core
     // kernels (whose time hardly grows with M below 128) overtake it
     const bool want_gemv =
@@ -247,6 +274,12 @@ int64_t soniq_packed_row_bytes(const soniq_layout* L, int32_t is_weight, int32_t
     return is_weight ? geo.w_row_bytes : geo.a_row_bytes;
 }
 
+int32_t soniq_scale_runs(const soniq_layout* L) {
+    LayoutGeom geo;
+    if (make_geom(L, 1, &geo) != SONIQ_OK) return -1;
+    return geo.nb;
+}
+
 soniq_status soniq_validate_layout(const soniq_layout* L, const int32_t* perm_host) {
     LayoutGeom geo;
     soniq_status st = make_geom(L, 1, &geo);
@@ -275,6 +308,10 @@ soniq_status soniq_pack_weights(const soniq_layout* L, const float* W, int32_t N
     if (W == nullptr || Wp == nullptr || s_w == nullptr || L->perm == nullptr) return SONIQ_ERR_INVALID_ARG;
     if (!aligned(W, 4) || !aligned(Wp, 16) || !aligned(s_w, 4)) return SONIQ_ERR_ALIGNMENT;
     cudaStream_t s = as_stream(stream);
+    if (geo.variant) {
+        if (scale_mode != SONIQ_SCALE_PER_ROW) return SONIQ_ERR_UNSUPPORTED;
+        return cuda_status(launch_variant_pack_weights(geo, L->perm, W, N, s_w, Wp, s));
+    }
     if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
         cudaError_t e = launch_weight_absmax(geo, L->perm, W, N, s_w, s);
         if (e != cudaSuccess) return cuda_status(e);
@@ -303,6 +340,7 @@ soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M,
         return SONIQ_ERR_ALIGNMENT;
     cudaStream_t s = as_stream(stream);
     const uint16_t* A16 = static_cast<const uint16_t*>(A);
+    if (geo.variant) return cuda_status(launch_variant_quantize_act(geo, L->perm, A16, M, scale_mode, s_a, Ap, s));
     if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
         // a small input (up to 16K values): one CTA finds the scale and quantizes, no scratch needed
         if (M * (int64_t)L->K <= 16384) {
@@ -330,6 +368,7 @@ soniq_status soniq_quantize_act_oneshot(const soniq_layout* L, const void* A, in
     LayoutGeom geo;
     soniq_status st = make_geom(L, 1, &geo);
     if (st != SONIQ_OK) return st;
+    if (geo.variant) return SONIQ_ERR_UNSUPPORTED;
     if (L->K > 32768) return SONIQ_ERR_UNSUPPORTED;
     if (M < 0) return SONIQ_ERR_INVALID_ARG;
     if (M == 0) return SONIQ_OK;
@@ -361,6 +400,7 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
         return SONIQ_ERR_INVALID_ARG;
     LayoutGeom geo_next;
     if (next != nullptr && (st = check_next(next, N, out_dtype, &geo_next)) != SONIQ_OK) return st;
+    if (next != nullptr && (geo.variant || geo_next.variant)) return SONIQ_ERR_UNSUPPORTED;
     if (M == 0 || N == 0) return SONIQ_OK;
     if (Ap == nullptr || s_a == nullptr || Wp == nullptr || s_w == nullptr || (Y == nullptr && next == nullptr))
         return SONIQ_ERR_INVALID_ARG;
@@ -416,6 +456,7 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
     LayoutGeom geo;
     soniq_status st = make_geom(L, cd->R * cd->S, &geo);
     if (st != SONIQ_OK) return st;
+    if (geo.variant) return SONIQ_ERR_UNSUPPORTED;   // the layout variants are for linear layers
     if (scale_mode != SONIQ_SCALE_PER_TENSOR && scale_mode != SONIQ_SCALE_CALIBRATED) return SONIQ_ERR_INVALID_ARG;
     if (out_dtype != SONIQ_OUT_F16 && out_dtype != SONIQ_OUT_BF16) return SONIQ_ERR_INVALID_ARG;
     const int32_t P = (cd->H + 2 * cd->pad_h - cd->R) / cd->stride_h + 1;
@@ -481,7 +522,9 @@ int32_t soniq_mp_gemm_path(const soniq_layout* L, int64_t M, int32_t N, uint32_t
 int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout* L, int64_t M, int32_t N, uint32_t flags) {
     LayoutGeom geo;
     if (make_geom(L, 1, &geo) != SONIQ_OK || M < 0 || N < 0) return -1;
-    if (M == 0 || N == 0 || (flags & SONIQ_FLAG_FORCE_FUSED)) return 0;
+    if (M == 0 || N == 0) return 0;
+    if (geo.variant) return staged_scratch_bytes(geo, M, N);
+    if (flags & SONIQ_FLAG_FORCE_FUSED) return 0;
     // the GEMV needs none
     const bool want_gemv =
         (flags & SONIQ_FLAG_FORCE_GEMV) ||

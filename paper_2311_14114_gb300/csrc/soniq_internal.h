@@ -29,6 +29,12 @@ struct LayoutGeom {
     int32_t a_row_bytes;
     int32_t w_row_bytes;
     GroupGeom g[2];
+    // layout variants: SONIQ_ACT_* per group, scale runs along K (0: none),
+    // scale entries per (row, group), and whether any variant is on
+    int32_t act_kind[2];
+    int32_t sub_k;
+    int32_t nb;
+    int32_t variant;
 };
 
 // Fills `geo` from a layout; returns SONIQ_OK or the validation error.
@@ -74,6 +80,13 @@ cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, con
 cudaError_t launch_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W,
                                 int32_t N, int32_t per_row, uint8_t* Wp, float* s_w,
                                 cudaStream_t st);
+
+// Layout variants (variant.cu): scales per (row or tensor, group, run), then
+// codes and packing; weights always per row.
+cudaError_t launch_variant_quantize_act(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
+                                        int32_t scale_mode, float* s_a, uint8_t* Ap, cudaStream_t st);
+cudaError_t launch_variant_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W, int32_t N,
+                                        float* s_w, uint8_t* Wp, cudaStream_t st);
 
 struct GemvArgs {
     const uint8_t* Ap;

@@ -123,6 +123,9 @@ struct SParams {
     int32_t next_row_bytes;
     int32_t next_pa0;      // first packed position of its group 1
     int32_t next_count[2], next_bits[2], next_off[2];
+    // scale runs along K: every job is one run of one group, scaled on its own;
+    // s_a is [rows or 1][2][nb], s_w [N][2][nb]
+    int32_t runs, nb;
     SGroup g[2];
 };
 
@@ -145,6 +148,10 @@ struct ExpandParams {
     int32_t cpt[2];
     uint64_t cpt_magic[2];     // ceil(2^32 / cpt): tap = (kb * magic) >> 32, exact for kb < 2^32 / cpt
     int32_t vec16[2];          // source blocks of the group can be read as 16-byte vectors
+    // code encoding of each group: 0 unsigned, 1 n-bit two's complement (weights,
+    // signed activations), 2 one-bit +-1 (bit 1 -> +1, bit 0 -> -1, positions
+    // from count[g] on -> 0)
+    int32_t code_kind[2], count[2];
 };
 
 // n-bit two's-complement patterns in the bytes of x -> E4M3 sign-magnitude bytes.
@@ -192,8 +199,9 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
         wq = qq * p.sw - p.pw;
     }
     const uint32_t flip = 0x01010101u << (N - 1);
+    const int ck = p.code_kind[g];
     const __half2 bias = __half2half2(__ushort_as_half(
-        (unsigned short)(0x6400u + (p.is_weight ? (1u << (N - 1)) : (uint32_t)p.center[g]))));
+        (unsigned short)(0x6400u + (ck == 1 ? (1u << (N - 1)) : (uint32_t)p.center[g]))));
     int32_t csum = 0;
     for (int kb = lane; kb < p.blk_dst[g]; kb += 32) {
         const uint8_t* src = nullptr;
@@ -219,9 +227,17 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
         uint32_t o[8];
         block_to_bytes<N>(words, o);
         if (kind == 0) {
-            if (p.is_weight) {
+            if (ck == 1) {
 #pragma unroll
                 for (int t = 0; t < 8; ++t) o[t] = twos_to_e4m3<N>(o[t]);
+            } else if (ck == 2) {
+                // one-bit +-1: bit 1 -> E4M3 +2^-9 (0x01), bit 0 -> -2^-9 (0x81); none past count
+#pragma unroll
+                for (int t = 0; t < 8; ++t) {
+                    const int valid = p.count[g] - (kb * 32 + 4 * t);
+                    const uint32_t keep = valid >= 4 ? 0xFFFFFFFFu : (valid <= 0 ? 0u : (1u << (8 * valid)) - 1u);
+                    o[t] = (0x81818181u - (o[t] & 0x01010101u) * 0x80u) & keep;
+                }
             }
             uint4* d = reinterpret_cast<uint4*>(drow + kb * 32);
             d[0] = make_uint4(o[0], o[1], o[2], o[3]);
@@ -230,8 +246,8 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
             uint32_t h[16];
 #pragma unroll
             for (int t = 0; t < 8; ++t) {
-                // weights: offset binary j + 2^(n-1); activations: the code u
-                const uint32_t x = p.is_weight ? (o[t] ^ flip) : o[t];
+                // signed codes: offset binary j + 2^(n-1); unsigned: the code u
+                const uint32_t x = ck == 1 ? (o[t] ^ flip) : o[t];
                 if (p.is_weight) csum += (int32_t)__dp4a(x, 0x01010101u, 0u);
                 uint32_t lo, hi;
                 bytes_to_magic_half2(x, lo, hi);
@@ -410,6 +426,102 @@ __device__ __forceinline__ void next_layer_codes(const SParams& p, uint32_t out_
     }
 }
 
+// Scale runs along K (epilogue warp, one tile): every job is one run b of one
+// group g, drained as its exact integer sum and added in fp32 with its own
+// scale, y += s_a(g, b) s_w(n, g, b) / (La Lw) * Acc(g, b); then the tile's
+// outputs.  `kw` is this warp's 128-float scratch for a run's column scales.
+// With debug accumulators, acc_dbg receives [2][nb][M][N].  Returns false
+// after a wait ran out.
+__device__ __noinline__ bool runs_tile(const SParams& p, uint32_t sbase, uint32_t bar0, uint32_t abort_flag,
+                                       uint32_t lane_base, uint32_t out_s, float* kw, int lane, int quad, int64_t m,
+                                       int64_t m0, int nc0, uint32_t& job) {
+    auto bar = [&](int i) { return bar0 + 8u * (uint32_t)i; };
+    float yr[EPI_COLS];
+#pragma unroll
+    for (int j = 0; j < EPI_COLS; ++j) yr[j] = 0.0f;
+    const bool dbg = p.acc_dbg != nullptr && m < p.M;
+    for (int g = 0; g < 2; ++g) {
+        const int nrun = p.g[g].stages > 0 ? p.g[g].n_seg : 0;
+        const float sc = p.g[g].acc_scale;
+#pragma unroll 1
+        for (int b = 0; b < nrun; ++b, ++job) {
+            const uint32_t r = job & 1u, use = job >> 1;
+            if (!__all_sync(0xffffffffu, wait_bounded(bar(BAR_REG_FULL + r), use & 1u, abort_flag, kTimeoutNs,
+                                                      p.err, kErrWait)))
+                return false;
+            tc_fence_after();
+            __syncwarp();
+#pragma unroll
+            for (int h = 0; h < EPI_COLS / 32; ++h) {
+                const int c = lane + 32 * h;
+                const int n = nc0 + c < p.N ? nc0 + c : p.N - 1;
+                kw[c] = __ldg(p.s_w + ((int64_t)n * 2 + g) * p.nb + b) * p.g[g].inv_levels;
+            }
+            __syncwarp();
+            const float sa = m < p.M ? __ldg(p.s_a + ((p.s_a_per_row ? m : 0) * 2 + g) * p.nb + b) : 0.0f;
+            const uint32_t taddr = lane_base + r * BN;
+#pragma unroll
+            for (int cc = 0; cc < EPI_COLS / 8; ++cc) {
+                uint32_t v[8];
+                tmem_ld8(taddr + cc * 8, v);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const int j = cc * 8 + q;
+                    const int32_t x = __float2int_rn(__uint_as_float(v[q]) * sc);
+                    yr[j] = fmaf(sa * kw[j], (float)x, yr[j]);
+                    if (dbg && nc0 + j < p.N)
+                        p.acc_dbg[(((int64_t)g * p.nb + b) * p.M + m) * p.N + nc0 + j] = x;
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(BAR_REG_EMPTY + r));
+        }
+    }
+    // the tile's outputs, 8 columns at a time
+    if (p.y_tma) {
+        if (lane == 0) bulk_wait_read0();
+        __syncwarp();
+    }
+#pragma unroll
+    for (int cc = 0; cc < EPI_COLS / 8; ++cc) {
+        float y[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) y[q] = yr[cc * 8 + q];
+        if (p.y_tma) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                if (p.out_bf16) {
+                    __nv_bfloat162 h2 = __floats2bfloat162_rn(y[2 * e], y[2 * e + 1]);
+                    w[e] = *reinterpret_cast<uint32_t*>(&h2);
+                } else {
+                    __half2 h2 = __floats2half2_rn(y[2 * e], y[2 * e + 1]);
+                    w[e] = *reinterpret_cast<uint32_t*>(&h2);
+                }
+            }
+            const uint32_t dst = out_s + (uint32_t)(cc >> 3) * 4096u + (uint32_t)lane * 128u +
+                                 ((((uint32_t)cc & 7u) ^ ((uint32_t)lane & 7u)) << 4);
+            asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+                         "r"(w[3])
+                         : "memory");
+        } else if (m < p.M) {
+            store_out8(p, m, nc0 + cc * 8, y);
+        }
+    }
+    if (p.y_tma) {
+        fence_proxy_async_shared();
+        __syncwarp();
+        if (lane == 0) {
+#pragma unroll
+            for (int bx = 0; bx < EPI_COLS / 64; ++bx)
+                tma_store_2d(&p.tma_y, nc0 + bx * 64, (int)(m0 + quad * 32), out_s + bx * 4096u);
+            bulk_commit();
+        }
+    }
+    return true;
+}
+
 // Instantiations: GENERAL = false compiles the common epilogue lean (no debug
 // accumulators, outputs through TMA stores), which keeps the unrolled output
 // loop small enough for the instruction cache; GENERAL = true handles the
@@ -495,7 +607,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     const int g = gi == 0 ? g_first : 1 - g_first;
                     const int ns = p.g[g].stages;
                     const bool f8 = p.g[g].kind == 0;
-                    const int per_job = g == p.seg_group ? p.g[g].seg_stages : ns;
+                    const int per_job = p.g[g].n_seg > 1 ? p.g[g].seg_stages : ns;
 #pragma unroll 1
                     for (int i = 0; i < ns && ok; ++job) {
                         const uint32_t r = job & 1u, use = job >> 1;
@@ -574,14 +686,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 sa0 = p.s_a_per_row ? __ldg(p.s_a + m * 2) : __ldg(p.s_a);
                 sa1 = p.s_a_per_row ? __ldg(p.s_a + m * 2 + 1) : __ldg(p.s_a + 1);
             }
+            if constexpr (GENERAL) {
+                if (p.runs) {
+                    if (!runs_tile(p, sbase, bar0, abort_flag, lane_base, out_s, reinterpret_cast<float*>(colc), lane,
+                                   quad, m, m0, nc0, job))
+                        ok = false;
+                    continue;
+                }
+            }
             // part: the exact accumulator of the first group (or the running
             // sum of the segments of the tile's only group)
             int32_t part[EPI_COLS];
 #pragma unroll
             for (int j = 0; j < EPI_COLS; ++j) part[j] = 0;
             const int gA = g_first, gB = 1 - g_first;
-            const int nA = p.g[gA].stages > 0 ? (gA == p.seg_group ? p.g[gA].n_seg : 1) : 0;
-            const int nB = p.g[gB].stages > 0 ? (gB == p.seg_group ? p.g[gB].n_seg : 1) : 0;
+            const int nA = p.g[gA].stages > 0 ? p.g[gA].n_seg : 0;
+            const int nB = p.g[gB].stages > 0 ? p.g[gB].n_seg : 0;
             const int njobs = nA + nB;
             const int g_last = nB > 0 ? gB : gA;        // group of the final job
             const bool part_is_other = nA > 0 && nB > 0;
@@ -749,23 +869,35 @@ bool staged_plan(const LayoutGeom& geo, StagedPlan* sp) {
     int nseg_groups = 0;
     int64_t x0 = 0;
     sp->seg_group = -1;
+    const bool runs = geo.sub_k > 0;
     for (int g = 0; g < 2; ++g) {
         const GroupGeom& G = geo.g[g];
         StagedGroup& S = sp->g[g];
+        const int ak = geo.act_kind[g];
         S.kind = (G.bits_a <= 4 && G.bits_w <= 4) ? 0 : 1;
         const int64_t bytes = (int64_t)G.pw * (S.kind == 0 ? 1 : 2);
         S.stages = (int32_t)(bytes / staged::KSTAGE);
         S.x0 = (int32_t)x0;
         x0 += bytes;
-        const int64_t maxprod = S.kind == 0 ? (int64_t)((1 << G.bits_a) - 1) * (1 << (G.bits_w - 1))
-                                            : (int64_t)(1 << (G.bits_a - 1)) * (1 << (G.bits_w - 1));
+        // unsigned fp16 activations are centred (halving the products) unless every
+        // run is scaled on its own, where the centring's weight sums would be per run
+        S.center = (S.kind == 1 && ak == SONIQ_ACT_UNSIGNED && !runs) ? (1 << (G.bits_a - 1)) : 0;
+        const int64_t amax = ak == SONIQ_ACT_PM1 ? 1
+                                                 : (ak == SONIQ_ACT_SIGNED || S.center ? (int64_t)1 << (G.bits_a - 1)
+                                                                                       : (1 << G.bits_a) - 1);
+        const int64_t wmax = ak == SONIQ_ACT_PM1 ? 1 : (int64_t)1 << (G.bits_w - 1);
+        const int64_t maxprod = amax * wmax;
         const int64_t codes_per_stage = S.kind == 0 ? staged::KSTAGE : staged::KSTAGE / 2;
-        const int64_t seg_stages = ((int64_t)1 << 24) / maxprod / codes_per_stage;
+        int64_t seg_stages = ((int64_t)1 << 24) / maxprod / codes_per_stage;
+        if (runs) {
+            // one job per run; its exact sum must stay within 2^24
+            if ((int64_t)geo.sub_k * maxprod > ((int64_t)1 << 24)) return false;
+            seg_stages = geo.sub_k / codes_per_stage;
+        }
         if (seg_stages < 1) return false;
         S.seg_stages = (int32_t)(seg_stages < S.stages ? seg_stages : (S.stages > 0 ? S.stages : 1));
         S.n_seg = S.stages > 0 ? (S.stages + S.seg_stages - 1) / S.seg_stages : 0;
-        S.center = S.kind == 1 ? (1 << (G.bits_a - 1)) : 0;
-        if (S.n_seg > 1) {
+        if (S.n_seg > 1 && !runs) {
             ++nseg_groups;
             sp->seg_group = g;
         }
@@ -810,6 +942,8 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         e.cpt[g] = G.pa / 32 > 0 ? G.pa / 32 : 1;
         e.cpt_magic[g] = (((uint64_t)1 << 32) + (uint64_t)e.cpt[g] - 1) / (uint64_t)e.cpt[g];
         e.vec16[g] = (G.a_off % 16 == 0 && geo.a_row_bytes % 16 == 0 && (uintptr_t)a.Ap % 16 == 0) ? 1 : 0;
+        e.code_kind[g] = geo.act_kind[g];
+        e.count[g] = G.count;
     }
     e.src = a.Ap;
     e.src_row_bytes = geo.a_row_bytes;
@@ -839,6 +973,7 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         w.blk_src[g] = G.pw / 32;
         w.center[g] = 0;
         w.vec16[g] = (G.w_off % 16 == 0 && geo.w_row_bytes % 16 == 0 && (uintptr_t)a.Wp % 16 == 0) ? 1 : 0;
+        w.code_kind[g] = geo.act_kind[g] == SONIQ_ACT_PM1 ? 2 : 1;
     }
     w.src = a.Wp;
     w.src_row_bytes = geo.w_row_bytes;
@@ -910,11 +1045,20 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         S.n_seg = sp.g[g].n_seg;
         S.center = sp.g[g].center;
         S.acc_scale = S.kind == 0 ? 262144.0f : 1.0f;   // 2^18
-        S.inv_levels = (float)(1.0 / ((double)((1 << G.bits_a) - 1) * (double)(1 << (G.bits_w - 1))));
+        // decode levels: activations 2^na - 1 (unsigned), 2^(na-1) (signed) or 1 (+-1);
+        // weights 2^(nw-1) or 1 (+-1)
+        const int ak = geo.act_kind[g];
+        const double la = ak == SONIQ_ACT_PM1 ? 1.0 : (ak == SONIQ_ACT_SIGNED ? (double)(1 << (G.bits_a - 1))
+                                                                             : (double)((1 << G.bits_a) - 1));
+        const double lw = ak == SONIQ_ACT_PM1 ? 1.0 : (double)(1 << (G.bits_w - 1));
+        S.inv_levels = (float)(1.0 / (la * lw));
     }
     // kernel instantiation: debug accumulators, outputs that cannot leave by
     // TMA stores, or no outputs at all take the general epilogue
-    const bool general = a.acc_dbg != nullptr || (p.write_y && !p.y_tma) || (!p.write_y && !p.has_next);
+    p.runs = geo.sub_k > 0 ? 1 : 0;
+    p.nb = geo.nb;
+    const bool general =
+        a.acc_dbg != nullptr || p.runs || (p.write_y && !p.y_tma) || (!p.write_y && !p.has_next);
     void (*kern)(SParams) = general ? (p.has_next ? staged_mma_kernel<true, true> : staged_mma_kernel<true, false>)
                                     : (p.has_next ? staged_mma_kernel<false, true> : staged_mma_kernel<false, false>);
     static bool attr_done[64][4] = {};

@@ -24,11 +24,12 @@ SCALE_PER_TENSOR, SCALE_PER_ROW, SCALE_CALIBRATED = 0, 1, 2
 OUT_F16, OUT_BF16 = 0, 1
 FLAG_FORCE_GEMV, FLAG_FORCE_MMA, FLAG_FORCE_FUSED, FLAG_FORCE_STAGED = 1, 2, 4, 8
 FLAG_FORCE_SKINNY, FLAG_TEST_DROP_ARRIVE = 16, 0x100
+ACT_UNSIGNED, ACT_SIGNED, ACT_PM1 = 0, 1, 2
 PATH_NAMES = {0: "CUDA-core GEMV", 1: "tensor-core fused kernel", 2: "tensor-core staged (expand + GEMM)",
               3: "tensor-core skinny (swap-AB)"}
 
 EXPORTED = ["soniq_abi_version", "soniq_status_string", "soniq_group_codes",
-            "soniq_packed_row_bytes", "soniq_validate_layout", "soniq_launch_count",
+            "soniq_packed_row_bytes", "soniq_scale_runs", "soniq_validate_layout", "soniq_launch_count",
             "soniq_pack_weights", "soniq_quantize_act", "soniq_quantize_act_scratch_bytes",
             "soniq_quantize_act_oneshot", "soniq_mp_gemm", "soniq_mp_gemm_path", "soniq_mp_gemm_scratch_bytes",
             "soniq_mp_conv2d", "soniq_mp_conv2d_scratch_bytes", "soniq_sync_status",
@@ -47,7 +48,7 @@ class CLayout(ctypes.Structure):
     _fields_ = [("K", ctypes.c_int32), ("n_groups", ctypes.c_int32),
                 ("count", ctypes.c_int32 * 2), ("bits_w", ctypes.c_int32 * 2),
                 ("bits_a", ctypes.c_int32 * 2), ("perm", ctypes.c_void_p),
-                ("pad_unit", ctypes.c_int32)]
+                ("pad_unit", ctypes.c_int32), ("act_kind", ctypes.c_int32 * 2), ("sub_k", ctypes.c_int32)]
 
 
 class CNextLayer(ctypes.Structure):
@@ -79,6 +80,8 @@ def lib() -> ctypes.CDLL:
         L.soniq_group_codes.restype = i64
         L.soniq_packed_row_bytes.argtypes = [P, i32, i32]
         L.soniq_packed_row_bytes.restype = i64
+        L.soniq_scale_runs.argtypes = [P]
+        L.soniq_scale_runs.restype = i32
         L.soniq_validate_layout.argtypes = [P, P]
         L.soniq_validate_layout.restype = i32
         L.soniq_launch_count.restype = i64
@@ -162,10 +165,13 @@ class Layout:
 
     perm[j] is the original channel at packed position j; positions
     [0, count[0]) form the low-precision group 0.  The permutation is kept in
-    device memory (the kernels gather through it)."""
+    device memory (the kernels gather through it).  act_kind (per group:
+    ACT_UNSIGNED, ACT_SIGNED, ACT_PM1) and sub_k (scale runs along K) select
+    the layout variants of soniq_layout."""
 
     def __init__(self, perm: Sequence[int], count: Sequence[int], bits_w: Sequence[int],
-                 bits_a: Optional[Sequence[int]] = None, pad_unit: int = 128, device=None):
+                 bits_a: Optional[Sequence[int]] = None, pad_unit: int = 128, device=None,
+                 act_kind: Sequence[int] = (0, 0), sub_k: int = 0):
         bits_a = bits_w if bits_a is None else bits_a
         perm_t = torch.as_tensor(perm, dtype=torch.int32).contiguous()
         self.K = int(perm_t.numel())
@@ -175,9 +181,11 @@ class Layout:
         self.bits_a = [int(b) for b in list(bits_a)[:2]] + [1] * (2 - len(bits_a))
         self.pad_unit = int(pad_unit)
         n_groups = 2 if self.count[1] > 0 else 1
+        self.act_kind = [int(k) for k in list(act_kind)[:2]] + [0] * (2 - len(act_kind))
+        self.sub_k = int(sub_k)
         host = CLayout(self.K, n_groups, (ctypes.c_int32 * 2)(*self.count),
                        (ctypes.c_int32 * 2)(*self.bits_w), (ctypes.c_int32 * 2)(*self.bits_a),
-                       None, self.pad_unit)
+                       None, self.pad_unit, (ctypes.c_int32 * 2)(*self.act_kind), self.sub_k)
         _check(lib().soniq_validate_layout(ctypes.byref(host),
                                            perm_t.numpy().ctypes.data_as(ctypes.c_void_p)),
                "soniq_validate_layout")
@@ -194,6 +202,15 @@ class Layout:
 
     def group_codes(self, g: int, is_weight: bool = False, taps: int = 1) -> int:
         return int(lib().soniq_group_codes(ctypes.byref(self.c), int(g), int(is_weight), int(taps)))
+
+    def scale_runs(self) -> int:
+        """Scale entries per (row, group): soniq_scale_runs."""
+        return int(lib().soniq_scale_runs(ctypes.byref(self.c)))
+
+    def scale_shape(self, rows: Optional[int]) -> tuple:
+        """Shape of a scale array: [rows][2] or [2], with a run axis when sub_k > 0."""
+        tail = (2,) if self.sub_k == 0 else (2, self.scale_runs())
+        return tail if rows is None else (rows,) + tail
 
 
 def next_layer_row_order(next_layout: Layout):
@@ -234,7 +251,7 @@ def pack_weights(layout: Layout, W: torch.Tensor, scale_mode: str = "row",
     if Wp is None:
         Wp = torch.empty((N, layout.row_bytes(True, taps)), dtype=torch.uint8, device=W.device)
     if s_w is None:
-        s_w = torch.empty((N, 2), dtype=torch.float32, device=W.device)
+        s_w = torch.empty(layout.scale_shape(N), dtype=torch.float32, device=W.device)
     mode = {"row": SCALE_PER_ROW, "tensor": SCALE_PER_TENSOR}[scale_mode]
     _check(lib().soniq_pack_weights(ctypes.byref(layout.c), _ptr(W), N, taps, mode, _ptr(Wp),
                                     _ptr(s_w), _stream(stream)), "soniq_pack_weights")
@@ -254,7 +271,7 @@ def quantize_act(layout: Layout, A: torch.Tensor, scale_mode: str = "tensor",
     if s_a is None:
         if mode == SCALE_CALIBRATED:
             raise ValueError("calibrated mode needs s_a")
-        s_a = torch.empty((M, 2) if mode == SCALE_PER_ROW else (2,), dtype=torch.float32,
+        s_a = torch.empty(layout.scale_shape(M if mode == SCALE_PER_ROW else None), dtype=torch.float32,
                           device=A.device)
     if Ap is None:
         Ap = torch.empty((M, layout.row_bytes(False)), dtype=torch.uint8, device=A.device)

@@ -39,11 +39,13 @@ def test_library_exports_every_declared_symbol(L):
     for name in names:
         assert hasattr(L, name), name
     assert sorted(soniq.EXPORTED) == names
-    assert L.soniq_abi_version() == 2
+    assert L.soniq_abi_version() == 3
 
 
-def _layout(soniq, K=300, count=(200, 100), bits=(3, 8), pad=128, perm=None):
+def _layout(soniq, K=300, count=(200, 100), bits=(3, 8), pad=128, perm=None, act_kind=(0, 0), sub_k=0):
     c = soniq.CLayout()
+    c.act_kind[0], c.act_kind[1] = act_kind
+    c.sub_k = sub_k
     c.K = K
     c.n_groups = 2 if count[1] else 1
     c.count[0], c.count[1] = count
@@ -153,3 +155,30 @@ def test_scratch_size_queries(L):
 def test_status_strings(L):
     L.soniq_status_string.restype = ctypes.c_char_p
     assert L.soniq_status_string(5) == b"device wait timed out"
+
+
+def test_layout_variant_checks(L):
+    """Host-side checks of the layout variants (signed activations, +-1 groups,
+    scale runs): validation, run counts, and that only the staged path takes them."""
+    from paper_2311_14114_gb300 import soniq
+    perm = np.arange(300, dtype=np.int32)
+    pp = perm.ctypes.data_as(ctypes.c_void_p)
+    ok = _layout(soniq, act_kind=(1, 1))
+    assert L.soniq_validate_layout(ctypes.byref(ok), pp) == 0
+    assert L.soniq_scale_runs(ctypes.byref(ok)) == 1
+    runs = _layout(soniq, sub_k=128)                          # PA = 256 and 128
+    assert L.soniq_scale_runs(ctypes.byref(runs)) == 2
+    assert L.soniq_scale_runs(ctypes.byref(_layout(soniq, sub_k=384))) == 1
+    for bad in (_layout(soniq, act_kind=(2, 0)),              # +-1 needs one-bit codes
+                _layout(soniq, act_kind=(3, 0)),
+                _layout(soniq, sub_k=100),
+                _layout(soniq, sub_k=-128)):
+        assert L.soniq_validate_layout(ctypes.byref(bad), pp) == 1
+    assert L.soniq_validate_layout(ctypes.byref(_layout(soniq, act_kind=(2, 0), bits=(1, 8))), pp) == 0
+    assert L.soniq_validate_layout(ctypes.byref(_layout(soniq, act_kind=(1, 0), pad=32)), pp) == 2
+    # staged path only, with its scratch; no GEMV / fused / skinny
+    need = L.soniq_mp_gemm_scratch_bytes(ctypes.byref(runs), 16, 64, 0)
+    assert need > 0
+    assert L.soniq_mp_gemm_path(ctypes.byref(runs), 16, 64, 0, need) == 2
+    assert L.soniq_mp_gemm_path(ctypes.byref(runs), 16, 64, 0, 0) == -1
+    assert L.soniq_mp_gemm_path(ctypes.byref(runs), 16, 64, 16, need) == -1
