@@ -376,7 +376,7 @@ def headline_config(spec, d, world):
 
 def run_suite(args, sq, wl, pk, flush, head):
     """Every workload family, each library call replayed as a CUDA graph after
-    an L2 flush (median of the replays)."""
+    an L2 flush (mean of the replays)."""
     import torch
     stream = torch.cuda.current_stream()
     steps = max(5, args.suite_steps)
@@ -476,7 +476,24 @@ def run_suite(args, sq, wl, pk, flush, head):
                      "fused_codes_only_us": round(codes_ms * 1e3, 2), "codes_identical": same})
 
     linear_case(wl.LINEAR_SMALL)
+    def phase2_case(spec):
+        """Algorithm 1 Phase II forward: every step quantizes both fp32 master
+        weight matrices and the activations on the fly, then runs the GEMMs."""
+        from paper_2311_14114_gb300.phase2 import FakeQuantMLP
+        d = wl.make_phase2(spec)
+        net = FakeQuantMLP(d["layers"], M=spec.M, sub_k=spec.sub_k)
+        X = torch.from_numpy(d["X"]).cuda()
+        step_ms = _time_fn(lambda: net.forward(X), steps, flush, stream)
+        macs = sum(K * N for K, N in zip(spec.widths[:-1], spec.widths[1:])) * spec.M
+        pack_ms = sum(_time_fn(lambda i=i: sq.pack_weights(net.layouts[i], net.W[i], Wp=net.Wp[i], s_w=net.s_w[i]),
+                               steps, flush, stream) for i in range(len(net.layouts)))
+        rows.append({"workload": spec.name, "M": spec.M, "widths": list(spec.widths), "bits": list(spec.bits),
+                     "step_us": round(step_ms * 1e3, 2), "TOPS": round(2 * macs / (step_ms * 1e-3) / 1e12, 2),
+                     "weight_quantize_us": round(pack_ms * 1e3, 2),
+                     "step": "pack both fp32 weight matrices, quantize the activations, GEMM, per layer"})
+
     fused_quant_case(wl.MLP_UP, [2, 8], 0.2)
+    phase2_case(wl.PHASE2_MLP)
     conv_case(wl.CONV_RESNET)
     conv_case(wl.CONV_RESNET_1B4B)
     linear_case(wl.MLP_UP)

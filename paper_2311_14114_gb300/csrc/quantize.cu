@@ -467,13 +467,23 @@ __global__ void __launch_bounds__(128) pack_weights_kernel(const PackWParams p) 
         const float half = (float)(1 << (nb - 1));
         const uint32_t mask = (1u << nb) - 1u;
         const float s = s_sh[g];
+        const float rh = s > 0.0f ? __frcp_rn(s) * half : 0.0f;   // half is a power of two: exact
         uint32_t* dst = reinterpret_cast<uint32_t*>(dst_row + G.w_off);
         for (int kb = warp; kb < G.pw / 32; kb += nwarps) {
             const int pos = kb * 32 + lane;
             const int t = pos / G.pa, c = pos - t * G.pa;
             int32_t j = 0;
-            if (t < p.taps && c < G.count)
-                j = weight_code(__ldg(Wn + (int64_t)t * p.K + p.perm[G.perm_base + c]), s, half);
+            if (t < p.taps && c < G.count && s > 0.0f) {
+                // Eq. (1) from the quotient estimate w * RN(1/s), within a few ulps of
+                // the correctly rounded w / s; |y| = |w / s| 2^(n-1) <= 128, so a y
+                // within 8 ulps of 128 of a half-integer redoes the IEEE division and
+                // every code is the exact rule's
+                const float w = __ldg(Wn + (int64_t)t * p.K + p.perm[G.perm_base + c]);
+                const float y = w * rh;
+                const float k = rintf(y);
+                j = fabsf(fabsf(y - k) - 0.5f) <= 8.0f * 0x1p-16f ? weight_code(w, s, half)
+                                                                 : (int32_t)fminf(fmaxf(k, -half), half - 1.0f);
+            }
             const uint32_t word = pack_block_warp((uint32_t)j & mask, nb);
             if (lane < nb) dst[kb * nb + lane] = word;
         }

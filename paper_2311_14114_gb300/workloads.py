@@ -179,3 +179,40 @@ def random_linear(seed: int, M: int, K: int, N: int, bits_lo: int, bits_hi: int,
     return make_linear(LinearSpec(f"rand_{seed}", M=M, K=K, N=N, bits_lo=bits_lo,
                                   bits_hi=bits_hi, frac_hi=frac_hi, n_outliers=n_outliers,
                                   outlier_scale=outlier_scale, seed=seed))
+
+
+# ---------------------------------------------------------------------------
+# Phase II workload (Algorithm 1, Phase II: quantized fine-tuning): a
+# transformer MLP block (up, then down projection) whose fp32 master weights
+# are quantized on the fly in every step; precisions per channel as Phase I
+# would leave them (about 15 % of the channels at the higher width).
+# ---------------------------------------------------------------------------
+
+@dataclasses.dataclass(frozen=True)
+class Phase2Spec:
+    name: str
+    M: int                      # tokens per step
+    widths: Tuple[int, ...]     # layer widths: input, hidden..., output
+    bits: Tuple[int, int]       # (low, high) bits of every layer
+    frac_hi: float
+    seed: int = 0
+    w_std: float = 0.02
+    sub_k: int = 0              # scale runs along K (0: one scale per group)
+
+
+PHASE2_MLP = Phase2Spec("phase2_mlp_2048x4096x11008x4096_3b6b", M=2048, widths=(4096, 11008, 4096),
+                        bits=(3, 6), frac_hi=0.15)
+
+
+def make_phase2(spec: Phase2Spec, M: Optional[int] = None) -> Dict[str, object]:
+    """Input X fp16 [M][widths[0]] and, per layer, fp32 master weights with
+    their channel permutation and group sizes."""
+    M = spec.M if M is None else M
+    rng = np.random.default_rng(spec.seed)
+    X = rng.standard_normal((M, spec.widths[0]), dtype=np.float32).astype(np.float16)
+    layers = []
+    for K, N in zip(spec.widths[:-1], spec.widths[1:]):
+        perm, count, _ = assignment(rng, K, spec.frac_hi, 0)
+        W = rng.standard_normal((N, K), dtype=np.float32) * np.float32(spec.w_std)
+        layers.append(dict(W=W, perm=perm, count=count, bits=list(spec.bits)))
+    return dict(X=X, layers=layers)
