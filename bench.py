@@ -44,7 +44,9 @@ KERNEL_SOURCES = ("paper_2311_14114_gb300/csrc/staged_gemm.cu", "paper_2311_1411
 # headline workload (its three kernels: activation expand, weight expand,
 # staged tcgen05 GEMM), from one ncu capture, keyed by the sha256 of the
 # kernel sources it was captured with: a different source reports null.
-TRAFFIC = {"sha256": None, "bytes": None, "capture": None}
+TRAFFIC = {"sha256": "3f38aac1f1569f1f023c03033290eaa31ccb796e263e948403ab4f40882988d0",
+           "bytes": 147591168,
+           "capture": "ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum: expand A 21.05 MB, expand W 10.57 MB, staged GEMM 73.73 MB read + 42.22 MB written (one call)"}
 
 
 def peaks():
