@@ -44,9 +44,9 @@ KERNEL_SOURCES = ("paper_2311_14114_gb300/csrc/staged_gemm.cu", "paper_2311_1411
 # headline workload (its three kernels: activation expand, weight expand,
 # staged tcgen05 GEMM), from one ncu capture, keyed by the sha256 of the
 # kernel sources it was captured with: a different source reports null.
-TRAFFIC = {"sha256": "3f38aac1f1569f1f023c03033290eaa31ccb796e263e948403ab4f40882988d0",
-           "bytes": 147591168,
-           "capture": "ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum: expand A 21.05 MB, expand W 10.57 MB, staged GEMM 73.73 MB read + 42.22 MB written (one call)"}
+TRAFFIC = {"sha256": "a9e01004f9e8001145ff8c97136d3d295e86317258bbaa95b711212e5e77579a",
+           "bytes": 148366336,
+           "capture": "ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum: expand A 21.05 MB, expand W 10.57 MB, staged GEMM 73.99 MB read + 42.72 MB written (one call)"}
 
 
 def peaks():
@@ -132,16 +132,31 @@ class ClockSampler:
 # rooflines
 # --------------------------------------------------------------------------
 
-def group_kinds(bits_a, bits_w):
-    """Tensor pipe of each group: 0 = E4M3 (codes <= 4 bits on both sides), 1 = fp16."""
-    return [0 if (a <= 4 and w <= 4) else 1 for a, w in zip(bits_a, bits_w)]
+def group_kinds(bits_a, bits_w, codes=None, N=None):
+    """Tensor pipe of each group on the staged path: 0 = E4M3 (codes <= 4 bits
+    on both sides), 1 = fp16, 2 = E2M1 (codes <= 2 bits on both sides, when such
+    groups hold at least 60 % of the padded weight codes `codes` and 240-column
+    tiles pad N by at most 7 %: the rule the library applies)."""
+    kinds = [0 if (a <= 4 and w <= 4) else 1 for a, w in zip(bits_a, bits_w)]
+    if codes is not None and N is not None and -(-N // 240) * 240 * 100 <= N * 107:
+        elig = [a <= 2 and w <= 2 and c > 0 for a, w, c in zip(bits_a, bits_w, codes)]
+        if 5 * sum(c for c, e in zip(codes, elig) if e) >= 3 * sum(codes):
+            kinds = [2 if e else k for k, e in zip(kinds, elig)]
+    return kinds
+
+
+def padded_codes(count, pad_unit=128, taps=1):
+    """Padded weight codes per group (the staged path's K per group)."""
+    ru = lambda x, u: (x + u - 1) // u * u
+    return [ru(taps * ru(c, pad_unit), 128) if c > 0 else 0 for c in count]
 
 
 def mixed_peak(ops, kinds, pk):
     """Tensor peak for work that runs ops[g] on the pipe of kinds[g] (E4M3 at
-    2x the measured bf16 rate, the nominal fp8:bf16 ratio; fp16 at the bf16
-    rate), time-weighted over the groups."""
-    t = sum(o / (pk["bf16"] * (2.0 if k == 0 else 1.0)) for o, k in zip(ops, kinds) if o > 0)
+    2x the measured bf16 rate and E2M1 at 6x, the nominal fp8:bf16 and
+    fp4:bf16 dense ratios; fp16 at the bf16 rate), time-weighted over the groups."""
+    ratio = {0: 2.0, 1: 1.0, 2: 6.0}
+    t = sum(o / (pk["bf16"] * ratio[k]) for o, k in zip(ops, kinds) if o > 0)
     return sum(ops) / t if t > 0 else pk["bf16"]
 
 
@@ -332,7 +347,7 @@ def run_gpu(args):
     # ---- roofline of the dominant kernel (the tensor-core GEMM) ----
     gemm_avg = statistics.mean(gemm_ms)
     achieved = ops / (gemm_avg * 1e-3) / 1e12
-    kinds = group_kinds(d["bits"], d["bits"])
+    kinds = group_kinds(d["bits"], d["bits"], padded_codes(d["count"]), spec.N)
     peak = mixed_peak(linear_ops(spec.M, spec.N, d["count"]), kinds, pk)
     sha = kernel_sha()
     traffic = TRAFFIC["bytes"] if TRAFFIC["sha256"] == sha else None
@@ -409,7 +424,9 @@ def run_suite(args, sq, wl, pk, flush, head):
             r["weight_bytes_algorithmic"] = int(wbytes)
             r["weight_bytes_moved"] = int(Wp.numel() + s_w.numel() * 4)
         else:
-            peak = mixed_peak(linear_ops(spec.M, spec.N, d["count"]), group_kinds(d["bits"], d["bits"]), pk)
+            staged = sq.gemm_path(lay, spec.M, spec.N).startswith("tensor-core staged")
+            kinds = group_kinds(d["bits"], d["bits"], padded_codes(d["count"]) if staged else None, spec.N)
+            peak = mixed_peak(linear_ops(spec.M, spec.N, d["count"]), kinds, pk)
             r["frac_tensor_peak"] = round(ops / (gemm_ms * 1e-3) / 1e12 / peak, 4)
             r["peak_TFLOPs"] = round(peak, 1)
         rows.append(r)
@@ -427,7 +444,9 @@ def run_suite(args, sq, wl, pk, flush, head):
         ms = _time_fn(lambda: sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y), steps, flush, stream)
         qms = _time_fn(lambda: sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp), steps, flush, stream)
         ops = [2 * spec.M * spec.C_out * spec.R * spec.S * c for c in d["count"]]
-        peak = mixed_peak(ops, group_kinds(d["bits"], d["bits"]), pk)
+        # the bench's convolutions take the staged path (E2M1 where the plan uses it)
+        peak = mixed_peak(ops, group_kinds(d["bits"], d["bits"], padded_codes(d["count"], 32, spec.R * spec.S),
+                                           spec.C_out), pk)
         qb = quant_bytes(spec.batch * spec.H * spec.W, spec.C, d["count"], d["bits"])
         rows.append({"workload": spec.name, "M": spec.M, "N": spec.C_out, "K": spec.K, "bits": d["bits"],
                      "count": d["count"], "conv_us": round(ms * 1e3, 2),

@@ -138,7 +138,7 @@ cudaError_t launch_skinny(const LayoutGeom& geo, const MmaArgs& a, cudaStream_t 
 // (E4M3 bytes for groups with <= 4-bit codes on both sides, fp16 otherwise),
 // then a persistent tcgen05 GEMM runs over them.
 struct StagedGroup {
-    int32_t kind;          // 0: E4M3, 1: fp16
+    int32_t kind;          // 0: E4M3, 1: fp16, 2: E2M1 (kind::mxf4)
     int32_t stages;        // K-stages of the ring (128 bytes of K each)
     int32_t x0;            // byte offset of the group in an expanded row
     int32_t seg_stages;    // K-stages per exact fp32 segment
@@ -149,9 +149,13 @@ struct StagedPlan {
     StagedGroup g[2];
     int64_t eb;            // bytes of an expanded row (both groups)
     int32_t seg_group;     // the group that needs segments, or -1
+    int32_t f4;            // some group runs on E2M1 operands (240-column tiles)
 };
 // False when the layout cannot take the staged path (two segmented groups).
-bool staged_plan(const LayoutGeom& geo, StagedPlan* sp);
+// With allow_f4, groups of <= 2-bit unsigned activations and <= 2-bit weights
+// run on E2M1 operands (their expanded rows are never longer than E4M3 ones,
+// so scratch sized without allow_f4 serves both).
+bool staged_plan(const LayoutGeom& geo, StagedPlan* sp, bool allow_f4 = false);
 // Scratch bytes of the staged path for rows_a activation rows (conv: output
 // pixels) and N weight rows; 0 if the layout cannot take it.
 int64_t staged_scratch_bytes(const LayoutGeom& geo, int64_t rows_a, int64_t N);

@@ -63,7 +63,10 @@ namespace staged {
 using namespace tc;
 
 constexpr int BM = 128;
-constexpr int BN = 256;
+constexpr int BN = 256;                              // tile width (layouts without E2M1 groups)
+constexpr int BN_F4 = 240;                           // tile width of layouts with E2M1 groups
+constexpr int REGION = 256;                          // TMEM columns per accumulator region
+constexpr int SF_COLS = 16;                          // E2M1 scale factors: region columns BN_F4 .. +15
 constexpr int KSTAGE = 128;                          // bytes of K per ring stage (128-byte swizzle)
 constexpr int STAGES = 3;
 constexpr int A_BYTES = BM * KSTAGE;
@@ -87,13 +90,13 @@ constexpr uint32_t IDESC = idesc(BM, BN);
 constexpr long long kTimeoutNs = 2000000000LL;
 
 struct SGroup {
-    int32_t kind;          // 0: E4M3 bytes, 1: fp16
+    int32_t kind;          // 0: E4M3 bytes, 1: fp16, 2: E2M1 nibbles (kind::mxf4)
     int32_t stages;        // 128-byte K-stages of the group
     int32_t x0;            // byte offset of the group in an expanded row
     int32_t seg_stages;    // K-stages per exact segment (segmented group only)
     int32_t n_seg;         // segments (1: accumulated in one piece)
     int32_t center;        // fp16 activations carry -center; the epilogue adds center * C[n]
-    float acc_scale;       // 2^18 (E4M3) or 1 (fp16)
+    float acc_scale;       // 2^18 (E4M3), 1 (fp16) or 4 (E2M1)
     float inv_levels;      // 1 / ((2^na - 1) * 2^(nw - 1))
 };
 
@@ -226,7 +229,19 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
         }
         uint32_t o[8];
         block_to_bytes<N>(words, o);
-        if (kind == 0) {
+        if (kind == 2) {
+            // E2M1, two codes per byte (the first in the low nibble): a code c with
+            // |c| <= 4 is sign << 3 | |c|, the value c / 2
+            uint32_t hw[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                const uint32_t x = ck == 1 ? twos_to_e4m3<N>(o[t]) : o[t];   // sign in bit 7, magnitude below
+                const uint32_t nib = ((x >> 4) & 0x08080808u) | (x & 0x07070707u);
+                const uint32_t y = nib | (nib >> 4);                        // bytes 0 and 2: two codes each
+                hw[t >> 1] |= (__byte_perm(y, 0u, 0x0020u) & 0xFFFFu) << (16 * (t & 1));
+            }
+            *reinterpret_cast<uint4*>(drow + kb * 16) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        } else if (kind == 0) {
             if (ck == 1) {
 #pragma unroll
                 for (int t = 0; t < 8; ++t) o[t] = twos_to_e4m3<N>(o[t]);
@@ -459,7 +474,7 @@ __device__ __noinline__ bool runs_tile(const SParams& p, uint32_t sbase, uint32_
             }
             __syncwarp();
             const float sa = m < p.M ? __ldg(p.s_a + ((p.s_a_per_row ? m : 0) * 2 + g) * p.nb + b) : 0.0f;
-            const uint32_t taddr = lane_base + r * BN;
+            const uint32_t taddr = lane_base + r * REGION;
 #pragma unroll
             for (int cc = 0; cc < EPI_COLS / 8; ++cc) {
                 uint32_t v[8];
@@ -526,8 +541,21 @@ __device__ __noinline__ bool runs_tile(const SParams& p, uint32_t sbase, uint32_
 // accumulators, outputs through TMA stores), which keeps the unrolled output
 // loop small enough for the instruction cache; GENERAL = true handles the
 // rest.  NEXT adds the next layer's codes (quantize-in-epilogue).
-template <bool GENERAL, bool NEXT>
+template <bool GENERAL, bool NEXT, int BNT>
 __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid_constant__ SParams p) {
+    // the tile width and what follows from it (BNT = 240: layouts with E2M1 groups,
+    // whose block scale factors sit in the 16 TMEM columns past each region's tile)
+    constexpr int BN = BNT;
+    constexpr int B_BYTES = BN * KSTAGE;
+    constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    constexpr int EPI_COLS = BN / (NUM_EPI_WARPS / 4);
+    constexpr int SMEM_OUT = STAGES * STAGE_BYTES;
+    constexpr int SMEM_COLS = SMEM_OUT + NUM_EPI_WARPS * OUT_PER_WARP;
+    constexpr int SMEM_BAR = SMEM_COLS + NUM_EPI_WARPS * COLS_PER_WARP;
+    constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;
+    constexpr uint32_t IDESC = idesc(BM, BN);
+    constexpr uint32_t IDESC_F4 = idesc_mxf4(BM, BN);
+    constexpr bool BOX8 = BN != 256;     // outputs leave in 8-column boxes (EPI_COLS is not a multiple of 64)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -563,6 +591,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    if constexpr (BN != REGION) {
+        // the E2M1 block scale factors: UE8M0 2^0 in every byte of each region's
+        // spare columns (one epilogue warp per TMEM lane quadrant)
+        if (warp >= WARP_EPI && warp < WARP_EPI + 4) {
+            const uint32_t lanes = (uint32_t)((warp & 3) * 32) << 16;
+            tmem_st16(tmem_base + lanes + (uint32_t)BN_F4, 0x7F7F7F7Fu);
+            tmem_st16(tmem_base + lanes + (uint32_t)(REGION + BN_F4), 0x7F7F7F7Fu);
+        }
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    }
 
     if (warp == WARP_TMA) {
         // ------------------------------------------------------------ producer
@@ -606,7 +646,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 for (int gi = 0; gi < 2 && ok; ++gi) {
                     const int g = gi == 0 ? g_first : 1 - g_first;
                     const int ns = p.g[g].stages;
-                    const bool f8 = p.g[g].kind == 0;
+                    const bool f8 = p.g[g].kind == 0, f4 = p.g[g].kind == 2;
                     const int per_job = p.g[g].n_seg > 1 ? p.g[g].seg_stages : ns;
 #pragma unroll 1
                     for (int i = 0; i < ns && ok; ++job) {
@@ -617,7 +657,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                             break;
                         }
                         tc_fence_after();
-                        const uint32_t d = tmem_base + r * BN;
+                        const uint32_t d = tmem_base + r * REGION;
                         const int jn = per_job < ns - i ? per_job : ns - i;
 #pragma unroll 1
                         for (int q = 0; q < jn; ++q, ++i, ++s) {
@@ -634,6 +674,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
 #pragma unroll
                                 for (int k = 0; k < KSTAGE / 32; ++k)
                                     mma_f8<IDESC>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
+                            } else if (f4) {
+                                // unit block scales (UE8M0 0x7F = 2^0) in this region's spare columns
+                                const uint32_t sf = d + (uint32_t)BN_F4;
+#pragma unroll
+                                for (int k = 0; k < KSTAGE / 32; ++k)
+                                    mma_f4(d, ad + 2 * k, bd + 2 * k, IDESC_F4, sf, sf + 8u,
+                                           (q == 0 && k == 0) ? 0u : 1u);
                             } else {
 #pragma unroll
                                 for (int k = 0; k < KSTAGE / 32; ++k)
@@ -669,8 +716,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
             const int nc0 = (t / p.m_tiles) * BN + cgrp * EPI_COLS;    // this warp's first column
             __syncwarp();
 #pragma unroll
-            for (int h = 0; h < EPI_COLS / 32; ++h) {
+            for (int h = 0; h < (EPI_COLS + 31) / 32; ++h) {
                 const int c = lane + 32 * h;
+                if (c >= EPI_COLS) break;
                 const int n = nc0 + c < p.N ? nc0 + c : p.N - 1;
                 float4 k;
                 k.x = __ldg(p.s_w + (int64_t)n * 2) * p.g[0].inv_levels;
@@ -686,7 +734,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 sa0 = p.s_a_per_row ? __ldg(p.s_a + m * 2) : __ldg(p.s_a);
                 sa1 = p.s_a_per_row ? __ldg(p.s_a + m * 2 + 1) : __ldg(p.s_a + 1);
             }
-            if constexpr (GENERAL) {
+            if constexpr (GENERAL && BN == REGION) {
                 if (p.runs) {
                     if (!runs_tile(p, sbase, bar0, abort_flag, lane_base, out_s, reinterpret_cast<float*>(colc), lane,
                                    quad, m, m0, nc0, job))
@@ -714,7 +762,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     break;
                 }
                 tc_fence_after();
-                const uint32_t taddr = lane_base + r * BN;
+                const uint32_t taddr = lane_base + r * REGION;
                 if (jj < njobs - 1) {
                     // accumulate: a whole first group, or a segment
                     const int gj = jj < nA ? gA : gB;
@@ -788,9 +836,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                             }
                         }
                         // box cc / 8 (64 columns), row `lane`, 16-byte chunk cc % 8, 128-byte swizzle
-                        // (the TMA store map's layout)
-                        const uint32_t dst = out_s + (uint32_t)(cc >> 3) * 4096u + (uint32_t)lane * 128u +
-                                             ((((uint32_t)cc & 7u) ^ ((uint32_t)lane & 7u)) << 4);
+                        // (the TMA store map's layout); with 8-column boxes, box cc of 32 x 16 bytes
+                        const uint32_t dst =
+                            BOX8 ? out_s + (uint32_t)cc * 512u + (uint32_t)lane * 16u
+                                 : out_s + (uint32_t)(cc >> 3) * 4096u + (uint32_t)lane * 128u +
+                                       ((((uint32_t)cc & 7u) ^ ((uint32_t)lane & 7u)) << 4);
                         asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w[0]), "r"(w[1]),
                                      "r"(w[2]), "r"(w[3])
                                      : "memory");
@@ -804,13 +854,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     mbar_arrive(bar(BAR_REG_EMPTY + r));
                     if (y_tma && write_y) {
                         // rows and columns beyond M and N are clipped by the store
+                        if constexpr (BOX8) {
 #pragma unroll
-                        for (int bx = 0; bx < EPI_COLS / 64; ++bx)
-                            tma_store_2d(&p.tma_y, nc0 + bx * 64, (int)(m0 + quad * 32), out_s + bx * 4096u);
+                            for (int bx = 0; bx < EPI_COLS / 8; ++bx)
+                                tma_store_2d(&p.tma_y, nc0 + bx * 8, (int)(m0 + quad * 32), out_s + bx * 512u);
+                        } else {
+#pragma unroll
+                            for (int bx = 0; bx < EPI_COLS / 64; ++bx)
+                                tma_store_2d(&p.tma_y, nc0 + bx * 64, (int)(m0 + quad * 32), out_s + bx * 4096u);
+                        }
                         bulk_commit();
                     }
                 }
-                if (has_next && m < p.M) next_layer_codes(p, out_s, lane, m, nc0);
+                if constexpr (BN == REGION) {
+                    if (has_next && m < p.M) next_layer_codes(p, out_s, lane, m, nc0);
+                }
             }
         }
         if (((GENERAL || NEXT) ? p.y_tma && p.write_y : true) && lane == 0) bulk_wait0();   // stores complete before the CTA exits
@@ -865,17 +923,38 @@ int64_t align1k(int64_t x) { return (x + 1023) / 1024 * 1024; }
 
 }  // namespace staged
 
-bool staged_plan(const LayoutGeom& geo, StagedPlan* sp) {
+bool staged_plan(const LayoutGeom& geo, StagedPlan* sp, bool allow_f4) {
     int nseg_groups = 0;
     int64_t x0 = 0;
     sp->seg_group = -1;
+    sp->f4 = 0;
     const bool runs = geo.sub_k > 0;
+    // E2M1 pays where its groups hold most of the K codes: the 240-column tiles
+    // it needs cost the other group (measured on the 8192 x 4096 x 4096 sweep:
+    // +20 % with all codes in E2M1 groups, +6 % at 75 %, -5 % at 50 %)
+    if (allow_f4) {
+        int64_t f4_codes = 0, all_codes = 0;
+        for (int g = 0; g < 2; ++g) {
+            const GroupGeom& G = geo.g[g];
+            all_codes += G.pw;
+            if (G.bits_a <= 2 && G.bits_w <= 2 && geo.act_kind[g] == SONIQ_ACT_UNSIGNED && !runs && G.count > 0)
+                f4_codes += G.pw;
+        }
+        if (f4_codes * 5 < all_codes * 3) allow_f4 = false;
+    }
     for (int g = 0; g < 2; ++g) {
         const GroupGeom& G = geo.g[g];
         StagedGroup& S = sp->g[g];
         const int ak = geo.act_kind[g];
         S.kind = (G.bits_a <= 4 && G.bits_w <= 4) ? 0 : 1;
-        const int64_t bytes = (int64_t)G.pw * (S.kind == 0 ? 1 : 2);
+        // E2M1 holds 0, 0.5, 1, 1.5, 2: codes u <= 3 and |j| <= 2 are exact as code / 2
+        if (allow_f4 && G.bits_a <= 2 && G.bits_w <= 2 && ak == SONIQ_ACT_UNSIGNED && !runs && G.count > 0) {
+            S.kind = 2;
+            sp->f4 = 1;
+        }
+        // E2M1 rows: two codes per byte, padded to whole 256-code stages
+        const int64_t bytes = S.kind == 2 ? (((int64_t)G.pw + 255) / 256 * 256) / 2
+                                          : (int64_t)G.pw * (S.kind == 0 ? 1 : 2);
         S.stages = (int32_t)(bytes / staged::KSTAGE);
         S.x0 = (int32_t)x0;
         x0 += bytes;
@@ -887,7 +966,7 @@ bool staged_plan(const LayoutGeom& geo, StagedPlan* sp) {
                                                                                        : (1 << G.bits_a) - 1);
         const int64_t wmax = ak == SONIQ_ACT_PM1 ? 1 : (int64_t)1 << (G.bits_w - 1);
         const int64_t maxprod = amax * wmax;
-        const int64_t codes_per_stage = S.kind == 0 ? staged::KSTAGE : staged::KSTAGE / 2;
+        const int64_t codes_per_stage = S.kind == 2 ? 2 * staged::KSTAGE : (S.kind == 0 ? staged::KSTAGE : staged::KSTAGE / 2);
         int64_t seg_stages = ((int64_t)1 << 24) / maxprod / codes_per_stage;
         if (runs) {
             // one job per run; its exact sum must stay within 2^24
@@ -917,7 +996,12 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
                           cudaStream_t st) {
     using namespace staged;
     StagedPlan sp;
-    if (!staged_plan(geo, &sp)) return cudaErrorNotSupported;
+    // E2M1 groups need 240-column tiles: not with a next layer (its codes are
+    // packed from 64-column output boxes), nor where the narrower tiles would
+    // add more than 7 % of padded columns (N = 256 would take two tiles)
+    const bool f4_ok = a.next == nullptr && (int64_t)((a.N + BN_F4 - 1) / BN_F4) * BN_F4 * 100 <= (int64_t)a.N * 107;
+    if (!staged_plan(geo, &sp, f4_ok)) return cudaErrorNotSupported;
+    const int tile_n = sp.f4 ? BN_F4 : BN;
     const int64_t rows_a = a.M;
     if ((int64_t)scratch_bytes < staged_scratch_bytes(geo, rows_a, a.N) || scratch == nullptr ||
         (uintptr_t)scratch % 256 != 0)
@@ -937,7 +1021,8 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         e.src_off[g] = G.a_off;
         e.dst_off[g] = sp.g[g].x0;
         e.blk_src[g] = G.pa / 32;
-        e.blk_dst[g] = G.pw / 32;
+        // E2M1 groups are written out to whole 256-code stages (zero codes)
+        e.blk_dst[g] = (sp.g[g].kind == 2 ? (G.pw + 255) / 256 * 256 : G.pw) / 32;
         e.center[g] = sp.g[g].center;
         e.cpt[g] = G.pa / 32 > 0 ? G.pa / 32 : 1;
         e.cpt_magic[g] = (((uint64_t)1 << 32) + (uint64_t)e.cpt[g] - 1) / (uint64_t)e.cpt[g];
@@ -991,7 +1076,7 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     memset(&p, 0, sizeof(p));
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;
-    if (!encode_rows(enc, &p.tma_a, xa, sp.eb, rows_a, BM) || !encode_rows(enc, &p.tma_b, xw, sp.eb, a.N, BN))
+    if (!encode_rows(enc, &p.tma_a, xa, sp.eb, rows_a, BM) || !encode_rows(enc, &p.tma_b, xw, sp.eb, a.N, tile_n))
         return cudaErrorInvalidValue;
     p.s_a = a.s_a;
     p.s_w = a.s_w;
@@ -1003,7 +1088,7 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     p.M = a.M;
     p.N = a.N;
     p.m_tiles = (int32_t)((a.M + BM - 1) / BM);
-    p.n_tiles = (a.N + BN - 1) / BN;
+    p.n_tiles = (a.N + tile_n - 1) / tile_n;
     p.total_tiles = p.m_tiles * p.n_tiles;
     p.s_a_per_row = a.s_a_per_row;
     p.out_bf16 = a.out_bf16;
@@ -1027,11 +1112,12 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     if (p.write_y && a.N % 8 == 0 && (uintptr_t)a.Y % 16 == 0) {
         cuuint64_t dims[2] = {(cuuint64_t)a.N, (cuuint64_t)a.M};
         cuuint64_t strides[1] = {(cuuint64_t)a.N * 2};
-        cuuint32_t box[2] = {64u, 32u};
+        // 64 x 32 boxes, 128-byte swizzled; 240-column tiles (120 columns per warp) use 8 x 32 boxes
+        cuuint32_t box[2] = {sp.f4 ? 8u : 64u, 32u};
         cuuint32_t estr[2] = {1, 1};
         if (enc(&p.tma_y, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, a.Y, dims, strides, box, estr,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+                CU_TENSOR_MAP_INTERLEAVE_NONE, sp.f4 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
         p.y_tma = 1;
     }
@@ -1044,7 +1130,7 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         S.seg_stages = sp.g[g].seg_stages;
         S.n_seg = sp.g[g].n_seg;
         S.center = sp.g[g].center;
-        S.acc_scale = S.kind == 0 ? 262144.0f : 1.0f;   // 2^18
+        S.acc_scale = S.kind == 0 ? 262144.0f : (S.kind == 2 ? 4.0f : 1.0f);   // 2^18, 1, or 4 (products u j / 4)
         // decode levels: activations 2^na - 1 (unsigned), 2^(na-1) (signed) or 1 (+-1);
         // weights 2^(nw-1) or 1 (+-1)
         const int ak = geo.act_kind[g];
@@ -1059,12 +1145,14 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     p.nb = geo.nb;
     const bool general =
         a.acc_dbg != nullptr || p.runs || (p.write_y && !p.y_tma) || (!p.write_y && !p.has_next);
-    void (*kern)(SParams) = general ? (p.has_next ? staged_mma_kernel<true, true> : staged_mma_kernel<true, false>)
-                                    : (p.has_next ? staged_mma_kernel<false, true> : staged_mma_kernel<false, false>);
-    static bool attr_done[64][4] = {};
+    void (*kern)(SParams) =
+        sp.f4 ? (general ? staged_mma_kernel<true, false, BN_F4> : staged_mma_kernel<false, false, BN_F4>)
+              : general ? (p.has_next ? staged_mma_kernel<true, true, BN> : staged_mma_kernel<true, false, BN>)
+                        : (p.has_next ? staged_mma_kernel<false, true, BN> : staged_mma_kernel<false, false, BN>);
+    static bool attr_done[64][6] = {};
     int dev = 0;
     cudaGetDevice(&dev);
-    const int kidx = (general ? 2 : 0) + (p.has_next ? 1 : 0);
+    const int kidx = sp.f4 ? 4 + (general ? 1 : 0) : (general ? 2 : 0) + (p.has_next ? 1 : 0);
     if (dev >= 0 && dev < 64 && !attr_done[dev][kidx]) {
         if ((err = cudaFuncSetAttribute((const void*)kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
             cudaSuccess)
