@@ -91,58 +91,78 @@ __global__ void __launch_bounds__(kThreads) absmax_kernel(const T* __restrict__ 
 
 // ---------------------------------------------------------------------------
 // fp16 activations, per-(tensor, group) max |a|.  Each thread owns a fixed
-// 16-byte column of the [rows][K] matrix (8 channels) and walks rows, so the
-// channel-to-group masks are computed once.  |a| is taken on the fp16 bit
-// patterns (sign cleared); for non-negative finite halves the integer order is
-// the float order, so two halves are maxed per instruction (__vmaxu2).  NaN
-// patterns are dropped, as fmaxf drops a NaN operand.
+// 16-byte column of the [rows][K] matrix (8 channels) and walks rows with
+// eight loads in flight, so the channel-to-group masks are computed once.
+// |a| is the fp16 bit pattern with the sign cleared, split by group with
+// those masks, and folded with the fp16x2 maximum, which returns the other
+// operand when one is NaN, as fmaxf does.  keep_l2: the loads carry an L2
+// evict-last policy, so that the quantize pass that follows finds the rows in
+// L2 (it resets the lines' priority as it reads them).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) act_absmax_kernel(const uint4* __restrict__ X, int64_t rows,
-                                                             int32_t K, const int32_t* __restrict__ perm,
-                                                             int32_t count0, unsigned* __restrict__ s_bits) {
+constexpr int kAbsmaxThreads = 512;
+
+__device__ __forceinline__ uint4 ld_nc_policy(const uint4* ptr, uint64_t pol) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(ptr), "l"(pol));
+    return v;
+}
+
+__global__ void __launch_bounds__(kAbsmaxThreads, 4) act_absmax_kernel(const uint4* __restrict__ X, int64_t rows,
+                                                                   int32_t K, const int32_t* __restrict__ perm,
+                                                                   int32_t count0, int32_t keep_l2,
+                                                                   unsigned* __restrict__ s_bits) {
     extern __shared__ uint8_t grp[];   // group of each original channel
     __shared__ float red[64];
-    for (int j = threadIdx.x; j < K; j += blockDim.x) grp[perm[j]] = (uint8_t)(j >= count0);
+    // the permutation's loads issued eight at a time
+    for (int j0 = threadIdx.x; j0 < K; j0 += 8 * kAbsmaxThreads) {
+        int ch[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) ch[u] = j0 + u * kAbsmaxThreads < K ? __ldg(perm + j0 + u * kAbsmaxThreads) : -1;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            if (ch[u] >= 0) grp[ch[u]] = (uint8_t)(j0 + u * kAbsmaxThreads >= count0);
+    }
+    uint64_t pol;
+    if (keep_l2) asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    else asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
     __syncthreads();
     const int KV = K >> 3;                         // 16-byte vectors per row
-    const int cols = KV < kThreads ? KV : kThreads;
-    const int rpar = kThreads / cols;              // rows in flight per CTA
+    const int cols = KV < kAbsmaxThreads ? KV : kAbsmaxThreads;
+    const int rpar = kAbsmaxThreads / cols;        // rows in flight per CTA
     const int tc = threadIdx.x % cols, tr = threadIdx.x / cols;
-    uint32_t g0 = 0u, g1 = 0u;                     // packed half maxima of group 0 / 1
+    __half2 g0 = __float2half2_rn(0.0f), g1 = g0;  // group maxima, two halves each
     if (tr < rpar) {
         for (int j = tc; j < KV; j += cols) {
-            uint32_t m1[4];                        // 0xFFFF in the halves of group-1 channels
+            uint32_t m1[4], m0[4];                 // 0x7FFF in the halves of group-1 / group-0 channels
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-                m1[q] = (grp[8 * j + 2 * q] ? 0x0000FFFFu : 0u) | (grp[8 * j + 2 * q + 1] ? 0xFFFF0000u : 0u);
-            // eight rows' loads in flight before they are reduced
+            for (int q = 0; q < 4; ++q) {
+                m1[q] = (grp[8 * j + 2 * q] ? 0x00007FFFu : 0u) | (grp[8 * j + 2 * q + 1] ? 0x7FFF0000u : 0u);
+                m0[q] = m1[q] ^ 0x7FFF7FFFu;
+            }
             const int64_t rstep = (int64_t)gridDim.x * rpar;
-            for (int64_t m0 = (int64_t)blockIdx.x * rpar + tr; m0 < rows; m0 += 8 * rstep) {
+            for (int64_t m0r = (int64_t)blockIdx.x * rpar + tr; m0r < rows; m0r += 8 * rstep) {
                 uint4 v[8];
 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
-                    const int64_t m = m0 + u * rstep;
-                    v[u] = m < rows ? __ldg(X + m * KV + j) : make_uint4(0u, 0u, 0u, 0u);
+                    const int64_t m = m0r + u * rstep;
+                    v[u] = m < rows ? ld_nc_policy(X + m * KV + j, pol) : make_uint4(0u, 0u, 0u, 0u);
                 }
 #pragma unroll
                 for (int u = 0; u < 8; ++u) {
                     const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
-                        uint32_t x = w[q] & 0x7FFF7FFFu;
-                        x &= __vcmpleu2(x, 0x7C007C00u);          // NaN -> 0
-                        g1 = __vmaxu2(g1, x & m1[q]);
-                        g0 = __vmaxu2(g0, x & ~m1[q]);
+                        uint32_t x1 = w[q] & m1[q], x0 = w[q] & m0[q];
+                        g1 = __hmax2(g1, *reinterpret_cast<__half2*>(&x1));
+                        g0 = __hmax2(g0, *reinterpret_cast<__half2*>(&x0));
                     }
                 }
             }
         }
     }
-    auto hmax = [](uint32_t g) {
-        const uint32_t h = max(g & 0xFFFFu, g >> 16);
-        return __half2float(__ushort_as_half((unsigned short)h));
-    };
-    float mx0 = hmax(g0), mx1 = hmax(g1);
+    float mx0 = fmaxf(__low2float(g0), __high2float(g0)), mx1 = fmaxf(__low2float(g1), __high2float(g1));
     block_max2(mx0, mx1, red);
     if (threadIdx.x == 0) {
         atomicMax(s_bits + 0, __float_as_uint(mx0));
@@ -689,20 +709,21 @@ int grid_for(int64_t work_items, int per_cta) {
 }  // namespace
 
 cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
-                              int64_t M, float* s_out, cudaStream_t st) {
+                              int64_t M, float* s_out, bool keep_l2, cudaStream_t st) {
     cudaError_t e = cudaMemsetAsync(s_out, 0, 2 * sizeof(float), st);
     if (e != cudaSuccess) return e;
     if (geo.K % 8 == 0 && (uintptr_t)A % 16 == 0) {
         const int KV = geo.K / 8;
-        const int rpar = kThreads / (KV < kThreads ? KV : kThreads);
-        // enough CTAs that each thread streams a handful of rows (eight loads in flight)
+        const int rpar = kAbsmaxThreads / (KV < kAbsmaxThreads ? KV : kAbsmaxThreads);
+        // eight rows per thread in flight; a resident grid of four CTAs per SM
         int64_t ctas = (M + 8 * rpar - 1) / (8 * rpar);
-        const int64_t cap = (int64_t)num_sms() * 8;
+        const int64_t cap = (int64_t)num_sms() * 4;
         if (ctas > cap) ctas = cap;
         if (ctas < 1) ctas = 1;
         if ((e = prefer_max_shared((const void*)act_absmax_kernel)) != cudaSuccess) return e;
-        act_absmax_kernel<<<(int)ctas, kThreads, geo.K, st>>>(reinterpret_cast<const uint4*>(A), M, geo.K, perm,
-                                                             geo.g[0].count, reinterpret_cast<unsigned*>(s_out));
+        act_absmax_kernel<<<(int)ctas, kAbsmaxThreads, geo.K, st>>>(reinterpret_cast<const uint4*>(A), M, geo.K,
+                                                                   perm, geo.g[0].count, keep_l2 ? 1 : 0,
+                                                                   reinterpret_cast<unsigned*>(s_out));
     } else {
         const int grid = grid_for(M * (int64_t)geo.K, kThreads * 4);
         absmax_kernel<__half><<<grid, kThreads, geo.K, st>>>(reinterpret_cast<const __half*>(A), M, geo.K, perm,

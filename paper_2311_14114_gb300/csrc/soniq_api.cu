@@ -357,9 +357,16 @@ soniq_status soniq_quantize_act(const soniq_layout* L, const void* A, int64_t M,
             if (e == cudaSuccess) return SONIQ_OK;
             if (e != cudaErrorNotSupported) return cuda_status(e);
         }
-        cudaError_t e = launch_act_absmax(geo, L->perm, A16, M, s_a, s);   // two passes
+    }
+    const bool gather = quantize_gather_supported(geo, scale_mode, A);
+    bool demote = false;
+    if (scale_mode == SONIQ_SCALE_PER_TENSOR) {
+        // two passes; an input that fits in L2 with room to spare stays there between them
+        demote = gather && M * (int64_t)L->K * 2 <= kKeepInL2Bytes;
+        cudaError_t e = launch_act_absmax(geo, L->perm, A16, M, s_a, demote, s);
         if (e != cudaSuccess) return cuda_status(e);
     }
+    if (gather) return cuda_status(launch_quantize_gather(geo, L->perm, A16, M, scale_mode, demote, s_a, Ap, s));
     return cuda_status(launch_quantize_rows(geo, L->perm, A16, M, scale_mode, false, s_a, Ap, s));
 }
 

@@ -50,6 +50,10 @@ constexpr unsigned kErrOneshotBarrier = 4u;   // grid barrier of soniq_quantize_
 // first 256 bytes, then the per-CTA maxima [kMaxGridPartials][2].
 constexpr int kMaxGridPartials = 1024;
 constexpr int64_t kQuantScratchBytes = 256 + 8 * kMaxGridPartials;
+// Per-tensor inputs up to this size are read by the absmax pass with an L2
+// evict-last policy, so that the quantize pass reads them from L2 (the L2
+// holds about 126 MB).
+constexpr int64_t kKeepInL2Bytes = 80ll << 20;
 // True once for the launch that the test hook soniq_test_drop_barrier_arrival armed.
 bool take_drop_arrival();
 void note_launch(int n = 1);
@@ -61,8 +65,10 @@ cudaError_t prefer_max_shared(const void* func);
 
 // ---- launchers (return the CUDA error of the launch) ----------------------
 
+// keep_l2: read with an L2 evict-last policy for a quantize pass that follows
+// with demote set (launch_quantize_gather).
 cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A,
-                              int64_t M, float* s_out, cudaStream_t st);
+                              int64_t M, float* s_out, bool keep_l2, cudaStream_t st);
 // One-pass per-tensor quantize (cooperative launch); its grid barrier (two
 // words, zero between launches) and per-CTA maxima [max_ctas][2] are `bar` and
 // `part`; a barrier wait that runs out ORs `err_bit` into the error word.
@@ -75,6 +81,15 @@ cudaError_t launch_quantize_fused(const LayoutGeom& geo, const int32_t* perm, co
 // per-tensor scale itself (cudaErrorNotSupported if M is too large).
 cudaError_t launch_quantize_rows(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
                                  int32_t scale_mode, bool tensor_in_cta, float* s_a, uint8_t* Ap, cudaStream_t st);
+// Tiled quantize with bulk-staged rows and permutation gathers (rows of
+// 16-byte multiples, 16-byte aligned); scale_mode PER_ROW finds the scales,
+// the other modes read s_a[2].  demote: the rows were read by
+// launch_act_absmax with keep_l2, and their L2 priority is reset here.
+// Returns cudaErrorNotSupported when the layout does not fit it
+// (quantize_gather_supported false).
+bool quantize_gather_supported(const LayoutGeom& geo, int32_t scale_mode, const void* A);
+cudaError_t launch_quantize_gather(const LayoutGeom& geo, const int32_t* perm, const uint16_t* A, int64_t M,
+                                   int32_t scale_mode, bool demote, float* s_a, uint8_t* Ap, cudaStream_t st);
 cudaError_t launch_weight_absmax(const LayoutGeom& geo, const int32_t* perm, const float* W,
                                  int32_t N, float* s_out, cudaStream_t st);
 cudaError_t launch_pack_weights(const LayoutGeom& geo, const int32_t* perm, const float* W,
