@@ -86,6 +86,15 @@ constexpr int SMEM_BAR = SMEM_COLS + NUM_EPI_WARPS * COLS_PER_WARP;
 constexpr int SMEM_MISC = SMEM_BAR + NUM_BARS * 8;   // tmem base, abort flag, a zero word
 constexpr int SMEM_TOTAL = SMEM_MISC + 16;
 constexpr int SMEM_ALLOC = SMEM_TOTAL + 1024;        // slack for 1024-byte alignment
+constexpr int PAIR_STAGES = 4;                       // ring of the 2-SM kernel (32 KB stages)
+
+// Dynamic shared memory of the 2-SM instantiations: the ring, the output
+// staging tile, the column constants, the barriers and misc words, the slack.
+constexpr int pair_smem_alloc() {
+    return PAIR_STAGES * (A_BYTES + BN / 2 * KSTAGE) + NUM_EPI_WARPS * OUT_PER_WARP + NUM_EPI_WARPS * COLS_PER_WARP +
+           (2 * PAIR_STAGES + 5) * 8 + 16 + 1024;
+}
+static_assert(pair_smem_alloc() <= 227 * 1024, "the 2-SM ring fits");
 constexpr uint32_t IDESC = idesc(BM, BN);
 constexpr long long kTimeoutNs = 2000000000LL;
 
@@ -103,6 +112,7 @@ struct SGroup {
 struct SParams {
     CUtensorMap tma_a;     // expanded activations [rows][eb]
     CUtensorMap tma_b;     // expanded weights [N][eb]
+    CUtensorMap tma_b2;    // the same, 128-row boxes (each CTA of a pair loads half the tile's rows)
     CUtensorMap tma_y;     // outputs [M][N] (2-byte elements), 64 x 32 boxes, when y_tma
     const float* s_a;
     const float* s_w;
@@ -113,6 +123,7 @@ struct SParams {
     int64_t M;
     int32_t N;
     int32_t m_tiles, n_tiles, total_tiles;
+    int32_t pair_tiles;    // CTA pairs: (m tile pair, n tile) units, m tile pairs = ceil(m_tiles / 2)
     int32_t s_a_per_row;
     int32_t out_bf16;
     int32_t seg_group;     // group accumulated in drained segments, or -1
@@ -541,14 +552,26 @@ __device__ __noinline__ bool runs_tile(const SParams& p, uint32_t sbase, uint32_
 // accumulators, outputs through TMA stores), which keeps the unrolled output
 // loop small enough for the instruction cache; GENERAL = true handles the
 // rest.  NEXT adds the next layer's codes (quantize-in-epilogue).
-template <bool GENERAL, bool NEXT, int BNT>
+template <bool GENERAL, bool NEXT, int BNT, bool PAIR>
 __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid_constant__ SParams p) {
     // the tile width and what follows from it (BNT = 240: layouts with E2M1 groups,
     // whose block scale factors sit in the 16 TMEM columns past each region's tile)
+    // PAIR: 2-SM MMAs.  CTAs run in clusters of two on a 256 x 256 tile: each
+    // stages its own 128 A rows and its half of the B columns (32 KB per
+    // K-stage instead of 48), the even-rank CTA issues M = 256 MMAs that read
+    // both CTAs' stages, and each CTA's TMEM receives its own 128 rows.  Both
+    // CTAs' operand bytes count on the issuing CTA's full barriers; its MMA
+    // commits arrive on both CTAs' empty and region-full barriers; both CTAs'
+    // epilogue warps arrive on its region-empty barriers.
+    static_assert(!PAIR || BNT == 256, "pairs split 256-column B boxes");
     constexpr int BN = BNT;
-    constexpr int B_BYTES = BN * KSTAGE;
+    constexpr int B_BYTES = (PAIR ? BN / 2 : BN) * KSTAGE;
     constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     constexpr int EPI_COLS = BN / (NUM_EPI_WARPS / 4);
+    constexpr int STAGES = PAIR ? PAIR_STAGES : staged::STAGES;
+    constexpr int BAR_FULL = 0, BAR_EMPTY = STAGES, BAR_REG_FULL = 2 * STAGES, BAR_REG_EMPTY = 2 * STAGES + 2,
+                  BAR_TEARDOWN = 2 * STAGES + 4, NUM_BARS = 2 * STAGES + 5;
+    constexpr uint32_t IDESC2 = idesc(2 * BM, BN);
     constexpr int SMEM_OUT = STAGES * STAGE_BYTES;
     constexpr int SMEM_COLS = SMEM_OUT + NUM_EPI_WARPS * OUT_PER_WARP;
     constexpr int SMEM_BAR = SMEM_COLS + NUM_EPI_WARPS * COLS_PER_WARP;
@@ -566,6 +589,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     const uint32_t abort_flag = smem_u32(smem + SMEM_MISC + 4);
     const uint32_t no_abort = smem_u32(smem + SMEM_MISC + 8);   // stays 0: waits that must run to completion
     const int g_first = first_group(p);
+    if constexpr (PAIR) {
+        // the pair instantiation works with cluster rank 1: outside a cluster
+        // of two it reports the launch as invalid and does nothing
+        if (cluster_size() != 2u) {
+            if (threadIdx.x == 0) atomicOr(p.err, kErrWait);
+            return;
+        }
+    }
+    // the tiles this CTA walks: unit u of first_u, first_u + step_u, ... < n_units
+    const uint32_t rank = PAIR ? cluster_rank() : 0u;
+    const bool issuer = rank == 0u;                   // the CTA that issues the (2-SM) MMAs
+    const int first_u = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const int step_u = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+    const int n_units = PAIR ? p.pair_tiles : p.total_tiles;
+    const int mp = (p.m_tiles + 1) >> 1;
+    auto tile_m = [&](int u) { return PAIR ? 2 * (u % mp) + (int)rank : u % p.m_tiles; };
+    auto tile_n = [&](int u) { return PAIR ? u / mp : u / p.m_tiles; };
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
@@ -574,7 +614,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(BAR_REG_FULL + i), 1);
-            mbar_init(bar(BAR_REG_EMPTY + i), NUM_EPI_WARPS);
+            mbar_init(bar(BAR_REG_EMPTY + i), PAIR ? 2 * NUM_EPI_WARPS : NUM_EPI_WARPS);
         }
         mbar_init(bar(BAR_TEARDOWN), 1);
         set_flag(abort_flag, 0);
@@ -582,14 +622,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == WARP_MMA) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(512)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        if constexpr (PAIR) {
+            // one warp of each CTA of the pair allocates, collectively
+            asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             smem_u32(tmem_slot)),
+                         "r"(512)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+        } else {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             smem_u32(tmem_slot)),
+                         "r"(512)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        }
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // both CTAs' barriers are initialised before the peer's loads or arrivals reach them
+    if constexpr (PAIR) cluster_sync();
     const uint32_t tmem_base = *tmem_slot;
     if constexpr (BN != REGION) {
         // the E2M1 block scale factors: UE8M0 2^0 in every byte of each region's
@@ -609,8 +661,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
         if (lane == 0) {
             uint32_t s = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
-                const int m0 = (t % p.m_tiles) * BM, n0 = (t / p.m_tiles) * BN;
+            for (int u = first_u; u < n_units && ok; u += step_u) {
+                const int m0 = tile_m(u) * BM, n0 = tile_n(u) * BN;
 #pragma unroll 1
                 for (int gi = 0; gi < 2 && ok; ++gi) {
                     const int g = gi == 0 ? g_first : 1 - g_first;
@@ -624,24 +676,37 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                         }
                         if (p.drop_first && s == 0) continue;   // the MMA's wait for it runs out
                         const uint32_t dst = sbase + slot * STAGE_BYTES;
-                        mbar_arrive_expect_tx(bar(BAR_FULL + slot), STAGE_BYTES);
-                        tma_load_2d(dst, &p.tma_a, x0 + i * KSTAGE, m0, bar(BAR_FULL + slot));
-                        tma_load_2d(dst + A_BYTES, &p.tma_b, x0 + i * KSTAGE, n0, bar(BAR_FULL + slot));
+                        if constexpr (PAIR) {
+                            // this CTA's A rows and B half; both CTAs' bytes complete on the
+                            // issuing CTA's full barrier
+                            const uint32_t fb = mapa_shared(bar(BAR_FULL + slot), 0u);
+                            if (issuer) mbar_arrive_expect_tx(bar(BAR_FULL + slot), 2 * STAGE_BYTES);
+                            tma_load_2d_pair(dst, &p.tma_a, x0 + i * KSTAGE, m0, fb);
+                            tma_load_2d_pair(dst + A_BYTES, &p.tma_b2, x0 + i * KSTAGE, n0 + (int)rank * (BN / 2), fb);
+                        } else {
+                            mbar_arrive_expect_tx(bar(BAR_FULL + slot), STAGE_BYTES);
+                            tma_load_2d(dst, &p.tma_a, x0 + i * KSTAGE, m0, bar(BAR_FULL + slot));
+                            tma_load_2d(dst + A_BYTES, &p.tma_b, x0 + i * KSTAGE, n0, bar(BAR_FULL + slot));
+                        }
                     }
                 }
             }
             // loads still in flight must land before the CTA's shared memory is released
-            for (uint32_t q = s > (uint32_t)STAGES ? s - STAGES : 0u; q < s; ++q)
-                if (!(p.drop_first && q == 0))
-                    wait_bounded(bar(BAR_FULL + q % STAGES), (q / STAGES) & 1u, no_abort, kTimeoutNs, p.err, kErrWait);
+            // (a pair's loads all complete on the issuing CTA's barriers; the other CTA
+            // stays until the pair's final cluster barrier)
+            if (!PAIR || issuer)
+                for (uint32_t q = s > (uint32_t)STAGES ? s - STAGES : 0u; q < s; ++q)
+                    if (!(p.drop_first && q == 0))
+                        wait_bounded(bar(BAR_FULL + q % STAGES), (q / STAGES) & 1u, no_abort, kTimeoutNs, p.err,
+                                     kErrWait);
         }
     } else if (warp == WARP_MMA) {
         // ------------------------------------------------------------------ MMA
-        if (lane == 0) {
+        if (lane == 0 && issuer) {
             uint32_t s = 0, job = 0;
             bool ok = true;
             const uint64_t a_desc0 = KSTAGE == 128 ? sw128_desc(sbase) : sw64_desc(sbase);
-            for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
+            for (int u = first_u; u < n_units && ok; u += step_u) {
 #pragma unroll 1
                 for (int gi = 0; gi < 2 && ok; ++gi) {
                     const int g = gi == 0 ? g_first : 1 - g_first;
@@ -670,7 +735,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                             // descriptors of this stage; +32 bytes of K is +2 in the start-address field
                             const uint64_t ad = a_desc0 + (uint64_t)((slot * STAGE_BYTES) >> 4);
                             const uint64_t bd = ad + (uint64_t)(A_BYTES >> 4);
-                            if (f8) {
+                            if (PAIR && f8) {
+#pragma unroll
+                                for (int k = 0; k < KSTAGE / 32; ++k)
+                                    mma2_f8<IDESC2>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
+                            } else if (PAIR) {
+#pragma unroll
+                                for (int k = 0; k < KSTAGE / 32; ++k)
+                                    mma2_f16<IDESC2>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
+                            } else if (f8) {
 #pragma unroll
                                 for (int k = 0; k < KSTAGE / 32; ++k)
                                     mma_f8<IDESC>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
@@ -686,14 +759,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                                 for (int k = 0; k < KSTAGE / 32; ++k)
                                     mma_f16<IDESC>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
                             }
-                            mma_commit(bar(BAR_EMPTY + slot));
+                            // the stage's slot is free again in both CTAs
+                            if constexpr (PAIR) mma2_commit_mc(bar(BAR_EMPTY + slot), (uint16_t)0x3);
+                            else mma_commit(bar(BAR_EMPTY + slot));
                         }
-                        if (ok) mma_commit(bar(BAR_REG_FULL + r));
+                        if (ok) {
+                            if constexpr (PAIR) mma2_commit_mc(bar(BAR_REG_FULL + r), (uint16_t)0x3);
+                            else mma_commit(bar(BAR_REG_FULL + r));
+                        }
                     }
                 }
             }
             // every issued MMA completes before TMEM and shared memory are released
-            mma_commit(bar(BAR_TEARDOWN));
+            if constexpr (PAIR) mma2_commit(bar(BAR_TEARDOWN));
+            else mma_commit(bar(BAR_TEARDOWN));
             wait_bounded(bar(BAR_TEARDOWN), 0u, no_abort, kTimeoutNs, p.err, kErrWait);
         }
     } else {
@@ -709,11 +788,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
         // s_w1 * inv_levels1, center0 * C0, center1 * C1} per column
         float4* colc = reinterpret_cast<float4*>(smem + SMEM_COLS + ew * COLS_PER_WARP);
         const uint32_t out_s = sbase + (uint32_t)(SMEM_OUT + ew * OUT_PER_WARP);   // 1024-aligned
+        // a drained TMEM region goes back to the CTA that issues the MMAs
+        auto release_region = [&](uint32_t r) {
+            if (PAIR && !issuer) mbar_arrive_cluster(mapa_shared(bar(BAR_REG_EMPTY + (int)r), 0u));
+            else mbar_arrive(bar(BAR_REG_EMPTY + (int)r));
+        };
         uint32_t job = 0;
         bool ok = true;
-        for (int t = blockIdx.x; t < p.total_tiles && ok; t += gridDim.x) {
-            const int64_t m0 = (int64_t)(t % p.m_tiles) * BM;
-            const int nc0 = (t / p.m_tiles) * BN + cgrp * EPI_COLS;    // this warp's first column
+        for (int u = first_u; u < n_units && ok; u += step_u) {
+            const int64_t m0 = (int64_t)tile_m(u) * BM;
+            const int nc0 = tile_n(u) * BN + cgrp * EPI_COLS;    // this warp's first column
             __syncwarp();
 #pragma unroll
             for (int h = 0; h < (EPI_COLS + 31) / 32; ++h) {
@@ -776,7 +860,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                     }
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(bar(BAR_REG_EMPTY + r));
+                    if (lane == 0) release_region(r);
                     if (jj == nA - 1 && part_is_other) {
                         // the first group is complete: add back its centring
 #pragma unroll
@@ -851,7 +935,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                 if (staged_out) fence_proxy_async_shared();
                 __syncwarp();
                 if (lane == 0) {
-                    mbar_arrive(bar(BAR_REG_EMPTY + r));
+                    release_region(r);
                     if (y_tma && write_y) {
                         // rows and columns beyond M and N are clipped by the store
                         if constexpr (BOX8) {
@@ -877,8 +961,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // the peer multicasts into this CTA's stages and arrives on its barriers until it is done
+    if constexpr (PAIR) cluster_sync();
     if (warp == WARP_MMA) {
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
+        if constexpr (PAIR)
+            asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
+        else
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
     }
 }
 
@@ -1143,25 +1232,62 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     // TMA stores, or no outputs at all take the general epilogue
     p.runs = geo.sub_k > 0 ? 1 : 0;
     p.nb = geo.nb;
-    const bool general =
-        a.acc_dbg != nullptr || p.runs || (p.write_y && !p.y_tma) || (!p.write_y && !p.has_next);
+    const bool general = a.acc_dbg != nullptr || p.runs || (p.write_y && !p.y_tma) ||
+                         (!p.write_y && !p.has_next) || p.drop_first;
+    // 2-SM pairs on 256 x 256 tiles: the lean epilogue on 256-column tiles (its
+    // instantiation below is the pair one, launched as clusters of two); each
+    // CTA loads 128-row halves of the B tile.  The next-layer epilogue, whose
+    // drain is longer, keeps one CTA per tile: a pair waits for the slower of
+    // its two epilogues before it reuses a TMEM region.
+    const bool pair = !general && !sp.f4 && !p.has_next;
+    p.pair_tiles = ((p.m_tiles + 1) / 2) * p.n_tiles;
+    if (pair && !encode_rows(enc, &p.tma_b2, xw, sp.eb, a.N, tile_n / 2)) return cudaErrorInvalidValue;
     void (*kern)(SParams) =
-        sp.f4 ? (general ? staged_mma_kernel<true, false, BN_F4> : staged_mma_kernel<false, false, BN_F4>)
-              : general ? (p.has_next ? staged_mma_kernel<true, true, BN> : staged_mma_kernel<true, false, BN>)
-                        : (p.has_next ? staged_mma_kernel<false, true, BN> : staged_mma_kernel<false, false, BN>);
+        sp.f4 ? (general ? staged_mma_kernel<true, false, BN_F4, false> : staged_mma_kernel<false, false, BN_F4, false>)
+        : general ? (p.has_next ? staged_mma_kernel<true, true, BN, false> : staged_mma_kernel<true, false, BN, false>)
+                  : (p.has_next ? staged_mma_kernel<false, true, BN, false> : staged_mma_kernel<false, false, BN, true>);
     static bool attr_done[64][6] = {};
+    static int max_pairs[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);
     const int kidx = sp.f4 ? 4 + (general ? 1 : 0) : (general ? 2 : 0) + (p.has_next ? 1 : 0);
-    if (dev >= 0 && dev < 64 && !attr_done[dev][kidx]) {
-        if ((err = cudaFuncSetAttribute((const void*)kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC)) !=
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    const int smem_alloc = pair ? pair_smem_alloc() : SMEM_ALLOC;
+    cfg.blockDim = dim3(NUM_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = smem_alloc;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (!attr_done[dev][kidx]) {
+        if ((err = cudaFuncSetAttribute((const void*)kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_alloc)) !=
             cudaSuccess)
             return err;
         if ((err = prefer_max_shared((const void*)kern)) != cudaSuccess) return err;
+        if (pair) {
+            // pairs that can be resident at once (one CTA per SM)
+            cfg.gridDim = dim3(2 * (unsigned)num_sms() / 2, 1, 1);
+            int n = 0;
+            if ((err = cudaOccupancyMaxActiveClusters(&n, (const void*)kern, &cfg)) != cudaSuccess) return err;
+            max_pairs[dev] = n;
+        }
         attr_done[dev][kidx] = true;
     }
-    const int grid = p.total_tiles < num_sms() ? p.total_tiles : num_sms();
-    kern<<<grid, NUM_THREADS, SMEM_ALLOC, st>>>(p);
+    if (pair) {
+        int pairs = max_pairs[dev];
+        if (pairs < 1) return cudaErrorNotSupported;
+        if (pairs > p.pair_tiles) pairs = p.pair_tiles;
+        cfg.gridDim = dim3(2 * (unsigned)pairs, 1, 1);
+        if ((err = cudaLaunchKernelEx(&cfg, kern, p)) != cudaSuccess) return err;
+    } else {
+        const int grid = p.total_tiles < num_sms() ? p.total_tiles : num_sms();
+        kern<<<grid, NUM_THREADS, smem_alloc, st>>>(p);
+    }
     note_launch();
     return cudaGetLastError();
 }

@@ -85,6 +85,51 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
         : "memory");
 }
 
+// 2-D tiled TMA load into this CTA's shared memory at `dst` whose completion
+// is signalled on `bar`, a shared::cluster address that may lie in the peer
+// CTA of a 2-SM pair (the MMA-issuing CTA counts both CTAs' operand bytes).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2 "
+        "[%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// shared::cluster address of the variable at shared address `addr` in the
+// CTA of cluster rank `rank`.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+// Arrival on an mbarrier of another CTA of the cluster (release at cluster scope).
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// Rank of this CTA in its cluster.
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// CTAs in this CTA's cluster (1 for a launch without clusters).
+__device__ __forceinline__ uint32_t cluster_size() {
+    uint32_t n;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(n));
+    return n;
+}
+
+// Every thread of every CTA of the cluster arrives and waits (release /
+// acquire): shared-memory writes and barrier initialisation before it are
+// visible cluster-wide after it.
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // Contiguous bulk copy global -> shared, completing on `bar` (transaction
 // bytes); both addresses 16-byte aligned, `bytes` a multiple of 16.
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
@@ -169,6 +214,42 @@ __device__ __forceinline__ void mma_f4(uint32_t d_tmem, uint64_t a, uint64_t b, 
 // UE8M0 scale factors (bit 23), scale-factor ids 0, N x M = bn x bm.
 __host__ __device__ constexpr uint32_t idesc_mxf4(int bm, int bn) {
     return (1u << 7) | (1u << 10) | ((uint32_t)(bn >> 3) << 17) | (1u << 23) | ((uint32_t)(bm >> 4) << 24);
+}
+
+// 2-SM MMAs (a CTA pair; issued by one thread of the even-rank CTA): A rows
+// 0..127 and B columns 0..N/2-1 come from this CTA's shared memory at the
+// descriptors' addresses, A rows 128..255 and B columns N/2..N-1 from the peer
+// CTA's at the same addresses; D rows 0..127 go to this CTA's TMEM, rows
+// 128..255 to the peer's, at the same TMEM address.
+template <uint32_t IDESC>
+__device__ __forceinline__ void mma2_f8(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(IDESC), "r"(acc));
+}
+
+template <uint32_t IDESC>
+__device__ __forceinline__ void mma2_f16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(IDESC), "r"(acc));
+}
+
+// Arrives on the mbarrier at offset `bar` of every CTA in `mask` once every
+// 2-SM tcgen05 operation this thread issued so far has completed.
+__device__ __forceinline__ void mma2_commit_mc(uint32_t bar, uint16_t mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            bar),
+        "h"(mask)
+        : "memory");
+}
+
+// Arrives on this CTA's `bar` once every 2-SM tcgen05 operation this thread issued so far has completed.
+__device__ __forceinline__ void mma2_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
 
 // Arrives on `bar` once every tcgen05 operation this thread issued so far has completed.
