@@ -652,7 +652,7 @@ def run_reference(args):
 def run_case(args):
     """One kernel family on one workload, for profiling (ncu) and tuning:
     headline | quant_headline | conv_4b8b | conv_1b4b | quant_conv | mlp_next | mlp_next_codes |
-    gemm:MxNxK:lo:hi:frac | gemv:M."""
+    gemm:MxNxK:lo:hi:frac | quant:MxNxK:lo:hi:frac | gemv:M."""
     import torch
     from paper_2311_14114_gb300 import soniq as sq
     from paper_2311_14114_gb300 import workloads as wl
@@ -673,8 +673,8 @@ def run_case(args):
             fn, ops = (lambda: sq.quantize_act(lay, X, "tensor", s_a=s_a, Ap=Xp)), 0
         else:
             fn, ops = (lambda: sq.mp_conv2d(lay, cd, Xp, s_a, Wp, s_w, Y=Y)), spec.ops
-    elif name.startswith("gemm:") or name in ("headline", "quant_headline"):
-        if name.startswith("gemm:"):
+    elif name.startswith(("gemm:", "quant:")) or name in ("headline", "quant_headline"):
+        if name.startswith(("gemm:", "quant:")):
             _, shape, lo, hi, frac = name.split(":")
             M, N, K = (int(x) for x in shape.split("x"))
             spec = wl.LinearSpec(name, M=M, K=K, N=N, bits_lo=int(lo), bits_hi=int(hi), frac_hi=float(frac))
@@ -686,7 +686,7 @@ def run_case(args):
         A = torch.from_numpy(d["A"]).cuda()
         Ap, s_a = sq.quantize_act(lay, A)
         Y = torch.empty((spec.M, spec.N), dtype=torch.float16, device="cuda")
-        if name == "quant_headline":
+        if name == "quant_headline" or name.startswith("quant:"):
             fn, ops = (lambda: sq.quantize_act(lay, A, "tensor", s_a=s_a, Ap=Ap)), 0
         else:
             fn, ops = (lambda: sq.mp_gemm(lay, Ap, s_a, Wp, s_w, Y=Y, flags=args.flags)), spec.ops

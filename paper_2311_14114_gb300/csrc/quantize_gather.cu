@@ -36,9 +36,9 @@
 namespace soniq {
 namespace {
 
-constexpr int kGatherConsumers = 512;                       // 16 code-forming warps
-constexpr int kGatherConsumerWarps = kGatherConsumers / 32;
-constexpr int kGatherThreads = kGatherConsumers + 32;       // + one producer warp
+constexpr int kGatherConsumerWarps = 20;                    // at most, code-forming warps
+constexpr int kGatherMinConsumerWarps = 8;                  // per-row maxima: one warp per tile row
+constexpr int kGatherThreads = (kGatherConsumerWarps + 1) * 32;   // + one producer warp
 constexpr int kGatherMaxRows = 8;        // rows per tile
 constexpr int kGatherTileRows = 8;       // preferred rows per tile
 constexpr int kGatherMaxStages = 4;      // tiles in the ring (all but one in flight)
@@ -60,7 +60,10 @@ struct GatherParams {
     int32_t row_stride;      // bytes between staged rows (2K + 16, rounded up to 16)
     int32_t nblk0, nblk;     // 32-code blocks of group 0 / of both groups per row
     int32_t bpw;             // 32-code blocks per warp; each warp takes blocks of one group
-    int32_t w0;              // warps 0 .. w0-1 take group 0, the rest group 1
+    int32_t w0;              // block ranges 0 .. w0-1 are of group 0, w0 .. wb-1 of group 1
+    int32_t wb;              // block ranges
+    int32_t rg;              // row groups: warp w takes range w % wb and rows w / wb, + rg, ...
+    int32_t nwc;             // consumer warps (the producer is warp nwc)
     GroupGeom g[2];
 };
 
@@ -148,6 +151,62 @@ __device__ __forceinline__ void row_group_max(const uint8_t* row, const uint32_t
 
 namespace {
 
+// Codes of nc <= 8 consecutive 32-code blocks of one group (positions pos0 +
+// 32 j of this lane) for rows rr0, rr0 + rgs, ... < nr of the tile, into the
+// code buffer.  Absent blocks of a short chunk read the zero slot and skip
+// their stores.  kc:
+// per-row quantizers (MODE 2), kg: the group's quantizer otherwise.
+template <int MODE, int RS>
+__device__ __forceinline__ void codes_chunk8(uint32_t rows_ba, uint32_t codes_a, const uint32_t* offs_s, int pos0, int nc,
+                                             int rr0, int rgs, int nr, uint32_t S, int npos, const GConst (*kc)[2],
+                                             const GConst& kg, int g, float lv, uint32_t zero_slot) {
+    // RS = 1: the warp takes every row of the tile (rr0 = 0); RS = 0: rows rr0 + k rgs
+    const int rstep = RS ? RS : rgs;
+    const int rfirst = RS ? 0 : rr0;
+    uint32_t off[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) off[j] = j < nc ? offs_s[pos0 + 32 * j] : zero_slot;
+#pragma unroll
+    for (int ri = 0; ri < kGatherMaxRows; ++ri) {
+        const int r = rfirst + ri * rstep;
+        if (r < nr) {
+            const uint32_t row = rows_ba + (uint32_t)r * S;
+            const uint32_t crow = codes_a + (uint32_t)(r * npos + pos0);
+            const GConst kk = MODE == 2 ? kc[r][g] : kg;
+            if (kk.mode == 1 && nc == 8) {
+                float a[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) a[j] = lds_half(row + off[j]);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const float q0 = __fmul_rn(a[j], kk.r);
+                    const float q = __fmaf_rn(__fmaf_rn(-q0, kk.s, a[j]), kk.r, q0);
+                    float u = fmaxf(__fmul_rn(q, lv), 0.0f);
+                    if (MODE == 0) u = fminf(u, lv);
+                    sts_u8(crow + 32u * j, __float_as_uint(__fadd_rn(u, 12582912.0f)));
+                }
+            } else if (kk.mode == 1) {
+                float a[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) a[j] = lds_half(row + off[j]);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const float q0 = __fmul_rn(a[j], kk.r);
+                    const float q = __fmaf_rn(__fmaf_rn(-q0, kk.s, a[j]), kk.r, q0);
+                    float u = fmaxf(__fmul_rn(q, lv), 0.0f);
+                    if (MODE == 0) u = fminf(u, lv);
+                    const uint32_t code = __float_as_uint(__fadd_rn(u, 12582912.0f));
+                    if (j < nc) sts_u8(crow + 32u * j, code);
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    if (j < nc) sts_u8(crow + 32u * j, quant_one(lds_half(row + off[j]), kk));
+            }
+        }
+    }
+}
+
 // MODE 0: calibrated scales s_a[2] (codes clip at the top); 1: per-tensor
 // scales s_a[2], the group maxima of these same values; 2: per-(row, group)
 // maxima found here.  With the group maximum as the scale, |a| <= s, so the
@@ -180,14 +239,14 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
     if (tid == 0) {
         for (int b = 0; b < NST; ++b) {
             tc::mbar_init(tc::smem_u32(&full_bar[b]), 1);
-            tc::mbar_init(tc::smem_u32(&empty_bar[b]), kGatherConsumerWarps);
+            tc::mbar_init(tc::smem_u32(&empty_bar[b]), (uint32_t)p.nwc);
         }
         tc::set_flag(abort_flag, 0);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
 
-    if (warp == kGatherConsumerWarps) {
+    if (warp == p.nwc) {
         // ---- producer: one lane streams tiles into the stage ring ----
         if (lane == 0) {
             int b = 0;
@@ -212,14 +271,15 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
         return;
     }
 
-    // ---- consumers (kGatherConsumerWarps warps) ----
-    auto consumer_sync = [] { asm volatile("bar.sync 1, %0;" ::"n"(kGatherConsumers) : "memory"); };
+    // ---- consumers (p.nwc warps) ----
+    const int nthr_c = 32 * p.nwc;
+    auto consumer_sync = [nthr_c] { asm volatile("bar.sync 1, %0;" ::"r"(nthr_c) : "memory"); };
     // offsets: the permutation's loads issued eight at a time
-    for (int q0 = tid; q0 < npos; q0 += 8 * kGatherConsumers) {
+    for (int q0 = tid; q0 < npos; q0 += 8 * nthr_c) {
         int ch[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            const int q = q0 + u * kGatherConsumers;
+            const int q = q0 + u * nthr_c;
             int j = -1;
             if (q < pa0) j = q < c0 ? q : -1;
             else if (q < npos) j = q - pa0 < c1 ? c0 + (q - pa0) : -1;
@@ -227,20 +287,20 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
         }
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            const int q = q0 + u * kGatherConsumers;
+            const int q = q0 + u * nthr_c;
             if (q < npos) offs_s[q] = ch[u] >= 0 ? 2u * (uint32_t)ch[u] : row_bytes;   // padding: the zero slot
         }
     }
     // the zero slot after every staged row (the bulk copies write only the row itself)
-    for (int r = tid; r < NST * TR; r += kGatherConsumers)
+    for (int r = tid; r < NST * TR; r += nthr_c)
         *reinterpret_cast<uint4*>(rows_s + (size_t)r * S + row_bytes) = make_uint4(0u, 0u, 0u, 0u);
     if (MODE == 2) {
-        for (int w = tid; w < K / 2; w += kGatherConsumers) grp_s[w] = 0u;
+        for (int w = tid; w < K / 2; w += nthr_c) grp_s[w] = 0u;
         consumer_sync();
-        for (int j0 = c0 + tid; j0 < K; j0 += 8 * kGatherConsumers) {
+        for (int j0 = c0 + tid; j0 < K; j0 += 8 * nthr_c) {
             int ch[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) ch[u] = j0 + u * kGatherConsumers < K ? __ldg(p.perm + j0 + u * kGatherConsumers) : -1;
+            for (int u = 0; u < 8; ++u) ch[u] = j0 + u * nthr_c < K ? __ldg(p.perm + j0 + u * nthr_c) : -1;
 #pragma unroll
             for (int u = 0; u < 8; ++u)
                 if (ch[u] >= 0) atomicOr(grp_s + (ch[u] >> 1), (ch[u] & 1) ? 0xFFFF0000u : 0x0000FFFFu);
@@ -248,11 +308,14 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
     }
     consumer_sync();
 
-    // this warp's group and its blocks bw0 .. bw0 + nbw - 1 within the group
-    const int g = warp < p.w0 ? 0 : 1;
-    const int bw0 = (g ? warp - p.w0 : warp) * p.bpw;
+    // this warp's group, its blocks bw0 .. bw0 + nbw - 1 within the group, and
+    // its rows rr0, rr0 + rg, ... of each tile (warps past wb * rg stay idle)
+    const bool active = warp < p.wb * p.rg;
+    const int wbi = warp % p.wb, rr0 = warp / p.wb, rgs = p.rg;
+    const int g = wbi < p.w0 ? 0 : 1;
+    const int bw0 = (g ? wbi - p.w0 : wbi) * p.bpw;
     const int nblk_g = g ? p.nblk - p.nblk0 : p.nblk0;
-    const int nbw = max(0, min(p.bpw, nblk_g - bw0));
+    const int nbw = active ? max(0, min(p.bpw, nblk_g - bw0)) : 0;
     const int gbase = g ? pa0 : 0;
     const int bits = p.g[g].bits_a;
     const int a_off = p.g[g].a_off;
@@ -276,7 +339,7 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
             const uint8_t* lo = A8 + m0 * (int64_t)row_bytes;
             const uint8_t* hi = lo + (int64_t)nr * row_bytes;
             const uint8_t* l0 = reinterpret_cast<const uint8_t*>(((uintptr_t)lo + 127u) & ~(uintptr_t)127u);
-            for (const uint8_t* l = l0 + 128 * tid; l < hi && l + 128 <= A_end; l += 128 * kGatherConsumers)
+            for (const uint8_t* l = l0 + 128 * tid; l < hi && l + 128 <= A_end; l += 128 * nthr_c)
                 asm volatile("applypriority.global.L2::evict_normal [%0], 128;" ::"l"(l) : "memory");
         }
         GConst (*kc)[2] = kc_s[it & 1];
@@ -293,41 +356,17 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
             }
             consumer_sync();
         }
-        // ---- codes: lane per packed position; rows outer, up to 8 blocks inner ----
+        // ---- codes: lane per packed position; rows outer, chunks of up to 8 blocks inner ----
         const uint32_t rows_ba = fresh(rows_a + (uint32_t)(b * TR) * S);
         const uint32_t codes_a = tc::smem_u32(codes_s);
         for (int c = 0; c < nbw; c += 8) {
             const int nc = min(8, nbw - c);
-            const int pos0 = gbase + (bw0 + c) * 32 + lane;
-            uint32_t off[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) off[j] = j < nc ? offs_s[pos0 + 32 * j] : row_bytes;
-#pragma unroll
-            for (int r = 0; r < kGatherMaxRows; ++r) {
-                if (r < nr) {
-                    const uint32_t row = rows_ba + (uint32_t)r * S;
-                    const uint32_t crow = codes_a + (uint32_t)(r * npos + pos0);
-                    const GConst kk = MODE == 2 ? kc[r][g] : kg;
-                    if (kk.mode == 1 && nc == 8) {
-                        float a[8];
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) a[j] = lds_half(row + off[j]);
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) {
-                            const float q0 = __fmul_rn(a[j], kk.r);
-                            const float q = __fmaf_rn(__fmaf_rn(-q0, kk.s, a[j]), kk.r, q0);
-                            float u = fmaxf(__fmul_rn(q, lv), 0.0f);
-                            if (MODE == 0) u = fminf(u, lv);
-                            sts_u8(crow + 32u * j, __float_as_uint(__fadd_rn(u, 12582912.0f)));
-                        }
-                    } else {
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) {
-                            if (j < nc) sts_u8(crow + 32u * j, quant_one(lds_half(row + off[j]), kk));
-                        }
-                    }
-                }
-            }
+            if (rgs == 1)
+                codes_chunk8<MODE, 1>(rows_ba, codes_a, offs_s, gbase + (bw0 + c) * 32 + lane, nc, rr0, rgs, nr, S,
+                                      npos, kc, kg, g, lv, row_bytes);
+            else
+                codes_chunk8<MODE, 0>(rows_ba, codes_a, offs_s, gbase + (bw0 + c) * 32 + lane, nc, rr0, rgs, nr, S,
+                                      npos, kc, kg, g, lv, row_bytes);
         }
         __syncwarp();
         // this warp no longer reads the stage's rows
@@ -339,7 +378,7 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
                 const int kbg = bw0 + c + j;
 #pragma unroll
                 for (int h = 0; h < kGatherMaxRows / 4; ++h) {
-                    const int r = (lane >> 3) + 4 * h;
+                    const int r = rr0 + ((lane >> 3) + 4 * h) * rgs;
                     if (r < nr) {
                         const uint4* src = reinterpret_cast<const uint4*>(codes_s + (size_t)r * npos + gbase + kbg * 32);
                         const uint4 lo = src[0], hi = src[1];
@@ -426,11 +465,19 @@ cudaError_t launch_quantize_gather(const LayoutGeom& geo, const int32_t* perm, c
     p.g[1] = geo.g[1];
     p.nblk0 = geo.g[0].pa / 32;
     p.nblk = p.nblk0 + geo.g[1].pa / 32;
+    // block ranges of 8 blocks (whole 8-wide chunks), or of a multiple of 8 where
+    // the row needs more ranges than there are warps; warps left over split
+    // the tile's rows
     const int nblk1 = p.nblk - p.nblk0;
-    for (p.bpw = 1;; ++p.bpw) {
+    for (p.bpw = 8;; p.bpw += 8) {
         p.w0 = (p.nblk0 + p.bpw - 1) / p.bpw;
-        if (p.w0 + (nblk1 + p.bpw - 1) / p.bpw <= kGatherConsumerWarps) break;
+        p.wb = p.w0 + (nblk1 + p.bpw - 1) / p.bpw;
+        if (p.wb <= kGatherConsumerWarps) break;
     }
+    p.rg = kGatherConsumerWarps / p.wb;
+    if (p.rg > pl.tile_rows) p.rg = pl.tile_rows;
+    // exactly the warps that take blocks, and one per tile row at least (per-row maxima)
+    p.nwc = p.wb * p.rg < kGatherMinConsumerWarps ? kGatherMinConsumerWarps : p.wb * p.rg;
     p.row_stride = pl.row_stride;
     const size_t budget = kGatherSmemBudget;
     const int64_t tr = pl.tile_rows;
@@ -452,9 +499,10 @@ cudaError_t launch_quantize_gather(const LayoutGeom& geo, const int32_t* perm, c
     const int64_t ntiles = (M + tr - 1) / tr;
     const int64_t cap = (int64_t)num_sms();
     const int ctas = (int)(ntiles < cap ? ntiles : cap);
-    if (mode == 0) quantize_gather_kernel<0><<<ctas, kGatherThreads, smem, st>>>(p);
-    else if (mode == 1) quantize_gather_kernel<1><<<ctas, kGatherThreads, smem, st>>>(p);
-    else quantize_gather_kernel<2><<<ctas, kGatherThreads, smem, st>>>(p);
+    const int threads = 32 * (p.nwc + 1);
+    if (mode == 0) quantize_gather_kernel<0><<<ctas, threads, smem, st>>>(p);
+    else if (mode == 1) quantize_gather_kernel<1><<<ctas, threads, smem, st>>>(p);
+    else quantize_gather_kernel<2><<<ctas, threads, smem, st>>>(p);
     note_launch();
     return cudaGetLastError();
 }
