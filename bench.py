@@ -135,10 +135,11 @@ class ClockSampler:
 def group_kinds(bits_a, bits_w, codes=None, N=None):
     """Tensor pipe of each group on the staged path: 0 = E4M3 (codes <= 4 bits
     on both sides), 1 = fp16, 2 = E2M1 (codes <= 2 bits on both sides, when such
-    groups hold at least 60 % of the padded weight codes `codes` and 240-column
-    tiles pad N by at most 7 %: the rule the library applies)."""
+    groups hold at least 60 % of the padded weight codes `codes`, the row holds
+    at least 2048 of them, and 240-column tiles pad N by at most 7 %: the rule
+    the library applies)."""
     kinds = [0 if (a <= 4 and w <= 4) else 1 for a, w in zip(bits_a, bits_w)]
-    if codes is not None and N is not None and -(-N // 240) * 240 * 100 <= N * 107:
+    if codes is not None and N is not None and sum(codes) >= 2048 and -(-N // 240) * 240 * 100 <= N * 107:
         elig = [a <= 2 and w <= 2 and c > 0 for a, w, c in zip(bits_a, bits_w, codes)]
         if 5 * sum(c for c, e in zip(codes, elig) if e) >= 3 * sum(codes):
             kinds = [2 if e else k for k, e in zip(kinds, elig)]

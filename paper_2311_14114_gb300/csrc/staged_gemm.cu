@@ -1030,6 +1030,11 @@ bool staged_plan(const LayoutGeom& geo, StagedPlan* sp, bool allow_f4) {
                 f4_codes += G.pw;
         }
         if (f4_codes * 5 < all_codes * 3) allow_f4 = false;
+        // and where K is long enough for the MMAs to dominate: at K = 768 (the
+        // 16384 x 768 -> 3072 MLP layer) the tile's epilogue sets the pace, and
+        // the 240-column epilogue (120 columns per warp, 8-column store boxes)
+        // was 10 % slower than the 256-column one
+        if (all_codes < 2048) allow_f4 = false;
     }
     for (int g = 0; g < 2; ++g) {
         const GroupGeom& G = geo.g[g];
@@ -1234,23 +1239,29 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     p.nb = geo.nb;
     const bool general = a.acc_dbg != nullptr || p.runs || (p.write_y && !p.y_tma) ||
                          (!p.write_y && !p.has_next) || p.drop_first;
-    // 2-SM pairs on 256 x 256 tiles: the lean epilogue on 256-column tiles (its
-    // instantiation below is the pair one, launched as clusters of two); each
-    // CTA loads 128-row halves of the B tile.  The next-layer epilogue, whose
-    // drain is longer, keeps one CTA per tile: a pair waits for the slower of
-    // its two epilogues before it reuses a TMEM region.
-    const bool pair = !general && !sp.f4 && !p.has_next;
+    // 2-SM pairs on 256 x 256 tiles: the lean epilogue on 256-column tiles, for
+    // rows of at least 3072 codes (launched as clusters of two; each CTA loads
+    // 128-row halves of the B tile).  A pair waits for the slower of its two
+    // epilogues before it reuses a TMEM region, so where the epilogue sets the
+    // pace (short K: the K = 768 MLP layer, 123 -> 138 us as pairs; the
+    // K = 2304 conv, even) and for the next-layer epilogue, whose drain is
+    // longer, one CTA takes one tile.
+    int64_t row_codes = 0;
+    for (int g = 0; g < 2; ++g) row_codes += geo.g[g].pw;
+    const bool pair = !general && !sp.f4 && !p.has_next && row_codes >= 3072;
     p.pair_tiles = ((p.m_tiles + 1) / 2) * p.n_tiles;
     if (pair && !encode_rows(enc, &p.tma_b2, xw, sp.eb, a.N, tile_n / 2)) return cudaErrorInvalidValue;
     void (*kern)(SParams) =
         sp.f4 ? (general ? staged_mma_kernel<true, false, BN_F4, false> : staged_mma_kernel<false, false, BN_F4, false>)
         : general ? (p.has_next ? staged_mma_kernel<true, true, BN, false> : staged_mma_kernel<true, false, BN, false>)
-                  : (p.has_next ? staged_mma_kernel<false, true, BN, false> : staged_mma_kernel<false, false, BN, true>);
-    static bool attr_done[64][6] = {};
+                  : p.has_next ? staged_mma_kernel<false, true, BN, false>
+                  : pair       ? staged_mma_kernel<false, false, BN, true>
+                               : staged_mma_kernel<false, false, BN, false>;
+    static bool attr_done[64][7] = {};
     static int max_pairs[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);
-    const int kidx = sp.f4 ? 4 + (general ? 1 : 0) : (general ? 2 : 0) + (p.has_next ? 1 : 0);
+    const int kidx = sp.f4 ? 4 + (general ? 1 : 0) : pair ? 6 : (general ? 2 : 0) + (p.has_next ? 1 : 0);
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];

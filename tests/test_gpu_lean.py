@@ -1,7 +1,8 @@
 """The lean epilogue of the staged tensor-core path: the kernel that runs when
-no debug accumulators are requested (on 256-column tiles, the 2-SM CTA-pair
-kernel: M = 256 MMAs over two CTAs' shared-memory stages, each CTA's TMEM
-holding its own 128 rows).
+no debug accumulators are requested.  On 256-column tiles with rows of at
+least 3072 codes it is the 2-SM CTA-pair kernel (M = 256 MMAs over two CTAs'
+shared-memory stages, each CTA's TMEM holding its own 128 rows); on shorter
+rows, one CTA per tile.
 
 Each case runs one layer twice, with and without `acc_dbg`.  Both epilogues
 evaluate the same fp32 expression from the same exact integer group sums
@@ -71,10 +72,15 @@ def check_lean(sq, d, rows=None, act_mode="tensor", out_dtype=torch.float16, fla
 
 
 @pytest.mark.parametrize("shape,bits,frac", [
-    ((300, 333, 264), (4, 8), 0.3),      # 3 row tiles: the second pair's rank-1 CTA lies past M
-    ((1000, 1000, 600), (2, 8), 0.25),
-    ((513, 700, 1100), (3, 6), 0.5),     # 5 column tiles, the last 76 wide
+    # 2-SM pairs (rows of at least 3072 codes)
+    ((300, 3333, 264), (4, 8), 0.3),     # 3 row tiles: the second pair's rank-1 CTA lies past M
+    ((513, 3100, 1100), (3, 6), 0.5),    # 5 column tiles, the last 76 wide
     ((257, 4096, 512), (4, 4), 0.0),     # one E4M3 group over K = 4096
+    ((384, 4096, 256), (8, 8), 1.0),     # one fp16 group in four exact segments
+    # one CTA per tile (shorter rows)
+    ((300, 333, 264), (4, 8), 0.3),
+    ((1000, 1000, 600), (2, 8), 0.25),
+    ((513, 700, 1100), (3, 6), 0.5),
     ((384, 2048, 256), (8, 8), 1.0),     # one fp16 group in two exact segments
     ((640, 1536, 768), (1, 8), 0.1),
 ])

@@ -29,11 +29,12 @@ def sq():
 
 @pytest.mark.parametrize("bits,frac", [((2, 8), 0.25), ((1, 8), 0.25), ((2, 4), 0.5), ((1, 2), 0.3),
                                        ((2, 2), 0.0), ((1, 6), 0.1), ((2, 6), 1.0), ((2, 4), 0.1)])
-@pytest.mark.parametrize("shape", [(300, 333, 470), (257, 1000, 465)])
+@pytest.mark.parametrize("shape", [(300, 2100, 470), (257, 3000, 465)])
 def test_e2m1_groups(sq, bits, frac, shape):
-    """Ragged M, K (groups not whole 256-code stages) and N (two 240-column
-    tiles, the second partial; widths that 240-column tiles would pad by more
-    than 7 % keep E4M3)."""
+    """Ragged M, K (groups not whole 256-code stages; K of at least 2048 codes,
+    where the library takes E2M1) and N (two 240-column tiles, the second
+    partial; widths that 240-column tiles would pad by more than 7 % keep
+    E4M3)."""
     M, K, N = shape
     d = wl.random_linear(1300 + bits[0] + 10 * bits[1] + K, M=M, K=K, N=N, bits_lo=bits[0], bits_hi=bits[1],
                          frac_hi=frac, n_outliers=2)
@@ -41,7 +42,7 @@ def test_e2m1_groups(sq, bits, frac, shape):
 
 
 def test_e2m1_row_scales_and_bf16(sq):
-    d = wl.random_linear(1350, M=200, K=700, N=480, bits_lo=2, bits_hi=8, frac_hi=0.2)
+    d = wl.random_linear(1350, M=200, K=2200, N=480, bits_lo=2, bits_hi=8, frac_hi=0.2)
     check_linear(sq, d, flags=STAGED, act_mode="row", what="e2m1 row scales")
     check_linear(sq, d, flags=STAGED, out_dtype=torch.bfloat16, what="e2m1 bf16")
 
