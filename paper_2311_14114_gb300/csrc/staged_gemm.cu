@@ -293,24 +293,34 @@ __device__ __forceinline__ void expand_row(const ExpandParams& p, int64_t r, int
     }
 }
 
-__global__ void __launch_bounds__(256) expand_kernel(const __grid_constant__ ExpandParams p) {
+// Item `it` (row it / 2, group it % 2) of one operand.
+__device__ __forceinline__ void expand_item(const ExpandParams& p, int64_t it, int lane) {
+    const int64_t r = it >> 1;
+    const int g = (int)(it & 1);
+    if (p.blk_dst[g] == 0) return;
+    switch (p.bits[g]) {
+        case 1: expand_row<1>(p, r, g, lane); break;
+        case 2: expand_row<2>(p, r, g, lane); break;
+        case 3: expand_row<3>(p, r, g, lane); break;
+        case 4: expand_row<4>(p, r, g, lane); break;
+        case 5: expand_row<5>(p, r, g, lane); break;
+        case 6: expand_row<6>(p, r, g, lane); break;
+        case 7: expand_row<7>(p, r, g, lane); break;
+        default: expand_row<8>(p, r, g, lane); break;
+    }
+}
+
+// Both operands in one launch: items 0 .. 2 rows_a - 1 are (row, group) of the
+// activations (pa), the rest of the weights (pw).
+__global__ void __launch_bounds__(256, 5) expand_kernel(const __grid_constant__ ExpandParams pa,
+                                                     const __grid_constant__ ExpandParams pw) {
     const int lane = threadIdx.x & 31;
     const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    for (int64_t item = warp_id; item < p.rows * 2; item += nwarps) {
-        const int64_t r = item >> 1;
-        const int g = (int)(item & 1);
-        if (p.blk_dst[g] == 0) continue;
-        switch (p.bits[g]) {
-            case 1: expand_row<1>(p, r, g, lane); break;
-            case 2: expand_row<2>(p, r, g, lane); break;
-            case 3: expand_row<3>(p, r, g, lane); break;
-            case 4: expand_row<4>(p, r, g, lane); break;
-            case 5: expand_row<5>(p, r, g, lane); break;
-            case 6: expand_row<6>(p, r, g, lane); break;
-            case 7: expand_row<7>(p, r, g, lane); break;
-            default: expand_row<8>(p, r, g, lane); break;
-        }
+    const int64_t items_a = pa.rows * 2;
+    for (int64_t item = warp_id; item < items_a + pw.rows * 2; item += nwarps) {
+        if (item < items_a) expand_item(pa, item, lane);
+        else expand_item(pw, item - items_a, lane);
     }
 }
 
@@ -1139,11 +1149,6 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         const int64_t cap = (int64_t)num_sms() * 16;
         return (int)(ctas < 1 ? 1 : (ctas > cap ? cap : ctas));
     };
-    expand_kernel<<<grid_for(rows_a * 2), 256, 0, st>>>(e);
-    note_launch();
-    cudaError_t err = cudaGetLastError();
-    if (err != cudaSuccess) return err;
-
     ExpandParams w = e;
     for (int g = 0; g < 2; ++g) {
         const GroupGeom& G = geo.g[g];
@@ -1161,9 +1166,11 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     w.is_weight = 1;
     w.colsum = colsum;
     w.conv = 0;
-    expand_kernel<<<grid_for((int64_t)a.N * 2), 256, 0, st>>>(w);
+    // activations and weights in one launch
+    expand_kernel<<<grid_for(rows_a * 2 + (int64_t)a.N * 2), 256, 0, st>>>(e, w);
     note_launch();
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
 
     // ---- the GEMM ----
     SParams p;
