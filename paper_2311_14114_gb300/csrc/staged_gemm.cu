@@ -573,7 +573,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     // CTAs' operand bytes count on the issuing CTA's full barriers; its MMA
     // commits arrive on both CTAs' empty and region-full barriers; both CTAs'
     // epilogue warps arrive on its region-empty barriers.
-    static_assert(!PAIR || BNT == 256, "pairs split 256-column B boxes");
+    static_assert(!PAIR || (BNT / 2) % 8 == 0, "pairs split B boxes into halves of whole 8-row swizzle atoms");
     constexpr int BN = BNT;
     constexpr int B_BYTES = (PAIR ? BN / 2 : BN) * KSTAGE;
     constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -582,6 +582,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     constexpr int BAR_FULL = 0, BAR_EMPTY = STAGES, BAR_REG_FULL = 2 * STAGES, BAR_REG_EMPTY = 2 * STAGES + 2,
                   BAR_TEARDOWN = 2 * STAGES + 4, NUM_BARS = 2 * STAGES + 5;
     constexpr uint32_t IDESC2 = idesc(2 * BM, BN);
+    constexpr uint32_t IDESC2_F4 = idesc_mxf4(2 * BM, BN);
     constexpr int SMEM_OUT = STAGES * STAGE_BYTES;
     constexpr int SMEM_COLS = SMEM_OUT + NUM_EPI_WARPS * OUT_PER_WARP;
     constexpr int SMEM_BAR = SMEM_COLS + NUM_EPI_WARPS * COLS_PER_WARP;
@@ -650,8 +651,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    // both CTAs' barriers are initialised before the peer's loads or arrivals reach them
-    if constexpr (PAIR) cluster_sync();
     const uint32_t tmem_base = *tmem_slot;
     if constexpr (BN != REGION) {
         // the E2M1 block scale factors: UE8M0 2^0 in every byte of each region's
@@ -665,6 +664,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
         __syncthreads();
         tc_fence_after();
     }
+    // both CTAs' barriers (and scale factors) are in place before the peer's
+    // loads, arrivals or MMAs reach them
+    if constexpr (PAIR) cluster_sync();
 
     if (warp == WARP_TMA) {
         // ------------------------------------------------------------ producer
@@ -745,7 +747,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
                             // descriptors of this stage; +32 bytes of K is +2 in the start-address field
                             const uint64_t ad = a_desc0 + (uint64_t)((slot * STAGE_BYTES) >> 4);
                             const uint64_t bd = ad + (uint64_t)(A_BYTES >> 4);
-                            if (PAIR && f8) {
+                            if (PAIR && f4) {
+                                // unit block scales in the spare columns of this region in both CTAs
+                                const uint32_t sf = d + (uint32_t)BN_F4;
+#pragma unroll
+                                for (int k = 0; k < KSTAGE / 32; ++k)
+                                    mma2_f4(d, ad + 2 * k, bd + 2 * k, IDESC2_F4, sf, sf + 8u, (q == 0 && k == 0) ? 0u : 1u);
+                            } else if (PAIR && f8) {
 #pragma unroll
                                 for (int k = 0; k < KSTAGE / 32; ++k)
                                     mma2_f8<IDESC2>(d, ad + 2 * k, bd + 2 * k, (q == 0 && k == 0) ? 0u : 1u);
@@ -1255,20 +1263,22 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     // longer, one CTA takes one tile.
     int64_t row_codes = 0;
     for (int g = 0; g < 2; ++g) row_codes += geo.g[g].pw;
-    const bool pair = !general && !sp.f4 && !p.has_next && row_codes >= 3072;
+    const bool pair = !general && !p.has_next && row_codes >= 3072;
     p.pair_tiles = ((p.m_tiles + 1) / 2) * p.n_tiles;
     if (pair && !encode_rows(enc, &p.tma_b2, xw, sp.eb, a.N, tile_n / 2)) return cudaErrorInvalidValue;
     void (*kern)(SParams) =
-        sp.f4 ? (general ? staged_mma_kernel<true, false, BN_F4, false> : staged_mma_kernel<false, false, BN_F4, false>)
+        sp.f4 ? (general ? staged_mma_kernel<true, false, BN_F4, false>
+                 : pair  ? staged_mma_kernel<false, false, BN_F4, true>
+                         : staged_mma_kernel<false, false, BN_F4, false>)
         : general ? (p.has_next ? staged_mma_kernel<true, true, BN, false> : staged_mma_kernel<true, false, BN, false>)
                   : p.has_next ? staged_mma_kernel<false, true, BN, false>
                   : pair       ? staged_mma_kernel<false, false, BN, true>
                                : staged_mma_kernel<false, false, BN, false>;
-    static bool attr_done[64][7] = {};
-    static int max_pairs[64] = {};
+    static bool attr_done[64][8] = {};
+    static int max_pairs[64][2] = {};
     int dev = 0;
     cudaGetDevice(&dev);
-    const int kidx = sp.f4 ? 4 + (general ? 1 : 0) : pair ? 6 : (general ? 2 : 0) + (p.has_next ? 1 : 0);
+    const int kidx = sp.f4 ? (pair ? 7 : 4 + (general ? 1 : 0)) : pair ? 6 : (general ? 2 : 0) + (p.has_next ? 1 : 0);
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
@@ -1292,12 +1302,12 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
             cfg.gridDim = dim3(2 * (unsigned)num_sms() / 2, 1, 1);
             int n = 0;
             if ((err = cudaOccupancyMaxActiveClusters(&n, (const void*)kern, &cfg)) != cudaSuccess) return err;
-            max_pairs[dev] = n;
+            max_pairs[dev][sp.f4 ? 1 : 0] = n;
         }
         attr_done[dev][kidx] = true;
     }
     if (pair) {
-        int pairs = max_pairs[dev];
+        int pairs = max_pairs[dev][sp.f4 ? 1 : 0];
         if (pairs < 1) return cudaErrorNotSupported;
         if (pairs > p.pair_tiles) pairs = p.pair_tiles;
         cfg.gridDim = dim3(2 * (unsigned)pairs, 1, 1);

@@ -237,6 +237,18 @@ __device__ __forceinline__ void mma2_f16(uint32_t d_tmem, uint64_t a, uint64_t b
         "l"(a), "l"(b), "r"(IDESC), "r"(acc));
 }
 
+// 2-SM block-scaled MMA on packed E2M1 operands (kind::mxf4, scale_vec::2X):
+// operands and accumulators split over the pair as for mma2_f8; the scale
+// factors are read from TMEM at sfa / sfb.
+__device__ __forceinline__ void mma2_f4(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t sfa,
+                                        uint32_t sfb, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %6, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::mxf4.block_scale.scale_vec::2X [%0], %1, %2, %3, [%4], [%5], p;\n\t}" ::"r"(
+            d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(sfa), "r"(sfb), "r"(acc));
+}
+
 // Arrives on the mbarrier at offset `bar` of every CTA in `mask` once every
 // 2-SM tcgen05 operation this thread issued so far has completed.
 __device__ __forceinline__ void mma2_commit_mc(uint32_t bar, uint16_t mask) {

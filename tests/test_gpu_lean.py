@@ -77,6 +77,10 @@ def check_lean(sq, d, rows=None, act_mode="tensor", out_dtype=torch.float16, fla
     ((513, 3100, 1100), (3, 6), 0.5),    # 5 column tiles, the last 76 wide
     ((257, 4096, 512), (4, 4), 0.0),     # one E4M3 group over K = 4096
     ((384, 4096, 256), (8, 8), 1.0),     # one fp16 group in four exact segments
+    # 2-SM pairs on E2M1 layouts (240-column tiles, 120-row B halves)
+    ((300, 3333, 470), (2, 8), 0.25),    # E2M1 beside fp16, the second column tile partial
+    ((257, 4096, 480), (1, 4), 0.0),     # one E2M1 group
+    ((640, 3500, 960), (2, 4), 0.1),     # E2M1 beside E4M3
     # one CTA per tile (shorter rows)
     ((300, 333, 264), (4, 8), 0.3),
     ((1000, 1000, 600), (2, 8), 0.25),
