@@ -14,6 +14,7 @@
 
 #include "soniq_device.cuh"
 #include "soniq_internal.h"
+#include "tc_ptx.cuh"
 
 namespace soniq {
 namespace {
@@ -115,6 +116,11 @@ __global__ void __launch_bounds__(kAbsmaxThreads, 4) act_absmax_kernel(const uin
                                                                    unsigned* __restrict__ s_bits) {
     extern __shared__ uint8_t grp[];   // group of each original channel
     __shared__ float red[64];
+    // launched after the previous kernel's start (launch_pdl): its outputs are
+    // visible past this wait; one wave of CTAs, so the quantize pass that
+    // follows may be scheduled at once
+    tc::pdl_wait();
+    tc::pdl_trigger();
     // the permutation's loads issued eight at a time
     for (int j0 = threadIdx.x; j0 < K; j0 += 8 * kAbsmaxThreads) {
         int ch[8];
@@ -721,9 +727,10 @@ cudaError_t launch_act_absmax(const LayoutGeom& geo, const int32_t* perm, const 
         if (ctas > cap) ctas = cap;
         if (ctas < 1) ctas = 1;
         if ((e = prefer_max_shared((const void*)act_absmax_kernel)) != cudaSuccess) return e;
-        act_absmax_kernel<<<(int)ctas, kAbsmaxThreads, geo.K, st>>>(reinterpret_cast<const uint4*>(A), M, geo.K,
-                                                                   perm, geo.g[0].count, keep_l2 ? 1 : 0,
-                                                                   reinterpret_cast<unsigned*>(s_out));
+        if ((e = launch_pdl(act_absmax_kernel, dim3((unsigned)ctas), dim3(kAbsmaxThreads), (size_t)geo.K, st,
+                            reinterpret_cast<const uint4*>(A), M, geo.K, perm, geo.g[0].count, keep_l2 ? 1 : 0,
+                            reinterpret_cast<unsigned*>(s_out))) != cudaSuccess)
+            return e;
     } else {
         const int grid = grid_for(M * (int64_t)geo.K, kThreads * 4);
         absmax_kernel<__half><<<grid, kThreads, geo.K, st>>>(reinterpret_cast<const __half*>(A), M, geo.K, perm,

@@ -245,6 +245,11 @@ __global__ void __launch_bounds__(kGatherThreads, 1) quantize_gather_kernel(cons
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
+    // launched after the previous kernel's start (launch_pdl): every global
+    // access comes after this wait; one wave of CTAs, so the kernel that
+    // follows may be scheduled at once
+    tc::pdl_wait();
+    tc::pdl_trigger();
 
     if (warp == p.nwc) {
         // ---- producer: one lane streams tiles into the stage ring ----
@@ -499,10 +504,11 @@ cudaError_t launch_quantize_gather(const LayoutGeom& geo, const int32_t* perm, c
     const int64_t ntiles = (M + tr - 1) / tr;
     const int64_t cap = (int64_t)num_sms();
     const int ctas = (int)(ntiles < cap ? ntiles : cap);
-    const int threads = 32 * (p.nwc + 1);
-    if (mode == 0) quantize_gather_kernel<0><<<ctas, threads, smem, st>>>(p);
-    else if (mode == 1) quantize_gather_kernel<1><<<ctas, threads, smem, st>>>(p);
-    else quantize_gather_kernel<2><<<ctas, threads, smem, st>>>(p);
+    const dim3 grid((unsigned)ctas), block((unsigned)(32 * (p.nwc + 1)));
+    cudaError_t e = mode == 0   ? launch_pdl(quantize_gather_kernel<0>, grid, block, smem, st, p)
+                    : mode == 1 ? launch_pdl(quantize_gather_kernel<1>, grid, block, smem, st, p)
+                                : launch_pdl(quantize_gather_kernel<2>, grid, block, smem, st, p);
+    if (e != cudaSuccess) return e;
     note_launch();
     return cudaGetLastError();
 }

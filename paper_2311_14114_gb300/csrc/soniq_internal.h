@@ -63,6 +63,24 @@ int num_sms();
 // consecutive calls do not make the SMs reconfigure between kernels.
 cudaError_t prefer_max_shared(const void* func);
 
+// Launches `kernel` with programmatic stream serialization: it may start (and
+// run up to its pdl_wait) while the previous kernel in the stream finishes.
+template <typename... Params, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // ---- launchers (return the CUDA error of the launch) ----------------------
 
 // keep_l2: read with an L2 evict-last policy for a quantize pass that follows

@@ -314,6 +314,7 @@ __device__ __forceinline__ void expand_item(const ExpandParams& p, int64_t it, i
 // activations (pa), the rest of the weights (pw).
 __global__ void __launch_bounds__(256, 5) expand_kernel(const __grid_constant__ ExpandParams pa,
                                                      const __grid_constant__ ExpandParams pw) {
+    tc::pdl_wait();   // launched with launch_pdl: the packed rows are written before this
     const int lane = threadIdx.x & 31;
     const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -667,6 +668,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) staged_mma_kernel(const __grid
     // both CTAs' barriers (and scale factors) are in place before the peer's
     // loads, arrivals or MMAs reach them
     if constexpr (PAIR) cluster_sync();
+    // launched with launch_pdl: the expanded operands and weight sums are
+    // written before this (the prologue above touches no global memory)
+    pdl_wait();
 
     if (warp == WARP_TMA) {
         // ------------------------------------------------------------ producer
@@ -1175,9 +1179,9 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     w.colsum = colsum;
     w.conv = 0;
     // activations and weights in one launch
-    expand_kernel<<<grid_for(rows_a * 2 + (int64_t)a.N * 2), 256, 0, st>>>(e, w);
+    cudaError_t err = launch_pdl(expand_kernel, dim3((unsigned)grid_for(rows_a * 2 + (int64_t)a.N * 2)), dim3(256), 0,
+                                 st, e, w);
     note_launch();
-    cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
 
     // ---- the GEMM ----
@@ -1281,11 +1285,13 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
     const int kidx = sp.f4 ? (pair ? 7 : 4 + (general ? 1 : 0)) : pair ? 6 : (general ? 2 : 0) + (p.has_next ? 1 : 0);
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     const int smem_alloc = pair ? pair_smem_alloc() : SMEM_ALLOC;
     cfg.blockDim = dim3(NUM_THREADS, 1, 1);
     cfg.dynamicSmemBytes = smem_alloc;
@@ -1311,10 +1317,13 @@ cudaError_t launch_staged(const LayoutGeom& geo, const MmaArgs& a, void* scratch
         if (pairs < 1) return cudaErrorNotSupported;
         if (pairs > p.pair_tiles) pairs = p.pair_tiles;
         cfg.gridDim = dim3(2 * (unsigned)pairs, 1, 1);
+        cfg.numAttrs = 2;
         if ((err = cudaLaunchKernelEx(&cfg, kern, p)) != cudaSuccess) return err;
     } else {
         const int grid = p.total_tiles < num_sms() ? p.total_tiles : num_sms();
-        kern<<<grid, NUM_THREADS, smem_alloc, st>>>(p);
+        if ((err = launch_pdl(kern, dim3((unsigned)grid), dim3(NUM_THREADS), (size_t)smem_alloc, st, p)) !=
+            cudaSuccess)
+            return err;
     }
     note_launch();
     return cudaGetLastError();

@@ -116,6 +116,14 @@ __device__ __forceinline__ uint32_t cluster_rank() {
     return r;
 }
 
+// Programmatic dependent launch.  pdl_wait: returns once every grid this one
+// depends on has completed and its memory is visible (at once for a launch
+// without the attribute); every global access of a kernel launched with
+// launch_pdl comes after it.  pdl_trigger: this CTA lets the grids that
+// depend on this one be scheduled before it completes.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // CTAs in this CTA's cluster (1 for a launch without clusters).
 __device__ __forceinline__ uint32_t cluster_size() {
     uint32_t n;
