@@ -195,6 +195,23 @@ __device__ __forceinline__ void quarter_codes(const uint4 x, int valid, const QC
     }
 }
 
+// pos_s[perm[j]] = staged position of logical channel j (group 0 first, then
+// group 1 from pa0), by the whole block; the permutation's loads are issued
+// four at a time.
+__device__ __forceinline__ void build_positions(uint16_t* pos_s, const int32_t* __restrict__ perm, int K, int c0,
+                                                int pa0) {
+    for (int j0 = threadIdx.x; j0 < K; j0 += 4 * blockDim.x) {
+        int ch[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) ch[u] = j0 + u * (int)blockDim.x < K ? __ldg(perm + j0 + u * blockDim.x) : -1;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int j = j0 + u * (int)blockDim.x;
+            if (ch[u] >= 0) pos_s[ch[u]] = (uint16_t)(j < c0 ? j : pa0 + (j - c0));
+        }
+    }
+}
+
 // ---------------------------------------------------------------------------
 // Per-tensor scales in one pass over the input (a cooperative launch, all
 // CTAs resident): each CTA stages its rows in shared memory (permuted and
@@ -275,7 +292,7 @@ __global__ void __launch_bounds__(1024) quantize_fused_kernel(const FusedParams 
     __shared__ int abort_s;
     const int RH = p.row_halves;
     const int c0 = p.g[0].count, pa0 = p.g[0].pa;
-    for (int j = threadIdx.x; j < p.K; j += blockDim.x) pos_s[p.perm[j]] = (uint16_t)(j < c0 ? j : pa0 + (j - c0));
+    build_positions(pos_s, p.perm, p.K, c0, pa0);
     if (threadIdx.x == 0) abort_s = 0;
     __syncthreads();
 
@@ -584,7 +601,7 @@ __global__ void __launch_bounds__(kTileThreads, 1) quantize_tiles_kernel(const T
     __shared__ float red[64];
     const int RH = p.row_halves, TR = p.tile_rows;
     const int c0 = p.g[0].count, pa0 = p.g[0].pa;
-    for (int j = threadIdx.x; j < p.K; j += blockDim.x) pos_s[p.perm[j]] = (uint16_t)(j < c0 ? j : pa0 + (j - c0));
+    build_positions(pos_s, p.perm, p.K, c0, pa0);
     {
         uint4* z = reinterpret_cast<uint4*>(rows_s);
         for (int i = threadIdx.x; i < TR * RH / 8; i += blockDim.x) z[i] = make_uint4(0u, 0u, 0u, 0u);
