@@ -601,19 +601,6 @@ __global__ void __launch_bounds__(kTileThreads, 1) quantize_tiles_kernel(const T
     __shared__ float red[64];
     const int RH = p.row_halves, TR = p.tile_rows;
     const int c0 = p.g[0].count, pa0 = p.g[0].pa;
-    build_positions(pos_s, p.perm, p.K, c0, pa0);
-    {
-        uint4* z = reinterpret_cast<uint4*>(rows_s);
-        for (int i = threadIdx.x; i < TR * RH / 8; i += blockDim.x) z[i] = make_uint4(0u, 0u, 0u, 0u);
-    }
-    const bool per_row = p.scale_mode == SONIQ_SCALE_PER_ROW;
-    QConst k0, k1;
-    if (!per_row && !p.tensor_in_cta) {
-        k0 = make_qconst(p.s_a[0], p.g[0].bits_a);
-        k1 = make_qconst(p.s_a[1], p.g[1].bits_a);
-    }
-    __syncthreads();
-    const uint32_t rows_a = (uint32_t)__cvta_generic_to_shared(rows_s);
     const int KV = p.K >> 3;
     const int64_t tstep = (int64_t)gridDim.x * TR;
     // staging map: vector v of a tile is row v / KV, column v % KV; this thread
@@ -629,6 +616,22 @@ __global__ void __launch_bounds__(kTileThreads, 1) quantize_tiles_kernel(const T
             if (v < tile_vecs && v < nr * KV) nxt[u] = __ldg(src + v);
         }
     };
+    // the first tile's loads are in flight while the permutation table is built
+    int64_t m0 = (int64_t)blockIdx.x * TR;
+    if (p.vec_ok && m0 < p.M) load_tile(m0);
+    build_positions(pos_s, p.perm, p.K, c0, pa0);
+    {
+        uint4* z = reinterpret_cast<uint4*>(rows_s);
+        for (int i = threadIdx.x; i < TR * RH / 8; i += blockDim.x) z[i] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    const bool per_row = p.scale_mode == SONIQ_SCALE_PER_ROW;
+    QConst k0, k1;
+    if (!per_row && !p.tensor_in_cta) {
+        k0 = make_qconst(p.s_a[0], p.g[0].bits_a);
+        k1 = make_qconst(p.s_a[1], p.g[1].bits_a);
+    }
+    __syncthreads();
+    const uint32_t rows_a = (uint32_t)__cvta_generic_to_shared(rows_s);
     auto store_tile = [&](int64_t m0) {
         const int nr = p.M - m0 < TR ? (int)(p.M - m0) : TR;
 #pragma unroll
@@ -648,8 +651,6 @@ __global__ void __launch_bounds__(kTileThreads, 1) quantize_tiles_kernel(const T
             }
         }
     };
-    int64_t m0 = (int64_t)blockIdx.x * TR;
-    if (p.vec_ok && m0 < p.M) load_tile(m0);
     for (; m0 < p.M; m0 += tstep) {
         const int nr = p.M - m0 < TR ? (int)(p.M - m0) : TR;
         // ---- stage this tile (from the registers), then start the next tile's loads ----
