@@ -6,14 +6,16 @@
 // producer warp copies each row of a tile into a ring of shared-memory stages
 // with one bulk copy (rows stay in their original channel order; a 16-byte
 // zero slot after every row stands in for the padding positions); a stage is
-// refilled as soon as the 16 consumer warps have released it through its
-// "empty" mbarrier, so no CTA-wide barrier sits in the tile loop.  Codes are
-// formed one lane per packed position: each consumer warp owns a contiguous
-// range of 32-code blocks of one precision group (its quantizer constants are
-// warp-uniform), holds the staged-row byte offsets of its lanes' channels,
-// and walks the tile's rows with up to 8 independent gathers per row, so
-// every gather instruction reads one row (conflict-free where the permutation
-// keeps channels in order, as it does within each group).  The code lands as
+// refilled as soon as the consumer warps (up to 20, as many as the layout's
+// block ranges need) have released it through its "empty" mbarrier, so no
+// CTA-wide barrier sits in the tile loop.  Codes are formed one lane per
+// packed position: each consumer warp owns a contiguous range of whole
+// 8-block chunks of one precision group (its quantizer constants are
+// warp-uniform) and, where warps are left over, a share of the tile's rows;
+// it holds the staged-row byte offsets of its lanes' channels and walks its
+// rows with up to 8 independent gathers per row, so every gather instruction
+// reads one row (conflict-free where the permutation keeps channels in order,
+// as it does within each group).  The code lands as
 // one byte in a per-tile code buffer; after a warp barrier each lane packs
 // whole 32-code blocks of that warp and stores them with 16-byte stores.
 //
