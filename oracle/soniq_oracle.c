@@ -119,7 +119,9 @@ void orc_weight_scales(const float *W, int32_t N, int32_t taps, int32_t K,
 /* ------------------------------------------------------------------------- */
 /* a3a Unsigned activation code, Sec. 3 step 2:                              */
 /*     b = clip(round(a / s_g * (2^n - 1)), 0, 2^n - 1)                      */
-/* A zero scale (all-zero group) gives code 0.                               */
+/* A zero scale (all-zero group) gives code 0.  Non-finite inputs: the clip  */
+/* takes +inf to 2^n - 1 and -inf to 0; a NaN quotient (a NaN input, or      */
+/* inf / inf) lies on neither side of the clip and is read as code 0.        */
 /* ------------------------------------------------------------------------- */
 int32_t orc_act_code(float a, float s, int32_t n) {
     if (!(s > 0.0f)) return 0;
@@ -127,6 +129,7 @@ int32_t orc_act_code(float a, float s, int32_t n) {
     float q = a / s;           /* fp32, IEEE division */
     float t = q * levels;      /* fp32 multiply, no fused op */
     float r = rintf(t);        /* round half to even */
+    if (isnan(r)) return 0;
     if (r < 0.0f) r = 0.0f;
     if (r > levels) r = levels;
     return (int32_t)r;
@@ -136,6 +139,8 @@ int32_t orc_act_code(float a, float s, int32_t n) {
 /* a3b Signed weight code, Sec. 3 step 3 and Eq. (1): the nearest n-bit      */
 /*     two's-complement fraction q = j / 2^(n-1), j in [-2^(n-1), 2^(n-1)-1], */
 /*     to w' = w / s_g (ties to even j).  Multiplying w' by 2^(n-1) is exact.*/
+/*     Non-finite inputs as for activations: +-inf clip to the end levels, a  */
+/*     NaN quotient is read as code 0.                                        */
 /* ------------------------------------------------------------------------- */
 int32_t orc_weight_code(float w, float s, int32_t n) {
     if (!(s > 0.0f)) return 0;
@@ -143,6 +148,7 @@ int32_t orc_weight_code(float w, float s, int32_t n) {
     float wp = w / s;
     float t = wp * half_range;
     float r = rintf(t);
+    if (isnan(r)) return 0;
     if (r < -half_range) r = -half_range;
     if (r > half_range - 1.0f) r = half_range - 1.0f;
     return (int32_t)r;

@@ -174,6 +174,43 @@ def test_scales_equal_numpy_max_abs():
     assert (swt[:, 1] == np.abs(d["W"][:, g1]).max()).all()
 
 
+@pytest.mark.parametrize("n", range(1, 9))
+def test_non_finite_inputs_follow_the_clip(n):
+    """Sec. 3 steps 2-3 clip the rounded level to the code range: +inf lands on
+    the top code, -inf on the bottom one, whatever the (finite, positive)
+    scale; a NaN quotient (a NaN input, or inf / inf under an infinite scale)
+    lies on neither side of the clip and is read as code 0."""
+    top_a, lo_w, top_w = 2 ** n - 1, -(2 ** (n - 1)), 2 ** (n - 1) - 1
+    nan, inf = float("nan"), float("inf")
+    for s in (1e-30, 0.37, 1.0, 3e4, 1e30):
+        assert oracle.act_code(inf, s, n) == top_a and oracle.act_code(-inf, s, n) == 0
+        assert oracle.act_code(nan, s, n) == 0
+        assert oracle.weight_code(inf, s, n) == top_w and oracle.weight_code(-inf, s, n) == lo_w
+        assert oracle.weight_code(nan, s, n) == 0
+    # an infinite scale (a group holding an infinity): finite inputs give 0, inf / inf is NaN
+    for x in (0.0, 1.0, -65504.0, 65504.0, inf, -inf, nan):
+        assert oracle.act_code(x, inf, n) == 0 and oracle.weight_code(x, inf, n) == 0
+
+
+def test_scales_drop_nan_and_keep_inf():
+    """max |a| as numpy's nanmax: NaN never becomes a scale, an infinity does."""
+    d = wl.random_linear(8, M=6, K=96, N=5, bits_lo=2, bits_hi=8, frac_hi=0.25)
+    A, W, perm, count = d["A"].astype(np.float32), d["W"].copy(), d["perm"], d["count"]
+    g0, g1 = perm[:count[0]], perm[count[0]:]
+    A[1, g0[3]] = np.nan
+    A[2, g1[0]] = -np.inf
+    W[0, g0[1]] = np.nan
+    W[3, g1[2]] = np.inf
+    sr = oracle.act_scales(A, perm, count, per_row=True)
+    assert (sr[:, 0] == np.nanmax(np.abs(A[:, g0]), 1)).all()
+    assert (sr[:, 1] == np.nanmax(np.abs(A[:, g1]), 1)).all()
+    assert sr[2, 1] == np.inf and np.isfinite(sr[1, 0])
+    s = oracle.act_scales(A, perm, count)
+    assert s[0] == np.nanmax(np.abs(A[:, g0])) and s[1] == np.inf
+    sw = oracle.weight_scales(W, perm, count)
+    assert (sw[:, 0] == np.nanmax(np.abs(W[:, g0]), 1)).all() and sw[3, 1] == np.inf
+
+
 # ---------------------------------------------------------------------------
 # Packing.
 # ---------------------------------------------------------------------------
