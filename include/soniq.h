@@ -222,7 +222,9 @@ SONIQ_API int64_t soniq_launch_count(void);
  * Weight quantize-and-pack (offline, once per layer).  Sec. 3 steps 1 and 3,
  * Eq. (1): per scale group s = max|w|, w' = w / s (fp32, IEEE), code
  * j = clamp(round_half_even(w' * 2^(n-1)), -2^(n-1), 2^(n-1) - 1), the nearest
- * level of Eq. (1); s = 0 gives j = 0.
+ * level of Eq. (1); s = 0 gives j = 0.  Non-finite weights: the max-abs scale
+ * skips NaN and keeps infinities (a group holding one gets s = inf, and every
+ * code of it is 0); a NaN w' (a NaN weight, or inf / inf) gives j = 0.
  *
  *   W          device fp32 [N][taps][K] (taps = 1: a linear layer [N][K];
  *              a convolution OHWI [C_out][R*S][C_in]), 4-byte aligned.
@@ -243,7 +245,10 @@ SONIQ_API soniq_status soniq_pack_weights(const soniq_layout *layout, const floa
  * Activation quantize-and-pack (per inference call).  Sec. 3 steps 1 and 2:
  * s = max|a| per scale group, code u = clip(round_half_even(fp32(a / s) *
  * (2^n - 1)), 0, 2^n - 1); s = 0 gives u = 0.  Channels are gathered through
- * layout->perm and each group is zero-padded to PA_g codes.
+ * layout->perm and each group is zero-padded to PA_g codes.  Non-finite
+ * inputs: under a finite scale +inf clips to 2^n - 1 and -inf to 0; a NaN
+ * quotient (a NaN input, or inf / inf) gives u = 0; max-abs scales skip NaN
+ * and keep infinities.
  *
  *   A          device fp16 [M][K] (IEEE binary16 bits), 2-byte aligned; K <= 32768.
  *   M          rows (tokens, or pixels of an NHWC image); 0 is a no-op.

@@ -521,11 +521,13 @@ __global__ void __launch_bounds__(128) pack_weights_kernel(const PackWParams p) 
                 // the correctly rounded w / s; |y| = |w / s| 2^(n-1) <= 128, so a y
                 // within 8 ulps of 128 of a half-integer redoes the IEEE division and
                 // every code is the exact rule's
+                // (the conversion saturates and takes NaN to 0, as weight_code does)
                 const float w = __ldg(Wn + (int64_t)t * p.K + p.perm[G.perm_base + c]);
                 const float y = w * rh;
                 const float k = rintf(y);
+                const int32_t h = 1 << (nb - 1);
                 j = fabsf(fabsf(y - k) - 0.5f) <= 8.0f * 0x1p-16f ? weight_code(w, s, half)
-                                                                 : (int32_t)fminf(fmaxf(k, -half), half - 1.0f);
+                                                                 : min(max(__float2int_rz(k), -h), h - 1);
             }
             const uint32_t word = pack_block_warp((uint32_t)j & mask, nb);
             if (lane < nb) dst[kb * nb + lane] = word;

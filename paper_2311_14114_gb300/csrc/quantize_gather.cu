@@ -25,7 +25,9 @@
 // otherwise; the clip is taken before rounding (its bounds are integers, so
 // clip and rint commute, and fmaxf maps NaN to 0 as the clip does); rint is
 // the addition of 1.5 * 2^23, after which the low byte of the sum's bits is
-// the integer.
+// the integer.  Under a calibrated scale the top clip is taken on the input
+// instead (a above s becomes s, whose quotient is exactly 1): +inf then
+// gets the top code, where the residual step would have made it NaN.
 //
 // Scale modes: given scales (per tensor after the separate absmax pass, or
 // calibrated), or per (row, group) maxima found from the staged rows.
@@ -181,10 +183,10 @@ __device__ __forceinline__ void codes_chunk8(uint32_t rows_ba, uint32_t codes_a,
                 for (int j = 0; j < 8; ++j) a[j] = lds_half(row + off[j]);
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
-                    const float q0 = __fmul_rn(a[j], kk.r);
-                    const float q = __fmaf_rn(__fmaf_rn(-q0, kk.s, a[j]), kk.r, q0);
-                    float u = fmaxf(__fmul_rn(q, lv), 0.0f);
-                    if (MODE == 0) u = fminf(u, lv);
+                    const float x = MODE == 0 ? fmin_keep_nan(a[j], kk.s) : a[j];
+                    const float q0 = __fmul_rn(x, kk.r);
+                    const float q = __fmaf_rn(__fmaf_rn(-q0, kk.s, x), kk.r, q0);
+                    const float u = fmaxf(__fmul_rn(q, lv), 0.0f);
                     sts_u8(crow + 32u * j, __float_as_uint(__fadd_rn(u, 12582912.0f)));
                 }
             } else if (kk.mode == 1) {
@@ -193,10 +195,10 @@ __device__ __forceinline__ void codes_chunk8(uint32_t rows_ba, uint32_t codes_a,
                 for (int j = 0; j < 8; ++j) a[j] = lds_half(row + off[j]);
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
-                    const float q0 = __fmul_rn(a[j], kk.r);
-                    const float q = __fmaf_rn(__fmaf_rn(-q0, kk.s, a[j]), kk.r, q0);
-                    float u = fmaxf(__fmul_rn(q, lv), 0.0f);
-                    if (MODE == 0) u = fminf(u, lv);
+                    const float x = MODE == 0 ? fmin_keep_nan(a[j], kk.s) : a[j];
+                    const float q0 = __fmul_rn(x, kk.r);
+                    const float q = __fmaf_rn(__fmaf_rn(-q0, kk.s, x), kk.r, q0);
+                    const float u = fmaxf(__fmul_rn(q, lv), 0.0f);
                     const uint32_t code = __float_as_uint(__fadd_rn(u, 12582912.0f));
                     if (j < nc) sts_u8(crow + 32u * j, code);
                 }

@@ -24,13 +24,21 @@ __device__ __forceinline__ uint32_t act_code(float a, float s, float levels) {
 }
 
 // Weight (Sec. 3 step 3, Eq. (1)): nearest level j / 2^(n-1) to w / s,
-// j in [-2^(n-1), 2^(n-1) - 1]; `half` = 2^(n-1).
+// j in [-2^(n-1), 2^(n-1) - 1]; `half` = 2^(n-1).  The conversion rounds half
+// to even and saturates, so +-inf reach the end levels through the clip and a
+// NaN quotient gives code 0.
 __device__ __forceinline__ int32_t weight_code(float w, float s, float half) {
     if (!(s > 0.0f)) return 0;
-    float t = __fmul_rn(__fdiv_rn(w, s), half);
-    float r = rintf(t);
-    r = fminf(fmaxf(r, -half), half - 1.0f);
-    return (int32_t)r;
+    const float t = __fmul_rn(__fdiv_rn(w, s), half);
+    const int32_t h = (int32_t)half;
+    return min(max(__float2int_rn(t), -h), h - 1);
+}
+
+// min(x, s) that keeps a NaN x (the plain fminf would return s).
+__device__ __forceinline__ float fmin_keep_nan(float x, float s) {
+    float r;
+    asm("min.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(x), "f"(s));
+    return r;
 }
 
 // The code of Sec. 3 step 2, t = (a / s) * (2^n - 1) rounded half to even and
@@ -39,17 +47,21 @@ __device__ __forceinline__ int32_t weight_code(float w, float s, float half) {
 // products fused; for |a| <= 65504 and s in [2^-60, 2^60] this is the
 // correctly rounded quotient (checked exhaustively over every fp16 a); other
 // scales take the IEEE division.  Rounding to an unsigned integer saturates
-// negative values (and NaN) at 0, which is the clip at 0.
+// negative values (and NaN) at 0, which is the clip at 0.  On the Markstein
+// path the top clip is taken on the input instead: a above s becomes s, whose
+// quotient is exactly 1, so every a >= s (+inf too, which the residual would
+// turn into NaN) gets the top code and no quotient exceeds 1; a NaN input
+// stays NaN and gets code 0.
 template <bool FAST>
 __device__ __forceinline__ uint32_t act_code_q(float a, float s, float r, float levels, uint32_t top) {
-    float q;
     if constexpr (FAST) {
-        const float q0 = a * r;
-        q = fmaf(fmaf(-q0, s, a), r, q0);
+        const float x = fmin_keep_nan(a, s);
+        const float q0 = x * r;
+        const float q = fmaf(fmaf(-q0, s, x), r, q0);
+        return __float2uint_rn(__fmul_rn(q, levels));
     } else {
-        q = __fdiv_rn(a, s);
+        return min(__float2uint_rn(__fmul_rn(__fdiv_rn(a, s), levels)), top);
     }
-    return min(__float2uint_rn(__fmul_rn(q, levels)), top);
 }
 
 // Quantizer constants of one (row or tensor, group): scale, its reciprocal,

@@ -9,7 +9,9 @@
  * every positive finite fp16 scale and a set of seeded random fp32 scales
  * spread over [2^-60, 2^60], and prints the number of mismatches (values
  * compared with ==, so the sign of a zero quotient is not counted: both zeros
- * quantize to code 0).
+ * quantize to code 0).  Under a calibrated scale the kernels clip an input
+ * above s to s before the quotient, so for every scale it also checks that
+ * the corrected quotient of s itself is exactly 1.
  * Build: gcc -O2 -ffp-contract=off -fno-fast-math markstein_check.c -lm
  */
 #include <math.h>
@@ -48,6 +50,10 @@ static long check_scale(float s, const float *a, int na) {
         /* equal values (a zero quotient may differ in sign only: -0 / s is -0,
            the corrected quotient +0; both give code 0) */
         if (!(q == ref)) ++bad;
+    }
+    {   /* the clipped input a = s */
+        const float q0 = s * r;
+        if (!(fmaf(fmaf(-q0, s, s), r, q0) == 1.0f)) ++bad;
     }
     return bad;
 }

@@ -3,7 +3,9 @@ RN(1 / s) instead of a division (Sec. 3 step 2 fixes the quotient; reading c2:
 the correctly rounded fp32 quotient).  This CPU test checks, exhaustively over
 every finite fp16 input and every positive finite fp16 scale plus seeded random
 fp32 scales in [2^-60, 2^60], that the two are the same fp32 value, so the
-codes the kernels decide are the ones the oracle's IEEE division decides."""
+codes the kernels decide are the ones the oracle's IEEE division decides; and
+that the corrected quotient of s by itself is exactly 1 (a calibrated scale
+clips larger inputs, +inf among them, to s before the quotient)."""
 import os
 import subprocess
 import tempfile
