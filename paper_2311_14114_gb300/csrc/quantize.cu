@@ -511,6 +511,9 @@ __global__ void __launch_bounds__(128) pack_weights_kernel(const PackWParams p) 
         const uint32_t mask = (1u << nb) - 1u;
         const float s = s_sh[g];
         const float rh = s > 0.0f ? __frcp_rn(s) * half : 0.0f;   // half is a power of two: exact
+        // the estimate below needs a finite RN(1/s) * 2^(n-1): scales under about
+        // 2^-121 overflow it, and their codes all take the IEEE division
+        const bool est = rh <= 3.402823466e38f;
         uint32_t* dst = reinterpret_cast<uint32_t*>(dst_row + G.w_off);
         for (int kb = warp; kb < G.pw / 32; kb += nwarps) {
             const int pos = kb * 32 + lane;
@@ -518,16 +521,16 @@ __global__ void __launch_bounds__(128) pack_weights_kernel(const PackWParams p) 
             int32_t j = 0;
             if (t < p.taps && c < G.count && s > 0.0f) {
                 // Eq. (1) from the quotient estimate w * RN(1/s), within a few ulps of
-                // the correctly rounded w / s; |y| = |w / s| 2^(n-1) <= 128, so a y
-                // within 8 ulps of 128 of a half-integer redoes the IEEE division and
-                // every code is the exact rule's
-                // (the conversion saturates and takes NaN to 0, as weight_code does)
+                // the correctly rounded w / s (under 3 ulps of 128 even where 1/s is
+                // subnormal); |y| = |w / s| 2^(n-1) <= 128, so a y within 8 ulps of 128
+                // of a half-integer redoes the IEEE division and every code is the exact
+                // rule's (the conversion saturates and takes NaN to 0, as weight_code does)
                 const float w = __ldg(Wn + (int64_t)t * p.K + p.perm[G.perm_base + c]);
                 const float y = w * rh;
                 const float k = rintf(y);
                 const int32_t h = 1 << (nb - 1);
-                j = fabsf(fabsf(y - k) - 0.5f) <= 8.0f * 0x1p-16f ? weight_code(w, s, half)
-                                                                 : min(max(__float2int_rz(k), -h), h - 1);
+                j = (!est || fabsf(fabsf(y - k) - 0.5f) <= 8.0f * 0x1p-16f) ? weight_code(w, s, half)
+                                                                            : min(max(__float2int_rz(k), -h), h - 1);
             }
             const uint32_t word = pack_block_warp((uint32_t)j & mask, nb);
             if (lane < nb) dst[kb * nb + lane] = word;

@@ -138,6 +138,35 @@ def test_pack_weights_non_finite(sq, taps, mode):
     assert np.array_equal(Wp.cpu().numpy(), oracle.pack_weight_rows(J, count, bits, pad))
 
 
+@pytest.mark.parametrize("mode", ["row", "tensor"])
+def test_pack_weights_extreme_scales(sq, mode):
+    """Row maxima from the smallest fp32 subnormal to 3e38: where RN(1/s) * 2^(n-1)
+    overflows (scales under about 2^-121) every code takes the IEEE division;
+    where 1/s is subnormal (scales over 2^126) the estimate stays inside the
+    tie window.  Per tensor, all rows share the largest maximum of the tiny ones."""
+    rng = np.random.default_rng(77 + (mode == "row"))
+    K = 200
+    perm, count, _ = wl.assignment(rng, K, 0.3, 0)
+    bases = np.array([1.4e-45, 1e-42, 1e-40, 3e-39, 1.2e-38, 1e-37, 3.7e-37, 1e-36, 1e-30, 1.0, 1e30, 8.6e37,
+                      1e38, 3e38], np.float64)
+    if mode == "tensor":
+        bases = bases[bases < 1e-35]
+    N = len(bases) * 4
+    W = (rng.uniform(-1.0, 1.0, (N, K)) * np.repeat(bases, 4)[:, None]).astype(np.float32)
+    # exact ties at half-levels and the maxima themselves
+    W[::4, :8] = (np.repeat(bases, 1)[:, None] * np.array([1, -1, 0.5, -0.5, 0.25, 0.75, 1 / 3, -1 / 7])).astype(
+        np.float32)
+    bits = [3, 8]
+    lay = sq.Layout(perm, count, bits)
+    Wp, s_w = sq.pack_weights(lay, _dev(W), scale_mode=mode)
+    assert sq.sync_status() == 0
+    W3 = W[:, None, :]
+    s_ref = oracle.weight_scales(W3, perm, count, per_row=(mode == "row"))
+    J = oracle.weight_codes(W3, perm, count, bits, s_ref)
+    assert np.array_equal(s_w.cpu().numpy(), s_ref)
+    assert np.array_equal(Wp.cpu().numpy(), oracle.pack_weight_rows(J, count, bits, 128))
+
+
 def test_next_layer_codes_of_overflowed_outputs(sq):
     """Outputs beyond the fp16 range round to +-inf; the epilogue's next-layer
     codes of them are the top code and 0 under the calibrated scales, as the
