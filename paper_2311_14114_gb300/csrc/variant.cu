@@ -46,7 +46,8 @@ __device__ __forceinline__ int run_of(int j, int sub_k) { return sub_k > 0 ? j /
 
 // Max |x| per (group, run) of each row (per_row) or of all rows; s must be
 // zero before a per-tensor launch (maxima are merged with atomicMax on the
-// bit patterns, which order non-negative floats).
+// bit patterns, which order non-negative floats and infinity; NaN, whose
+// patterns lie above infinity's, is skipped as the other max-abs passes skip it).
 template <typename T>
 __global__ void __launch_bounds__(kAbsmaxThreads) variant_absmax_kernel(const T* X, int64_t rows, const int32_t* perm,
                                                                         VGeo v, int per_row, float* s) {
@@ -59,7 +60,7 @@ __global__ void __launch_bounds__(kAbsmaxThreads) variant_absmax_kernel(const T*
             const int g = p < v.count0 ? 0 : 1;
             const int j = g == 0 ? p : p - v.count0;
             const float a = fabsf(load_x<T>(X, m * v.K + perm[p]));
-            atomicMax(&smax[g * v.nb + run_of(j, v.sub_k)], __float_as_uint(a));
+            if (a == a) atomicMax(&smax[g * v.nb + run_of(j, v.sub_k)], __float_as_uint(a));
         }
         if (per_row) {
             __syncthreads();

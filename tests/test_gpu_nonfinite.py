@@ -167,6 +167,35 @@ def test_pack_weights_extreme_scales(sq, mode):
     assert np.array_equal(Wp.cpu().numpy(), oracle.pack_weight_rows(J, count, bits, 128))
 
 
+@pytest.mark.parametrize("kind,sub_k,lo", [((1, 1), 0, 3), ((1, 0), 128, 3), ((0, 1), 256, 3), ((2, 1), 128, 1)])
+@pytest.mark.parametrize("act_mode", ["tensor", "row"])
+def test_variant_layouts_non_finite(sq, kind, sub_k, lo, act_mode):
+    """Signed (Eq. (1)) and +-1 groups and scale runs: the run maxima skip NaN
+    and keep infinities; signed codes of +-inf clip to the end levels under a
+    finite scale, NaN codes to 0 (+-1 groups take -1 for NaN, as x >= 0 fails)."""
+    d = wl.random_linear(1700 + 10 * kind[0] + kind[1] + sub_k, M=40, K=700, N=64, bits_lo=lo, bits_hi=6,
+                         frac_hi=0.4)
+    rng = np.random.default_rng(sub_k + kind[0])
+    perm, count = d["perm"], d["count"]
+    A = d["A"].copy()
+    A = _plant(A, _cells(rng, A.shape[0], perm[:count[0]], 12), [NAN, INF, -INF])
+    A[5, perm[count[0] + 3]] = NAN             # a finite-scale NaN in group 1
+    W = d["W"].copy()
+    W[2, perm[4]] = np.nan
+    W[9, perm[count[0] + 1]] = np.nan
+    W[11, perm[count[0] + 7]] = -np.inf         # row 11, group 1 (a run of it): scale inf
+    lay = sq.Layout(perm, count, d["bits"], act_kind=kind, sub_k=sub_k)
+    Wp, s_w = sq.pack_weights(lay, _dev(W))
+    Ap, s_a = sq.quantize_act(lay, _dev(A), scale_mode=act_mode)
+    assert sq.sync_status() == 0
+    r = oracle.linear_variant(A, W, perm, count, d["bits"], d["bits"], kind=kind, sub_k=sub_k, act_mode=act_mode)
+    s_a_ref = (r["s_a"] if sub_k else r["s_a"][..., 0]).reshape(tuple(s_a.shape))
+    assert np.array_equal(s_a.cpu().numpy(), s_a_ref), "activation scales"
+    assert np.array_equal(s_w.cpu().numpy(), r["s_w"].reshape(tuple(s_w.shape))), "weight scales"
+    assert np.array_equal(Ap.cpu().numpy(), r["Ap"]), "packed activations"
+    assert np.array_equal(Wp.cpu().numpy(), r["Wp"]), "packed weights"
+
+
 def test_next_layer_codes_of_overflowed_outputs(sq):
     """Outputs beyond the fp16 range round to +-inf; the epilogue's next-layer
     codes of them are the top code and 0 under the calibrated scales, as the
