@@ -344,7 +344,7 @@ SONIQ_API soniq_status soniq_quantize_act_oneshot(const soniq_layout *layout, co
  *              then be NULL).  Needs the staged path: scratch of at least
  *              soniq_mp_gemm_scratch_bytes(..., flags | SONIQ_FLAG_FORCE_STAGED),
  *              else SONIQ_ERR_UNSUPPORTED.
- *   Limits (SONIQ_ERR_UNSUPPORTED otherwise): K <= 65536.  The tensor-core
+ *   Limits (SONIQ_ERR_UNSUPPORTED otherwise): K <= 65536, M < 2^31.  The tensor-core
  *   kernel accumulates integer codes in fp32, exact while every partial sum
  *   stays within 2^24; a group whose worst-case sum over its K range could
  *   exceed that is accumulated in bounded segments that are drained to int32,
@@ -382,7 +382,8 @@ SONIQ_API int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout *layout, int64_
  * blocks; Sec. 6 evaluates conv layers).  K = R*S*C_in in the weight order
  * (group, tap, channel); input positions outside the image contribute 0.
  *
- *   cd         geometry; P, Q > 0.
+ *   cd         geometry; P, Q > 0 (SONIQ_ERR_INVALID_ARG otherwise);
+ *              batch * P * Q < 2^31 and R * S < 2^31 (SONIQ_ERR_UNSUPPORTED otherwise).
  *   Xp, s_a    soniq_quantize_act of the NHWC input viewed as [batch*H*W][C_in],
  *              with a per-tensor or calibrated scale (a per-pixel scale would
  *              break the shared scale of one dot product, C2).

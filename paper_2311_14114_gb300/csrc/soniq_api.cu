@@ -231,10 +231,28 @@ soniq_status check_next(const soniq_next_layer* next, int64_t N, int32_t out_dty
     return SONIQ_OK;
 }
 
-int64_t conv_rows(const soniq_conv_desc* cd) {
-    const int64_t P = (cd->H + 2 * cd->pad_h - cd->R) / cd->stride_h + 1;
-    const int64_t Q = (cd->W + 2 * cd->pad_w - cd->S) / cd->stride_w + 1;
-    return (int64_t)cd->batch * P * Q;
+// Rows of a GEMM (output pixels of a convolution) the kernels address: their
+// tile and TMA row coordinates are 32-bit.
+constexpr int64_t kMaxRows = 2147483647;
+
+// Taps, output size and output rows of a convolution, in 64-bit arithmetic:
+// SONIQ_ERR_INVALID_ARG for a malformed geometry (the filter larger than the
+// padded image included), SONIQ_ERR_UNSUPPORTED beyond the addressable sizes.
+soniq_status conv_geometry(const soniq_conv_desc* cd, int32_t* taps, int32_t* P, int32_t* Q, int64_t* rows) {
+    if (cd == nullptr || cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->pad_h < 0 ||
+        cd->pad_w < 0 || cd->batch < 0 || cd->H < 1 || cd->W < 1 || cd->C_out < 0)
+        return SONIQ_ERR_INVALID_ARG;
+    const int64_t hp = (int64_t)cd->H + 2 * (int64_t)cd->pad_h, wp = (int64_t)cd->W + 2 * (int64_t)cd->pad_w;
+    if (hp < cd->R || wp < cd->S) return SONIQ_ERR_INVALID_ARG;
+    const int64_t t = (int64_t)cd->R * cd->S;
+    const int64_t p = (hp - cd->R) / cd->stride_h + 1, q = (wp - cd->S) / cd->stride_w + 1;
+    if (t > kMaxRows || p > kMaxRows || q > kMaxRows || p * q > kMaxRows || (int64_t)cd->batch * (p * q) > kMaxRows)
+        return SONIQ_ERR_UNSUPPORTED;
+    *taps = (int32_t)t;
+    *P = (int32_t)p;
+    *Q = (int32_t)q;
+    *rows = (int64_t)cd->batch * p * q;
+    return SONIQ_OK;
 }
 
 soniq_status check_scale_mode_act(int32_t mode) {
@@ -398,6 +416,7 @@ soniq_status soniq_mp_gemm(const soniq_layout* L, const uint8_t* Ap, const float
     soniq_status st = make_geom(L, 1, &geo);
     if (st != SONIQ_OK) return st;
     if (M < 0 || N < 0) return SONIQ_ERR_INVALID_ARG;
+    if (M > kMaxRows) return SONIQ_ERR_UNSUPPORTED;
     if ((st = check_scale_mode_act(scale_mode)) != SONIQ_OK) return st;
     if (out_dtype != SONIQ_OUT_F16 && out_dtype != SONIQ_OUT_BF16) return SONIQ_ERR_INVALID_ARG;
     if ((flags & SONIQ_FLAG_FORCE_GEMV) && (flags & SONIQ_FLAG_FORCE_MMA)) return SONIQ_ERR_INVALID_ARG;
@@ -456,21 +475,15 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
                              void* Y, int32_t out_dtype, int32_t* acc_dbg, uint32_t flags,
                              void* scratch, size_t scratch_bytes, const soniq_next_layer* next,
                              soniq_stream_t stream) {
-    if (cd == nullptr) return SONIQ_ERR_INVALID_ARG;
-    if (cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->pad_h < 0 || cd->pad_w < 0 ||
-        cd->batch < 0 || cd->H < 1 || cd->W < 1 || cd->C_out < 0)
-        return SONIQ_ERR_INVALID_ARG;
-    LayoutGeom geo;
-    soniq_status st = make_geom(L, cd->R * cd->S, &geo);
+    int32_t taps = 0, P = 0, Q = 0;
+    int64_t M = 0;
+    soniq_status st = conv_geometry(cd, &taps, &P, &Q, &M);
     if (st != SONIQ_OK) return st;
+    LayoutGeom geo;
+    if ((st = make_geom(L, taps, &geo)) != SONIQ_OK) return st;
     if (geo.variant) return SONIQ_ERR_UNSUPPORTED;   // the layout variants are for linear layers
     if (scale_mode != SONIQ_SCALE_PER_TENSOR && scale_mode != SONIQ_SCALE_CALIBRATED) return SONIQ_ERR_INVALID_ARG;
     if (out_dtype != SONIQ_OUT_F16 && out_dtype != SONIQ_OUT_BF16) return SONIQ_ERR_INVALID_ARG;
-    const int32_t P = (cd->H + 2 * cd->pad_h - cd->R) / cd->stride_h + 1;
-    const int32_t Q = (cd->W + 2 * cd->pad_w - cd->S) / cd->stride_w + 1;
-    if (cd->H + 2 * cd->pad_h < cd->R || cd->W + 2 * cd->pad_w < cd->S || P < 1 || Q < 1)
-        return SONIQ_ERR_INVALID_ARG;
-    const int64_t M = (int64_t)cd->batch * P * Q;
     LayoutGeom geo_next;
     if (next != nullptr && (st = check_next(next, cd->C_out, out_dtype, &geo_next)) != SONIQ_OK) return st;
     if (next != nullptr) flags |= SONIQ_FLAG_FORCE_STAGED;
@@ -520,7 +533,7 @@ soniq_status soniq_mp_conv2d(const soniq_layout* L, const soniq_conv_desc* cd, c
 
 int32_t soniq_mp_gemm_path(const soniq_layout* L, int64_t M, int32_t N, uint32_t flags, size_t scratch_bytes) {
     LayoutGeom geo;
-    if (make_geom(L, 1, &geo) != SONIQ_OK || M < 1 || N < 1) return -1;
+    if (make_geom(L, 1, &geo) != SONIQ_OK || M < 1 || M > kMaxRows || N < 1) return -1;
     if ((flags & SONIQ_FLAG_FORCE_GEMV) && (flags & SONIQ_FLAG_FORCE_MMA)) return -1;
     const int p = gemm_path(geo, M, N, flags, scratch_bytes);
     return p < 0 ? -1 : p;
@@ -528,7 +541,7 @@ int32_t soniq_mp_gemm_path(const soniq_layout* L, int64_t M, int32_t N, uint32_t
 
 int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout* L, int64_t M, int32_t N, uint32_t flags) {
     LayoutGeom geo;
-    if (make_geom(L, 1, &geo) != SONIQ_OK || M < 0 || N < 0) return -1;
+    if (make_geom(L, 1, &geo) != SONIQ_OK || M < 0 || M > kMaxRows || N < 0) return -1;
     if (M == 0 || N == 0) return 0;
     if (geo.variant) return staged_scratch_bytes(geo, M, N);
     if (flags & SONIQ_FLAG_FORCE_FUSED) return 0;
@@ -546,12 +559,11 @@ int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout* L, int64_t M, int32_t N,
 
 int64_t soniq_mp_conv2d_scratch_bytes(const soniq_layout* L, const soniq_conv_desc* cd, uint32_t flags) {
     LayoutGeom geo;
-    if (cd == nullptr || cd->R < 1 || cd->S < 1 || cd->stride_h < 1 || cd->stride_w < 1 || cd->batch < 0 ||
-        cd->C_out < 0 || make_geom(L, cd->R * cd->S, &geo) != SONIQ_OK)
-        return -1;
-    if (cd->H + 2 * cd->pad_h < cd->R || cd->W + 2 * cd->pad_w < cd->S) return -1;
-    if (flags & SONIQ_FLAG_FORCE_FUSED || !staged_worthwhile(geo, conv_rows(cd), cd->C_out, flags)) return 0;
-    return staged_scratch_bytes(geo, conv_rows(cd), cd->C_out);
+    int32_t taps = 0, P = 0, Q = 0;
+    int64_t rows = 0;
+    if (conv_geometry(cd, &taps, &P, &Q, &rows) != SONIQ_OK || make_geom(L, taps, &geo) != SONIQ_OK) return -1;
+    if (flags & SONIQ_FLAG_FORCE_FUSED || !staged_worthwhile(geo, rows, cd->C_out, flags)) return 0;
+    return staged_scratch_bytes(geo, rows, cd->C_out);
 }
 
 soniq_status soniq_sync_status(soniq_stream_t stream) {

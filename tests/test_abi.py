@@ -116,6 +116,23 @@ def test_host_side_argument_errors_need_no_gpu(L):
     # K beyond the supported range
     big = _layout(soniq, K=70000, count=(70000, 0), bits=(2, 2), perm=ctypes.c_void_p(16))
     assert L.soniq_mp_gemm(ctypes.byref(big), fake, fake, 0, 4, fake, fake, 8, fake, 0, None, 0, None, 0, None, None) == 2
+    # M beyond the 32-bit row coordinates
+    assert L.soniq_mp_gemm(ctypes.byref(lay), fake, fake, 0, 2 ** 31, fake, fake, 8, fake, 0, None, 0, None, 0, None,
+                           None) == 2
+    assert L.soniq_mp_gemm_path(ctypes.byref(lay), 2 ** 31, 8, 0, 0) == -1
+    assert L.soniq_mp_gemm_scratch_bytes(ctypes.byref(lay), 2 ** 31, 8, 0) == -1
+    # conv geometry in 64-bit arithmetic: a pad that overflows 32 bits, and output rows past 2^31
+    cd = soniq.conv_desc(1, 8, 8, 16, pad=(2 ** 30, 1))
+    assert L.soniq_mp_conv2d(ctypes.byref(lay), ctypes.byref(cd), fake, fake, 0, fake, fake, fake, 0,
+                             None, 0, None, 0, None, None) == 2
+    cd = soniq.conv_desc(2 ** 20, 2 ** 10, 2 ** 10, 16)
+    assert L.soniq_mp_conv2d(ctypes.byref(lay), ctypes.byref(cd), fake, fake, 0, fake, fake, fake, 0,
+                             None, 0, None, 0, None, None) == 2
+    assert L.soniq_mp_conv2d_scratch_bytes(ctypes.byref(lay), ctypes.byref(cd), 0) == -1
+    # a negative pad is malformed
+    cd = soniq.conv_desc(1, 8, 8, 16, pad=(-1, 1))
+    assert L.soniq_mp_conv2d(ctypes.byref(lay), ctypes.byref(cd), fake, fake, 0, fake, fake, fake, 0,
+                             None, 0, None, 0, None, None) == 1
 
 
 def test_next_layer_descriptor_checks(L):
