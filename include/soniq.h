@@ -229,7 +229,7 @@ SONIQ_API int64_t soniq_launch_count(void);
  *   W          device fp32 [N][taps][K] (taps = 1: a linear layer [N][K];
  *              a convolution OHWI [C_out][R*S][C_in]), 4-byte aligned.
  *   N          output rows (>= 0; 0 is a no-op).
- *   taps       filter taps R*S (>= 1).
+ *   taps       filter taps R*S, 1 to 4096.
  *   scale_mode SONIQ_SCALE_PER_ROW (one scale per (n, group) over all taps)
  *              or SONIQ_SCALE_PER_TENSOR (one per group; written to every row).
  *   Wp         device out [N][soniq_packed_row_bytes(layout, 1, taps)], 16-byte aligned.
@@ -382,8 +382,8 @@ SONIQ_API int64_t soniq_mp_gemm_scratch_bytes(const soniq_layout *layout, int64_
  * blocks; Sec. 6 evaluates conv layers).  K = R*S*C_in in the weight order
  * (group, tap, channel); input positions outside the image contribute 0.
  *
- *   cd         geometry; P, Q > 0 (SONIQ_ERR_INVALID_ARG otherwise);
- *              batch * P * Q < 2^31 and R * S < 2^31 (SONIQ_ERR_UNSUPPORTED otherwise).
+ *   cd         geometry; P, Q > 0 and R * S <= 4096 (SONIQ_ERR_INVALID_ARG otherwise);
+ *              batch * P * Q < 2^31 (SONIQ_ERR_UNSUPPORTED otherwise).
  *   Xp, s_a    soniq_quantize_act of the NHWC input viewed as [batch*H*W][C_in],
  *              with a per-tensor or calibrated scale (a per-pixel scale would
  *              break the shared scale of one dot product, C2).
