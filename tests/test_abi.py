@@ -199,3 +199,15 @@ def test_layout_variant_checks(L):
     assert L.soniq_mp_gemm_path(ctypes.byref(runs), 16, 64, 0, need) == 2
     assert L.soniq_mp_gemm_path(ctypes.byref(runs), 16, 64, 0, 0) == -1
     assert L.soniq_mp_gemm_path(ctypes.byref(runs), 16, 64, 16, need) == -1
+
+
+def test_binding_refuses_to_run_without_the_library(monkeypatch):
+    """No CPU fallback: without libsoniq.so every call of the binding raises."""
+    from paper_2311_14114_gb300 import soniq
+    monkeypatch.setattr(soniq, "_lib", None)
+    monkeypatch.setattr(soniq, "LIB_PATH", os.path.join(ROOT, "no_such_dir", "libsoniq.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        soniq.lib()
+    # the first call a user makes (a layout, validated by the library) raises too
+    with pytest.raises(RuntimeError, match="not built"):
+        soniq.Layout(np.arange(64, dtype=np.int32), [48, 16], [2, 8])
