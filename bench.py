@@ -204,6 +204,24 @@ def _time_graph(g, steps, flush, stream, warm=3):
     return [a.elapsed_time(b) for a, b in ev]
 
 
+def max_over_ranks(x, world, device):
+    """The largest x over the ranks of the process group (x itself for one
+    rank): the job's time is its slowest replica's."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t[0])
+
+
+def job_tops(ops_per_rank, ms_per_step, world):
+    """Whole-job throughput: the operations of every replica over the slowest
+    replica's time per step."""
+    return world * ops_per_rank / (ms_per_step * 1e-3) / 1e12
+
+
 def _time_fn(fn, steps, flush, stream):
     """Mean device time (ms) of a library call replayed as a CUDA graph (the
     mean, not the median: event timestamps here tick in steps of about 2 us,
@@ -278,14 +296,10 @@ def run_gpu(args):
     # the two kernels alone, same flush and replay discipline
     gemm_ms = _time_graph(g_gemm, args.steps, flush, stream)
     quant_ms = _time_graph(g_quant, args.steps, flush, stream)
-    total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t[0])
+    total_ms = max_over_ranks(sum(step_ms), world, "cuda")
     ms_per_step = total_ms / args.steps
     ops = spec.ops
-    value = world * ops / (ms_per_step * 1e-3) / 1e12
+    value = job_tops(ops, ms_per_step, world)
 
     # ---- end to end through host buffers ----
     # Every step uploads its own input from pinned host memory, runs the two
@@ -338,12 +352,8 @@ def run_gpu(args):
     torch.cuda.synchronize()
     if sq.sync_status() != 0:
         raise RuntimeError("device error during the end-to-end steps")
-    e2e_ms = e_start.elapsed_time(e_end) / args.steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t[0])
-    e2e_value = world * ops / (e2e_ms * 1e-3) / 1e12
+    e2e_ms = max_over_ranks(e_start.elapsed_time(e_end) / args.steps, world, "cuda")
+    e2e_value = job_tops(ops, e2e_ms, world)
 
     # ---- roofline of the dominant kernel (the tensor-core GEMM) ----
     gemm_avg = statistics.mean(gemm_ms)
