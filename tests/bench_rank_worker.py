@@ -15,6 +15,8 @@ dist.init_process_group("gloo")
 ms = 10.0 + 5.0 * rank                       # the higher ranks are the slower replicas
 slowest = bench.max_over_ranks(ms, world, "cpu")
 value = bench.job_tops(2.0e12, slowest, world)
-dist.barrier()
-print(json.dumps({"rank": rank, "world": world, "slowest_ms": slowest, "tops": value}), flush=True)
+results = [None] * world
+dist.all_gather_object(results, {"rank": rank, "slowest_ms": slowest, "tops": value})
+if rank == 0:    # one line: the ranks share stdout
+    print(json.dumps({"world": world, "ranks": results}), flush=True)
 dist.destroy_process_group()
